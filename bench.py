@@ -1,0 +1,382 @@
+#!/usr/bin/env python
+"""Benchmark of the MeqMuon optimizer step (all 2D hidden weights of a model).
+
+Metric: milliseconds per optimizer step for the whole model (lower is
+better), with NS TFLOP/s and the bandwidth kernels' GB/s as fractions of the
+measured GB300 peaks.
+
+Default workload: Llama-130M hidden weights (84 matrices, 84.9M elements),
+seeded synthetic gradients (see paper_2609_35701_gb300/workloads.py); the
+state (params + grads + momentum = 1.02 GB) is larger than L2, so no flush
+is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the fp64 CPU oracle on host cores
+
+With N > 1 (torchrun), the matrices are split across ranks (flop-balanced,
+no data-path collective); the time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+LR, MU, WD, EPS = 0.02, 0.95, 0.1, 1e-7
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+BW_BYTES_PER_ELEM = 24  # read G, B; write B; write X_0 (2 B); read U (2 B); read + write W
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def ns_flops(s, l, K):
+    """Algorithmic NS flops of one matrix (Eq. (5), K iterations), counting
+    the symmetric halves of A = X X^T and A^2 once, and the dense count."""
+    sym = K * (s * (s + 1) * l + s * s * (s + 1) + 2 * s * s * l)
+    dense = K * (4 * s * s * l + 2 * s * s * s)
+    return sym, dense
+
+
+def partition(shapes, world, K=5):
+    """Greedy flop-balanced split of matrix indices over ranks."""
+    w = [(ns_flops(min(r, c), max(r, c), K)[0], i) for i, (r, c) in enumerate(shapes)]
+    w.sort(reverse=True)
+    load = [0] * world
+    parts = [[] for _ in range(world)]
+    for f, i in w:
+        k = min(range(world), key=lambda j: load[j])
+        parts[k].append(i)
+        load[k] += f
+    return [sorted(p) for p in parts]
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits", "-lms", "50",
+                 "-i", str(self.gpu_id)], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.12)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for r in rows for k in range(4) if r[5 + k].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def oracle_sample(wl, seed_step=0, max_per_class=1):
+    """Times the fp64 oracle on one matrix of every (rows, cols) class of the
+    workload and extrapolates to the whole model step (ms)."""
+    import numpy as np
+    import torch
+
+    from oracle import meqmuon as O
+    from paper_2609_35701_gb300 import workloads as W
+
+    classes = {}
+    for i, (_, r, c) in enumerate(wl.shapes):
+        classes.setdefault((r, c), []).append(i)
+    total_ms = 0.0
+    sampled = []
+    for (r, c), idx in classes.items():
+        i = idx[0]
+        G = W.gradient(wl, i, seed_step).double().numpy()
+        W0 = np.zeros((r, c))
+        Bp = np.zeros((r, c))
+        t0 = time.perf_counter()
+        O.hidden_step(W0, G, Bp, LR, MU, WD, eps=EPS)
+        dt = (time.perf_counter() - t0) * 1e3
+        total_ms += dt * len(idx)
+        sampled.append(f"{r}x{c}")
+    return total_ms, sampled
+
+
+def cpu_cores():
+    try:
+        n = len(os.sched_getaffinity(0))
+    except Exception:
+        n = os.cpu_count() or 1
+    for v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(v, "").isdigit():
+            n = min(n, int(os.environ[v]))
+    return n
+
+
+def run_reference(args):
+    """--impl reference: the fp64 CPU oracle, as it stands, on the host cores."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2609_35701_gb300 import workloads as W
+
+    wl = W.get_workload(args.workload)
+    for w in range(args.warmup):
+        oracle_sample(wl, w)
+    vals = []
+    sampled = None
+    for k in range(args.steps):
+        ms, sampled = oracle_sample(wl, k)
+        vals.append(ms)
+    v = statistics.median(vals)
+    cores = cpu_cores()
+    sample = (f"one matrix per shape class ({', '.join(sampled)}) per step, fp64 oracle, "
+              f"extrapolated by class counts to all {len(wl.shapes)} matrices")
+    line = {
+        "impl": "reference", "metric": "MeqMuon optimizer step time (all hidden 2D weights)", "value": v,
+        "unit": "ms/step", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": v, "higher_is_better": False, "scaling": "strong", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": args.workload, "matrices": len(wl.shapes), "elements": wl.numel},
+        "cpu_baseline": {"value": v, "unit": "ms/step", "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": v, "unit": "ms/step", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama130m")
+    ap.add_argument("--ns-fp16-mask", type=lambda x: int(x, 0), default=0xFFFFFFFF)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    if args.impl == "reference":
+        run_reference(args)
+        return
+
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    import __graft_entry__
+
+    __graft_entry__.build()
+    from paper_2609_35701_gb300 import meq
+    from paper_2609_35701_gb300 import workloads as W
+
+    wl = W.get_workload(args.workload)
+    mine = partition([(r, c) for _, r, c in wl.shapes], world)[rank]
+    shapes = [(wl.shapes[i][1], wl.shapes[i][2]) for i in mine]
+    dev = torch.device("cuda", local)
+
+    # Flat, 256-byte aligned device buffers with one view per matrix.
+    def flat_views(nums, device, pin=False):
+        offs, tot = [], 0
+        for n in nums:
+            offs.append(tot)
+            tot += (n + 63) // 64 * 64
+        if device == "cpu":
+            buf = torch.empty(tot, dtype=torch.float32, pin_memory=pin)
+        else:
+            buf = torch.empty(tot, dtype=torch.float32, device=device)
+        return buf, [buf[o:o + n] for o, n in zip(offs, nums)]
+
+    nums = [r * c for r, c in shapes]
+    pbuf, pviews = flat_views(nums, dev)
+    gbufs = []
+    for t in range(2):
+        gb, gv = flat_views(nums, dev)
+        for j, i in enumerate(mine):
+            gv[j].copy_(W.gradient(wl, i, t, device=dev).reshape(-1))
+        gbufs.append((gb, gv))
+    w0 = W.initial_weights(wl, device=dev)
+    for j, i in enumerate(mine):
+        pviews[j].copy_(w0[i].reshape(-1))
+    del w0
+    params = [v.view(r, c) for v, (r, c) in zip(pviews, shapes)]
+    grads = [[v.view(r, c) for v, (r, c) in zip(gv, shapes)] for _, gv in gbufs]
+
+    opt = meq.MeqMuon(shapes, ns_fp16_mask=args.ns_fp16_mask)
+    stream = torch.cuda.current_stream()
+    for k in range(args.warmup):
+        opt.step(params, grads[k % 2], LR, MU, WD, EPS)
+    opt.sync()
+
+    props = torch.cuda.get_device_properties(local)
+    gpu_id = getattr(props, "uuid", None)
+    gpu_id = f"GPU-{gpu_id}" if gpu_id is not None and not str(gpu_id).startswith("GPU-") else (gpu_id or local)
+    clocks = ClockSampler(gpu_id)
+    clocks.start()
+    time.sleep(0.15)
+    # ---------------- timed region: K steps, CUDA events on the launch stream
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for k in range(args.steps):
+        opt.step(params, grads[k % 2], LR, MU, WD, EPS)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    opt.sync()
+    ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    # ---------------- per-phase timing (events between phases, eager launches)
+    opt.set_profiling(True)
+    for k in range(args.steps):
+        opt.step(params, grads[k % 2], LR, MU, WD, EPS)
+    phases, nprof = opt.read_profile()
+    opt.set_profiling(False)
+    ph = {k: v / max(nprof, 1) for k, v in phases.items()}
+
+    K = 5
+    sym = sum(ns_flops(min(r, c), max(r, c), K)[0] for r, c in shapes)
+    dense = sum(ns_flops(min(r, c), max(r, c), K)[1] for r, c in shapes)
+    n_gemm_launches = opt.kernels_per_step - 5
+    peaks, peak_src = load_peaks()
+    ns_tflops = sym / (ph["ns_gemm"] * 1e-3) / 1e12
+    ns_dense_tflops = dense / (ph["ns_gemm"] * 1e-3) / 1e12
+    numel = sum(nums)
+    bw_ms = ph["momentum"] + ph["cast_x0"] + ph["stats"] + ph["apply"]
+    bw_gbs = BW_BYTES_PER_ELEM * numel / (bw_ms * 1e-3) / 1e9
+
+    # ---------------- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        hg = []
+        for gb, _ in gbufs:
+            h = torch.empty(gb.numel(), dtype=torch.float32, pin_memory=True)
+            h.copy_(gb)
+            hg.append(h)
+        hp = torch.empty(pbuf.numel(), dtype=torch.float32, pin_memory=True)
+        n_e2e = max(3, min(args.steps, 50))
+        torch.cuda.synchronize()
+        a0 = torch.cuda.Event(enable_timing=True)
+        a1 = torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for k in range(n_e2e):
+            gbufs[k % 2][0].copy_(hg[k % 2], non_blocking=True)
+            opt.step(params, grads[k % 2], LR, MU, WD, EPS)
+            hp.copy_(pbuf, non_blocking=True)
+        a1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = a0.elapsed_time(a1) / n_e2e
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        e2e = {"value": e2e_ms, "unit": "ms/step", "h2d_bytes_per_step": 4 * numel * (world if world > 1 else 1),
+               "d2h_bytes_per_step": 4 * numel * (world if world > 1 else 1), "steps": n_e2e}
+    opt.sync()
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        vals, sampled = [], None
+        t_start = time.perf_counter()
+        while True:
+            v, sampled = oracle_sample(wl, len(vals))
+            vals.append(v)
+            if time.perf_counter() - t_start > 10.0 or len(vals) >= 5:
+                break
+        cpu = {"value": statistics.median(vals), "unit": "ms/step", "cores": cpu_cores(), "kind": "oracle",
+               "sample": (f"fp64 oracle on one matrix per shape class ({', '.join(sampled)}), {len(vals)} repeats, "
+                          f"extrapolated by class counts to all {len(wl.shapes)} matrices")}
+
+    if rank == 0:
+        line = {
+            "metric": "MeqMuon optimizer step time (all hidden 2D weights)",
+            "value": ms, "unit": "ms/step", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": ms, "higher_is_better": False, "scaling": "strong", "vs_baseline": None,
+            "dtype": "fp16" if args.ns_fp16_mask == 0xFFFFFFFF else ("bf16" if args.ns_fp16_mask == 0 else "bf16/fp16"),
+            "data": "synthetic",
+            "config": {"workload": args.workload, "matrices": len(wl.shapes), "elements": wl.numel,
+                       "ns_steps": K, "ns_operands": "fp16" if args.ns_fp16_mask == 0xFFFFFFFF else hex(args.ns_fp16_mask),
+                       "accumulate": "fp32", "l2": "inputs larger than L2 (params+grads+momentum %.2f GB)" % (12 * wl.numel / 1e9),
+                       "parallelism": f"matrices split over {world} GPU(s)" if world > 1 else "single GPU"},
+            "roofline": {
+                "bound": "tensor", "kernel": "ns_gemm_kernel",
+                "achieved": ns_tflops, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": ns_tflops / peaks["bf16_tflops"], "peak_source": f"{peak_src} bf16 dense burst (fp16 rate = bf16 rate)",
+                "traffic": None,
+                "flops_per_launch": sym / max(n_gemm_launches, 1),
+                "avg_launch_ms": ph["ns_gemm"] / max(n_gemm_launches, 1),
+                "dense_equivalent_tflops": ns_dense_tflops,
+            },
+            "bandwidth_kernels": {
+                "bound": "hbm", "achieved": bw_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": bw_gbs / peaks["hbm_gbs"], "bytes_per_elem": BW_BYTES_PER_ELEM,
+                "phase_ms": {k: round(v, 4) for k, v in ph.items()},
+            },
+            "gpu_launches": opt.kernels_per_step * args.steps,
+            "kernels_per_step": opt.kernels_per_step,
+            "clocks": clk,
+            "e2e": e2e,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    opt.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,153 @@
+/*
+ * meq.h -- C ABI of the GB300 (sm_103a) MeqMuon optimizer step for 2D
+ * hidden-layer weights.
+ *
+ * The step follows the paper "MeqMuon: Matrix-Equilibrating Muon for LLM
+ * Pretraining", Algorithm 1 (hidden-weight branch), for every matrix W_i:
+ *
+ *   B_t   = mu B_{t-1} + G_t                                   Eq. (10)
+ *   U_t   = NS_K(B_t)  (X_0 = B/||B||_F;
+ *           X_{k+1} = a X_k + (b A_k + c A_k^2) X_k, A_k = X_k X_k^T)  Eq. (5)
+ *   r_i = ||U_{i,:}||/sqrt(n), c_j = ||U_{:,j}||/sqrt(m)       Eq. (7)
+ *   gamma = std/mean over entries > eps                        Eq. (8)
+ *   U~  = diag(r^-1) U  if gamma_r >= gamma_c, else U diag(c^-1)  Eqs. (9), (11)
+ *   W  <- (1 - lr*wd) W - rho*lr*U~                            Eq. (14)
+ *
+ * Everything runs in the library's own CUDA kernels, asynchronously on the
+ * caller's stream. Newton-Schulz runs on the tensor cores (tcgen05, TMA, TMEM)
+ * with 16-bit operands and fp32 accumulation; all other arithmetic is fp32
+ * (CV statistics in fp64).
+ *
+ * Conventions shared by every call:
+ *   - Matrices are fp32, row-major, contiguous, rows = output features and
+ *     columns = input features (the PyTorch layout the paper uses, Section 3.1).
+ *   - Device pointers must be 16-byte aligned.
+ *   - A meq_state is not thread-safe: one host thread drives it at a time.
+ *   - Validation errors are returned synchronously and nothing is enqueued.
+ *     Errors raised on the device (a bounded wait that expired) are reported
+ *     by the next meq_sync() as MEQ_ERR_TIMEOUT / MEQ_ERR_CUDA.
+ */
+#ifndef MEQ_H
+#define MEQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MEQ_OK = 0,
+  MEQ_ERR_INVALID_ARG = 1,   /* null pointer, bad size, misaligned pointer, shape list differs from init */
+  MEQ_ERR_OOM = 2,           /* device allocation failed or the workspace limit was exceeded */
+  MEQ_ERR_CUDA = 3,          /* a CUDA runtime call failed (see meq_last_error) */
+  MEQ_ERR_NONFINITE = 4,     /* reserved: non-finite gradient detected */
+  MEQ_ERR_TIMEOUT = 5,       /* a device-side bounded wait expired; the kernel returned early */
+  MEQ_ERR_UNSUPPORTED = 6    /* no sm_103a device, or a size beyond the library's limits */
+} meq_status;
+
+/* One matrix: rows = out features (m), cols = in features (n). */
+typedef struct {
+  int64_t rows;
+  int64_t cols;
+} meq_shape;
+
+/* Options fixed at init. meq_default_options() fills the paper's values. */
+typedef struct {
+  float rho;              /* RMS alignment coefficient, Eq. (14); 0.2 (Section 4) */
+  int ns_steps;           /* K of Eq. (5); 5 (Sections 2 and 4); 1..16 */
+  float ns_a, ns_b, ns_c; /* (3.4445, -4.7750, 2.0315), Section 2 */
+  int nesterov;           /* 0: NS input B_t (Eq. (10), Algorithm 1);
+                             1: NS input G_t + mu B_t (Nesterov look-ahead, Section 4) */
+  uint32_t ns_fp16_mask;  /* bit k set: NS iteration k uses fp16 operands, else bf16.
+                             Default 0xFFFFFFFF (all fp16; same tensor-core rate as bf16,
+                             three more mantissa bits). 0 = all bf16. */
+  float tie_atol;         /* Eq. (11) chooses row when gamma_r >= gamma_c - tie_atol; 1e-6 */
+  int use_graph;          /* 1: the step's kernels are replayed from a CUDA graph (default) */
+  int64_t workspace_limit_bytes; /* 0 = no limit; else init fails with MEQ_ERR_OOM above it */
+  float wait_timeout_ms;  /* bound of every device-side spin wait; default 4000 */
+} meq_options;
+
+typedef struct meq_state meq_state; /* opaque */
+
+void meq_default_options(meq_options* opt);
+
+/* Bytes the state would allocate for this shape list, computed on the host
+ * without touching the GPU. persistent = momentum buffers (4 bytes per
+ * element: the only state MeqMuon keeps, Section 4 "Memory overhead");
+ * workspace = transient NS / statistics buffers. Either output may be NULL. */
+meq_status meq_state_bytes(const meq_shape* shapes, int n, const meq_options* opt,
+                           size_t* persistent_bytes, size_t* workspace_bytes);
+
+/* Create the state for n matrices: zeroed momentum (B_{-1} = 0, Algorithm 1)
+ * and the workspace, on the current CUDA device. opt may be NULL (defaults).
+ * cuda_stream (cudaStream_t, may be NULL) orders the zero-fill. The shape
+ * list is copied. On success *out owns device memory until meq_free. */
+meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt,
+                          void* cuda_stream, meq_state** out);
+
+/* One MeqMuon step over all n matrices (Algorithm 1, hidden branch).
+ *   params[i]: device fp32 W_i (rows x cols), updated in place.
+ *   grads[i] : device fp32 G_i, read only.
+ *   shapes/n : must equal the list given to meq_init_state.
+ *   lr = eta_t (the caller applies warm-up / decay), momentum = mu,
+ *   weight_decay = lambda, eps = delta of Section 3.1 (1e-7).
+ * All work is enqueued on cuda_stream (cudaStream_t; NULL = legacy default
+ * stream) with no host synchronisation. params/grads must stay valid until
+ * the enqueued work has run. */
+meq_status meq_step(float* const* params, const float* const* grads, meq_state* st,
+                    const meq_shape* shapes, int n, float lr, float momentum,
+                    float weight_decay, float eps, void* cuda_stream);
+
+/* Wait for the state's enqueued work and report device-side errors
+ * (MEQ_ERR_TIMEOUT for an expired bounded wait, MEQ_ERR_CUDA otherwise). */
+meq_status meq_sync(meq_state* st);
+
+/* Release all device memory of the state (synchronises first). NULL is a no-op. */
+meq_status meq_free(meq_state* st);
+
+/* Human-readable text of the last error of st (or of the last init failure
+ * when st is NULL). Valid until the next call on the same state. */
+const char* meq_last_error(const meq_state* st);
+const char* meq_status_string(meq_status s);
+
+/* ---- inspection and checkpointing (synchronise the state first) ---------- */
+
+/* Copy momentum B_i (rows x cols fp32) to dst (host or device memory). */
+meq_status meq_read_momentum(meq_state* st, int i, float* dst);
+/* Overwrite momentum B_i from src (host or device), e.g. to resume. */
+meq_status meq_write_momentum(meq_state* st, int i, const float* src);
+/* Copy the last step's Newton-Schulz output U_i (rows x cols fp32, before
+ * equilibration) to dst (host or device). */
+meq_status meq_read_ns_output(meq_state* st, int i, float* dst);
+/* Last step's statistics of U_i: r (rows floats), c (cols floats) of Eq. (7),
+ * gamma_r, gamma_c of Eq. (8) and the direction of Eq. (11) (0 = row,
+ * 1 = column). Any output may be NULL; r and c are host or device memory. */
+meq_status meq_read_stats(meq_state* st, int i, float* r, float* c,
+                          double* gamma_r, double* gamma_c, int* direction);
+/* Number of kernels one meq_step launches (for launch accounting). */
+int meq_kernels_per_step(const meq_state* st);
+
+/* Per-phase timing with CUDA events on the launch stream. While enabled,
+ * meq_step launches its kernels directly (not from the CUDA graph) and
+ * records an event between phases. meq_read_profile synchronises and returns
+ * the summed milliseconds of each phase since profiling was enabled:
+ *   phase_ms[0] momentum update + norms, [1] X_0 cast, [2] all NS GEMMs,
+ *   [3] statistics + direction, [4] apply; *steps = profiled steps. */
+meq_status meq_set_profiling(meq_state* st, int enable);
+meq_status meq_read_profile(meq_state* st, double* phase_ms /* 5 */, int64_t* steps);
+
+/* Failure-path self test of the device-side bounded waits: launches one
+ * kernel that spins on a flag nothing ever sets, with the given limit
+ * (0 < timeout_ms <= 10000), then synchronises. The kernel gives up when the
+ * limit expires, records the timeout and returns, so the expected result is
+ * MEQ_ERR_TIMEOUT with the context still usable. The paper has no
+ * counterpart; this exists to test error reporting without faulting a GPU. */
+meq_status meq_debug_wait_selftest(meq_state* st, float timeout_ms);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MEQ_H */

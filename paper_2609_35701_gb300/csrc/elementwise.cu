@@ -1,0 +1,415 @@
+// Bandwidth-bound kernels of the MeqMuon step (everything except the NS GEMMs).
+//
+//   momentum_norm : B <- mu B + G (Eq. (10)) in place over every matrix, with
+//                   deterministic per-chunk partial sums of the squared NS
+//                   input; the last chunk of each matrix reduces them (fp64)
+//                   into the X_0 scale alpha0 / ||H||_F of Eq. (5).
+//   cast_x0       : X-hat_0 = 16-bit(alpha0 H / ||H||_F) in the oriented NS
+//                   layout (transposed through shared memory for tall W).
+//   stats         : row sums of squares and per-slab column partial sums of
+//                   U (Eq. (7)), deterministic.
+//   finalize      : r, c (Eq. (7)), gamma_r, gamma_c (Eq. (8), fp64), the
+//                   direction (Eq. (11)) and the scale vector of Eq. (9).
+//   apply         : W <- (1 - lr wd) W - rho lr s (.) U (Eq. (14)).
+#include "meq_elementwise.cuh"
+
+namespace meq {
+namespace {
+
+constexpr int kThreads = 256;
+
+__device__ __forceinline__ int find_mat(const MatInfo* mats, int nmat, int64_t key, int which) {
+  // Largest i with begin(i) <= key; begin is nondecreasing in i.
+  int lo = 0, hi = nmat - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    const int64_t b = which == 0 ? mats[mid].chunk_begin : (which == 1 ? mats[mid].tile_begin : mats[mid].slab_begin);
+    if (b <= key) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+__device__ __forceinline__ float block_sum_f32(float v, float* sh) {
+  const unsigned FULL = 0xffffffffu;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL, v, o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) sh[w] = v;
+  __syncthreads();
+  float r = 0.f;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) r += sh[i];
+    sh[0] = r;
+  }
+  __syncthreads();
+  return sh[0];
+}
+
+__device__ __forceinline__ double block_sum_f64(double v, double* sh) {
+  const unsigned FULL = 0xffffffffu;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL, v, o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) sh[w] = v;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double r = 0.0;
+    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) r += sh[i];
+    sh[0] = r;
+  }
+  __syncthreads();
+  return sh[0];
+}
+
+// ------------------------------------------------------------- momentum + norm
+__global__ void __launch_bounds__(kThreads) momentum_norm_kernel(const MatInfo* __restrict__ mats, int nmat,
+                                                                 const GroupInfo* __restrict__ groups,
+                                                                 float* __restrict__ mom,
+                                                                 const float* const* __restrict__ grads,
+                                                                 const StepScalars* __restrict__ sc,
+                                                                 float* __restrict__ partials,
+                                                                 unsigned int* __restrict__ counters,
+                                                                 float* __restrict__ x0scale) {
+  __shared__ double shd[32];
+  __shared__ float shf[32];
+  __shared__ int is_last;
+  const int64_t chunk = blockIdx.x;
+  const int mi = find_mat(mats, nmat, chunk, 0);
+  const MatInfo& M = mats[mi];
+  const int64_t numel = M.m * M.n;
+  const int64_t e0 = (chunk - M.chunk_begin) * kChunk;
+  const int64_t e1 = min(e0 + kChunk, numel);
+  const float mu = sc->mu;
+  const int nesterov = sc->nesterov;
+  float* B = mom + M.mom_off;
+  const float* G = grads[mi];
+  float ss = 0.f;
+  // numel of a matrix need not be a multiple of 4: vector body + scalar tail.
+  const int64_t vec_end = e0 + ((e1 - e0) & ~int64_t(3));
+  for (int64_t e = e0 + 4 * threadIdx.x; e < vec_end; e += 4 * kThreads) {
+    const float4 g = __ldcs(reinterpret_cast<const float4*>(G + e));
+    float4 b = *reinterpret_cast<const float4*>(B + e);
+    b.x = fmaf(mu, b.x, g.x);
+    b.y = fmaf(mu, b.y, g.y);
+    b.z = fmaf(mu, b.z, g.z);
+    b.w = fmaf(mu, b.w, g.w);
+    *reinterpret_cast<float4*>(B + e) = b;
+    if (nesterov) {
+      const float hx = fmaf(mu, b.x, g.x), hy = fmaf(mu, b.y, g.y), hz = fmaf(mu, b.z, g.z), hw = fmaf(mu, b.w, g.w);
+      ss += hx * hx + hy * hy + hz * hz + hw * hw;
+    } else {
+      ss += b.x * b.x + b.y * b.y + b.z * b.z + b.w * b.w;
+    }
+  }
+  for (int64_t e = vec_end + threadIdx.x; e < e1; e += kThreads) {
+    const float g = G[e];
+    const float b = fmaf(mu, B[e], g);
+    B[e] = b;
+    const float h = nesterov ? fmaf(mu, b, g) : b;
+    ss += h * h;
+  }
+  const float part = block_sum_f32(ss, shf);
+  if (threadIdx.x == 0) {
+    partials[chunk] = part;
+    __threadfence();
+    const unsigned int nchunks = static_cast<unsigned int>((numel + kChunk - 1) / kChunk);
+    const unsigned int prev = atomicAdd(&counters[mi], 1u);
+    is_last = (prev + 1 == nchunks);
+  }
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  // Last chunk of this matrix: fixed-order fp64 reduction of its partials.
+  const int64_t nchunks = (numel + kChunk - 1) / kChunk;
+  double acc = 0.0;
+  for (int64_t c = threadIdx.x; c < nchunks; c += kThreads) acc += static_cast<double>(__ldcg(partials + M.chunk_begin + c));
+  const double total = block_sum_f64(acc, shd);
+  if (threadIdx.x == 0) {
+    const double nrm = sqrt(total);
+    const double alpha0 = static_cast<double>(groups[M.group].alpha0);
+    // Zero input: U = 0 (Eq. (5) is defined for a nonzero input only).
+    x0scale[mi] = nrm > 0.0 ? static_cast<float>(alpha0 / nrm) : 0.f;
+    counters[mi] = 0u;
+  }
+}
+
+// ------------------------------------------------------------------ X_0 cast
+template <bool kFp16>
+__device__ __forceinline__ uint16_t half_bits(float v) {
+  if (kFp16) {
+    __half h = __float2half_rn(v);
+    return *reinterpret_cast<uint16_t*>(&h);
+  }
+  __nv_bfloat16 h = __float2bfloat16_rn(v);
+  return *reinterpret_cast<uint16_t*>(&h);
+}
+
+template <bool kFp16>
+__global__ void __launch_bounds__(kThreads) cast_x0_kernel(const MatInfo* __restrict__ mats, int nmat,
+                                                           const GroupInfo* __restrict__ groups,
+                                                           const float* __restrict__ mom,
+                                                           const float* const* __restrict__ grads,
+                                                           const StepScalars* __restrict__ sc,
+                                                           const float* __restrict__ x0scale) {
+  __shared__ float tile[kCastTile][kCastTile + 1];
+  const int64_t t = blockIdx.x;
+  const int mi = find_mat(mats, nmat, t, 1);
+  const MatInfo& M = mats[mi];
+  const GroupInfo& Gi = groups[M.group];
+  const int64_t tiles_n = (M.n + kCastTile - 1) / kCastTile;
+  const int64_t lt = t - M.tile_begin;
+  const int64_t r0 = (lt / tiles_n) * kCastTile;
+  const int64_t c0 = (lt % tiles_n) * kCastTile;
+  const float scale = x0scale[mi];
+  const float mu = sc->mu;
+  const int nesterov = sc->nesterov;
+  const float* B = mom + M.mom_off;
+  const float* G = grads[mi];
+  uint16_t* X = static_cast<uint16_t*>(Gi.x0) + M.gidx * Gi.s * Gi.lp;
+  const int tx = threadIdx.x % kCastTile;
+  const int ty = threadIdx.x / kCastTile;
+  constexpr int kRowsPerPass = kThreads / kCastTile;
+  if (!M.trans) {
+    const int64_t c = c0 + tx;
+    if (c < M.n) {
+      for (int r = ty; r < kCastTile; r += kRowsPerPass) {
+        const int64_t row = r0 + r;
+        if (row >= M.m) break;
+        float h = B[row * M.n + c];
+        if (nesterov) h = fmaf(mu, h, G[row * M.n + c]);
+        X[row * Gi.lp + c] = half_bits<kFp16>(h * scale);
+      }
+    }
+  } else {
+    for (int r = ty; r < kCastTile; r += kRowsPerPass) {
+      const int64_t row = r0 + r, c = c0 + tx;
+      float h = 0.f;
+      if (row < M.m && c < M.n) {
+        h = B[row * M.n + c];
+        if (nesterov) h = fmaf(mu, h, G[row * M.n + c]);
+      }
+      tile[r][tx] = h * scale;
+    }
+    __syncthreads();
+    // X row = W column (c0 + r), X column = W row (r0 + tx).
+    for (int r = ty; r < kCastTile; r += kRowsPerPass) {
+      const int64_t xrow = c0 + r, xcol = r0 + tx;
+      if (xrow < M.n && xcol < M.m) X[xrow * Gi.lp + xcol] = half_bits<kFp16>(tile[tx][r]);
+    }
+  }
+}
+
+// ----------------------------------------------------------------- statistics
+__global__ void __launch_bounds__(kThreads) stats_kernel(const MatInfo* __restrict__ mats, int nmat,
+                                                         const float* __restrict__ uslab,
+                                                         float* __restrict__ rowss,
+                                                         float* __restrict__ cpart) {
+  __shared__ float shr[kThreads / 32][32];
+  const int64_t slab = blockIdx.x;
+  const int mi = find_mat(mats, nmat, slab, 2);
+  const MatInfo& M = mats[mi];
+  const int64_t ls = slab - M.slab_begin;
+  const int64_t r0 = ls * kSlab;
+  const int nr = static_cast<int>(M.m - r0 < kSlab ? M.m - r0 : kSlab);
+  const float* U = uslab + M.u_off + r0 * M.un;
+  float racc[kSlab];
+#pragma unroll
+  for (int r = 0; r < kSlab; ++r) racc[r] = 0.f;
+  float* cp = cpart + M.cpart_off + ls * M.n;
+  for (int64_t c = threadIdx.x; c < M.n; c += kThreads) {
+    float cacc = 0.f;
+#pragma unroll
+    for (int r = 0; r < kSlab; ++r) {
+      if (r < nr) {
+        const float u = __ldcs(U + r * M.un + c);
+        const float u2 = u * u;
+        cacc += u2;
+        racc[r] += u2;
+      }
+    }
+    cp[c] = cacc;
+  }
+  // Transpose-reduce the 32 row accumulators across the warp: lane l ends
+  // with the warp's sum for row l.
+  const unsigned FULL = 0xffffffffu;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const bool up = (lane & o) != 0;
+      const float send = up ? racc[i] : racc[i + o];
+      const float keep = up ? racc[i + o] : racc[i];
+      racc[i] = keep + __shfl_xor_sync(FULL, send, o);
+    }
+  }
+  shr[w][lane] = racc[0];
+  __syncthreads();
+  if (threadIdx.x < nr) {
+    float s = 0.f;
+    for (int i = 0; i < kThreads / 32; ++i) s += shr[i][threadIdx.x];
+    rowss[M.vec_off + r0 + threadIdx.x] = s;
+  }
+}
+
+// Row / column RMS, CVs (fp64), direction and scale vector; one block per matrix.
+__global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __restrict__ mats,
+                                                               const StepScalars* __restrict__ sc,
+                                                               const float* __restrict__ rowss,
+                                                               const float* __restrict__ cpart,
+                                                               float* __restrict__ rvec, float* __restrict__ cvec,
+                                                               float* __restrict__ svec,
+                                                               MatStats* __restrict__ stats) {
+  __shared__ double shd[32];
+  const MatInfo& M = mats[blockIdx.x];
+  const float delta = sc->eps;
+  const int64_t nslabs = (M.m + kSlab - 1) / kSlab;
+  float* r = rvec + M.vec_off;
+  float* c = cvec + M.vec_off;
+  float* s = svec + M.vec_off;
+  const float inv_n = 1.0f / static_cast<float>(M.n);
+  const float inv_m = 1.0f / static_cast<float>(M.m);
+  for (int64_t i = threadIdx.x; i < M.m; i += blockDim.x) r[i] = sqrtf(rowss[M.vec_off + i] * inv_n);
+  for (int64_t j = threadIdx.x; j < M.n; j += blockDim.x) {
+    float acc = 0.f;
+    const float* cp = cpart + M.cpart_off + j;
+    for (int64_t k = 0; k < nslabs; ++k) acc += cp[k * M.n];
+    c[j] = sqrtf(acc * inv_m);
+  }
+  __syncthreads();
+  double gam[2];
+  for (int side = 0; side < 2; ++side) {
+    const float* v = side == 0 ? r : c;
+    const int64_t len = side == 0 ? M.m : M.n;
+    double cnt = 0.0, sum = 0.0;
+    for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
+      const float x = v[i];
+      if (x > delta) cnt += 1.0, sum += static_cast<double>(x);
+    }
+    cnt = block_sum_f64(cnt, shd);
+    sum = block_sum_f64(sum, shd);
+    const double mean = cnt > 0.0 ? sum / cnt : 0.0;
+    double var = 0.0;
+    for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
+      const double x = static_cast<double>(v[i]);
+      if (v[i] > delta) var += (x - mean) * (x - mean);
+    }
+    var = block_sum_f64(var, shd);
+    gam[side] = cnt > 0.0 ? sqrt(var / cnt) / mean : 0.0;
+  }
+  const int dir = gam[0] >= gam[1] - static_cast<double>(sc->tie_atol) ? 0 : 1;
+  const float* v = dir == 0 ? r : c;
+  const int64_t len = dir == 0 ? M.m : M.n;
+  for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
+    const float x = v[i];
+    s[i] = x > delta ? 1.0f / x : 0.0f;   // RMS at or below delta: treated as zero
+  }
+  if (threadIdx.x == 0) {
+    stats[blockIdx.x].gamma_r = gam[0];
+    stats[blockIdx.x].gamma_c = gam[1];
+    stats[blockIdx.x].direction = dir;
+  }
+}
+
+// ----------------------------------------------------------------------- apply
+__global__ void __launch_bounds__(kThreads) apply_kernel(const MatInfo* __restrict__ mats, int nmat,
+                                                         float* const* __restrict__ params,
+                                                         const float* __restrict__ uslab,
+                                                         const float* __restrict__ svec,
+                                                         const MatStats* __restrict__ stats,
+                                                         const StepScalars* __restrict__ sc) {
+  const int64_t chunk = blockIdx.x;
+  const int mi = find_mat(mats, nmat, chunk, 0);
+  const MatInfo& M = mats[mi];
+  const int64_t numel = M.m * M.n;
+  const int64_t e0 = (chunk - M.chunk_begin) * kChunk;
+  const int64_t e1 = min(e0 + kChunk, numel);
+  const float decay = 1.0f - sc->lr * sc->wd;
+  const float step = sc->rho * sc->lr;
+  const int dir = stats[mi].direction;
+  const float* sv = svec + M.vec_off;
+  const float* U = uslab + M.u_off;
+  float* W = params[mi];
+  if ((M.n & 3) == 0) {
+    // Rows are whole float4s and the U stride equals n.
+    for (int64_t e = e0 + 4 * threadIdx.x; e < e1; e += 4 * kThreads) {
+      const int64_t i = e / M.n, j = e - i * M.n;
+      float4 w = *reinterpret_cast<const float4*>(W + e);
+      const float4 u = __ldcs(reinterpret_cast<const float4*>(U + e));
+      float s0, s1, s2, s3;
+      if (dir == 0) {
+        s0 = s1 = s2 = s3 = sv[i];
+      } else {
+        const float4 s4 = *reinterpret_cast<const float4*>(sv + j);
+        s0 = s4.x, s1 = s4.y, s2 = s4.z, s3 = s4.w;
+      }
+      w.x = fmaf(decay, w.x, -step * (s0 * u.x));
+      w.y = fmaf(decay, w.y, -step * (s1 * u.y));
+      w.z = fmaf(decay, w.z, -step * (s2 * u.z));
+      w.w = fmaf(decay, w.w, -step * (s3 * u.w));
+      *reinterpret_cast<float4*>(W + e) = w;
+    }
+  } else {
+    for (int64_t e = e0 + threadIdx.x; e < e1; e += kThreads) {
+      const int64_t i = e / M.n, j = e - i * M.n;
+      const float u = U[i * M.un + j];
+      const float s = dir == 0 ? sv[i] : sv[j];
+      W[e] = fmaf(decay, W[e], -step * (s * u));
+    }
+  }
+}
+
+// Bounded-wait self test: waits on a flag nobody sets and reports a timeout.
+__global__ void wait_selftest_kernel(const volatile int* flag, int* err, unsigned long long timeout_ns) {
+  unsigned long long t0;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+  for (unsigned int it = 0;; ++it) {
+    if (*flag != 0) return;
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    if (t - t0 > timeout_ns || it >= (1u << 28)) {
+      atomicCAS(err, 0, DEV_TIMEOUT_TEST);
+      return;
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_momentum_norm(const LaunchCtx& L, cudaStream_t st) {
+  momentum_norm_kernel<<<(unsigned)L.total_chunks, kThreads, 0, st>>>(L.mats, L.nmat, L.groups, L.mom, L.grads, L.sc,
+                                                                    L.partials, L.counters, L.x0scale);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st) {
+  if (fp16)
+    cast_x0_kernel<true><<<(unsigned)L.total_tiles, kThreads, 0, st>>>(L.mats, L.nmat, L.groups, L.mom, L.grads, L.sc,
+                                                                      L.x0scale);
+  else
+    cast_x0_kernel<false><<<(unsigned)L.total_tiles, kThreads, 0, st>>>(L.mats, L.nmat, L.groups, L.mom, L.grads, L.sc,
+                                                                       L.x0scale);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st) {
+  stats_kernel<<<(unsigned)L.total_slabs, kThreads, 0, st>>>(L.mats, L.nmat, L.uslab, L.rowss, L.cpart);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  finalize_kernel<<<L.nmat, kFinThreads, 0, st>>>(L.mats, L.sc, L.rowss, L.cpart, L.rvec, L.cvec, L.svec, L.stats);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_apply(const LaunchCtx& L, cudaStream_t st) {
+  apply_kernel<<<(unsigned)L.total_chunks, kThreads, 0, st>>>(L.mats, L.nmat, L.params, L.uslab, L.svec, L.stats, L.sc);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wait_selftest(const int* flag, int* err, unsigned long long timeout_ns, cudaStream_t st) {
+  wait_selftest_kernel<<<1, 1, 0, st>>>(flag, err, timeout_ns);
+  return cudaGetLastError();
+}
+
+}  // namespace meq

@@ -1,0 +1,778 @@
+// Host side of the MeqMuon C ABI: planning, workspace, launch sequence.
+//
+// Planning (at meq_init_state):
+//   * every matrix W (m x n) is oriented for Newton-Schulz as s x l with
+//     s = min(m, n): X = W for m <= n, X = W^T for m > n. In exact arithmetic
+//     X (X^T X)^k = (X X^T)^k X, so the iterate of W^T is the transpose of the
+//     iterate of W and the result is the same matrix (Eq. (5));
+//   * matrices with the same (s, l) form a group whose X buffers are stacked
+//     [count][s][l_pad] so one 3D TMA tensor map covers the whole group, and
+//     one GEMM launch covers up to kMaxGroups groups;
+//   * one device arena holds momentum, NS buffers and statistics.
+// Per step (meq_step), on the caller's stream:
+//   upload step scalars + pointer tables, then
+//   momentum_norm, cast_x0, K x (GRAM, POLY, XUPD|XLAST), stats, finalize, apply
+// optionally replayed from a CUDA graph captured at the first step.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/meq.h"
+#include "meq_elementwise.cuh"
+
+using namespace meq;
+
+namespace {
+
+constexpr int64_t kAlignBytes = 1024;
+
+int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+std::string g_init_error;  // last meq_init_state failure text
+
+struct Group {
+  int64_t s = 0, l = 0, lp = 0, sp = 0, count = 0;
+  std::vector<int> mats;
+  uint16_t* x[2] = {nullptr, nullptr};
+  float* a32 = nullptr;
+  uint16_t* a16 = nullptr;
+  uint16_t* p16 = nullptr;
+  float alpha0 = 1.f, alpha = 1.f;
+};
+
+// Sub-allocation plan of the arena (offsets in bytes).
+struct Layout {
+  int64_t total = 0;
+  int64_t add(int64_t bytes) {
+    const int64_t off = total;
+    total += round_up(std::max<int64_t>(bytes, 1), kAlignBytes);
+    return off;
+  }
+};
+
+}  // namespace
+
+struct meq_state {
+  int n = 0;
+  std::vector<meq_shape> shapes;
+  meq_options opt{};
+  int device = 0;
+  int num_sms = 0;
+  std::vector<MatInfo> mats;
+  std::vector<Group> groups;
+  int64_t total_chunks = 0, total_tiles = 0, total_slabs = 0;
+  int64_t mom_floats = 0, u_floats = 0, vec_floats = 0, cpart_floats = 0;
+  char* arena = nullptr;
+  int64_t arena_bytes = 0;
+  // device views
+  MatInfo* d_mats = nullptr;
+  MatInfo* d_mats_bg = nullptr;
+  GroupInfo* d_groups = nullptr;
+  float* d_mom = nullptr;
+  float* d_u = nullptr;
+  float* d_rvec = nullptr;
+  float* d_cvec = nullptr;
+  float* d_svec = nullptr;
+  float* d_rowss = nullptr;
+  float* d_cpart = nullptr;
+  float* d_partials = nullptr;
+  unsigned int* d_counters = nullptr;
+  float* d_x0scale = nullptr;
+  MatStats* d_stats = nullptr;
+  char* d_step = nullptr;  // StepScalars, params[n], grads[n]
+  int* d_err = nullptr;
+  int* d_flag = nullptr;
+  int64_t step_bytes = 0;
+  std::vector<char> step_host;
+  // launch plan
+  std::vector<GemmParams> gemm;  // in launch order
+  std::vector<int> gemm_grid;
+  LaunchCtx ctx{};
+  bool graph_ready = false;
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t gexec = nullptr;
+  cudaStream_t last_stream = nullptr;
+  int kernels_per_step = 0;
+  bool profiling = false;
+  std::vector<std::vector<cudaEvent_t>> prof_events;  // 6 events per profiled step
+  std::string last_error;
+  int64_t persistent_bytes = 0;
+};
+
+namespace {
+
+meq_status fail(meq_state* st, meq_status s, const std::string& msg) {
+  if (st) st->last_error = msg; else g_init_error = msg;
+  return s;
+}
+
+meq_status cuda_fail(meq_state* st, cudaError_t e, const char* what) {
+  return fail(st, MEQ_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+bool valid_options(const meq_options& o, std::string* why) {
+  if (o.ns_steps < 1 || o.ns_steps > 16) { *why = "ns_steps must be in 1..16"; return false; }
+  if (!(o.rho > 0.f) || !std::isfinite(o.rho)) { *why = "rho must be positive and finite"; return false; }
+  if (!std::isfinite(o.ns_a) || !std::isfinite(o.ns_b) || !std::isfinite(o.ns_c)) { *why = "NS coefficients must be finite"; return false; }
+  if (!(o.tie_atol >= 0.f)) { *why = "tie_atol must be >= 0"; return false; }
+  if (!(o.wait_timeout_ms > 0.f)) { *why = "wait_timeout_ms must be > 0"; return false; }
+  if (o.workspace_limit_bytes < 0) { *why = "workspace_limit_bytes must be >= 0"; return false; }
+  return true;
+}
+
+bool valid_shapes(const meq_shape* shapes, int n, std::string* why) {
+  if (n <= 0) { *why = "n must be positive"; return false; }
+  if (!shapes) { *why = "shapes is NULL"; return false; }
+  for (int i = 0; i < n; ++i) {
+    const int64_t m = shapes[i].rows, c = shapes[i].cols;
+    if (m <= 0 || c <= 0) { *why = "matrix " + std::to_string(i) + " has a non-positive dimension"; return false; }
+    // TMA coordinates are 32-bit and the GEMM tile counters are int.
+    if (m > (int64_t(1) << 20) || c > (int64_t(1) << 20) || m * c > (int64_t(1) << 34)) {
+      *why = "matrix " + std::to_string(i) + " exceeds the supported size (dims <= 2^20, elements <= 2^34)";
+      return false;
+    }
+  }
+  return true;
+}
+
+float pow2_round(double x) { return static_cast<float>(std::ldexp(1.0, static_cast<int>(std::lround(std::log2(std::max(x, 1.0)))))); }
+
+// Builds the whole plan (shapes -> groups, offsets, sizes). Allocation-free.
+void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* off_vec4, int64_t* off_cpart,
+          int64_t* off_partials, int64_t* off_counters, int64_t* off_x0s, int64_t* off_stats, int64_t* off_step,
+          int64_t* off_err, int64_t* off_mats, int64_t* off_mats_bg, int64_t* off_groups,
+          std::vector<int64_t>* group_offs) {
+  const int n = st->n;
+  st->mats.assign(n, MatInfo{});
+  std::map<std::pair<int64_t, int64_t>, int> gmap;
+  st->groups.clear();
+  for (int i = 0; i < n; ++i) {
+    const int64_t m = st->shapes[i].rows, c = st->shapes[i].cols;
+    MatInfo& M = st->mats[i];
+    M.m = m, M.n = c;
+    M.s = std::min(m, c), M.l = std::max(m, c);
+    M.trans = m > c ? 1 : 0;
+    auto key = std::make_pair(M.s, M.l);
+    auto it = gmap.find(key);
+    int g;
+    if (it == gmap.end()) {
+      g = static_cast<int>(st->groups.size());
+      gmap[key] = g;
+      Group G;
+      G.s = M.s, G.l = M.l;
+      G.lp = round_up(M.l, 64), G.sp = round_up(M.s, 64);
+      G.alpha0 = std::min(pow2_round(std::sqrt(static_cast<double>(M.s) * static_cast<double>(M.l))), 16384.f);
+      G.alpha = std::min(pow2_round(std::sqrt(static_cast<double>(M.l))), 16384.f);
+      st->groups.push_back(G);
+    } else {
+      g = it->second;
+    }
+    M.group = g;
+    M.gidx = st->groups[g].count++;
+    st->groups[g].mats.push_back(i);
+  }
+  int64_t mom = 0, u = 0, vec = 0, cp = 0, chunks = 0, tiles = 0, slabs = 0;
+  for (int i = 0; i < n; ++i) {
+    MatInfo& M = st->mats[i];
+    M.un = round_up(M.n, 4);
+    M.mom_off = mom;
+    mom += round_up(M.m * M.n, 64);
+    M.u_off = u;
+    u += round_up(M.m * M.un, 64);
+    M.vec_off = vec;
+    vec += round_up(std::max(M.m, M.n), 64);
+    M.chunk_begin = chunks;
+    chunks += (M.m * M.n + kChunk - 1) / kChunk;
+    M.tile_begin = tiles;
+    tiles += ((M.m + kCastTile - 1) / kCastTile) * ((M.n + kCastTile - 1) / kCastTile);
+    M.slab_begin = slabs;
+    const int64_t ns = (M.m + kSlab - 1) / kSlab;
+    slabs += ns;
+    M.cpart_off = cp;
+    cp += round_up(ns * M.n, 64);
+  }
+  st->mom_floats = mom, st->u_floats = u, st->vec_floats = vec, st->cpart_floats = cp;
+  st->total_chunks = chunks, st->total_tiles = tiles, st->total_slabs = slabs;
+  st->persistent_bytes = 0;
+  for (int i = 0; i < n; ++i) st->persistent_bytes += 4 * st->mats[i].m * st->mats[i].n;
+
+  *off_mom = L->add(mom * 4);
+  *off_u = L->add(u * 4);
+  *off_vec4 = L->add(vec * 4 * 4);  // r, c, scale, row sums of squares
+  *off_cpart = L->add(cp * 4);
+  *off_partials = L->add(chunks * 4);
+  *off_counters = L->add(int64_t(n) * 4);
+  *off_x0s = L->add(int64_t(n) * 4);
+  *off_stats = L->add(int64_t(n) * sizeof(MatStats));
+  st->step_bytes = sizeof(StepScalars) + 2 * int64_t(n) * sizeof(void*);
+  *off_step = L->add(st->step_bytes);
+  *off_err = L->add(64);
+  *off_mats = L->add(int64_t(n) * sizeof(MatInfo));
+  *off_mats_bg = L->add(int64_t(n) * sizeof(MatInfo));
+  *off_groups = L->add(int64_t(st->groups.size()) * sizeof(GroupInfo));
+  group_offs->clear();
+  for (auto& G : st->groups) {
+    const int64_t xb = G.count * G.s * G.lp * 2;
+    const int64_t sb = G.count * G.s * G.sp;
+    group_offs->push_back(L->add(xb));
+    group_offs->push_back(L->add(xb));
+    group_offs->push_back(L->add(sb * 4));
+    group_offs->push_back(L->add(sb * 2));
+    group_offs->push_back(L->add(sb * 2));
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 3D map over [count][rows][row_stride] 16-bit elements, 128-byte swizzle.
+bool encode_map(CUtensorMap* m, void* base, int64_t inner, int64_t rows, int64_t count, int64_t row_stride_elems,
+                uint32_t box_inner, uint32_t box_rows) {
+  auto enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows), static_cast<cuuint64_t>(count)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(row_stride_elems * 2),
+                           static_cast<cuuint64_t>(rows * row_stride_elems * 2)};
+  cuuint32_t box[3] = {box_inner, box_rows, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT16, 3, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// tcgen05 kind::f16 instruction descriptor: D fp32, A/B fp16 (0) or bf16 (1),
+// A K-major, B K-major or MN-major, N = 256, M = 128.
+uint32_t make_idesc(bool fp16, bool b_mn_major) {
+  const uint32_t fmt = fp16 ? 0u : 1u;
+  return (1u << 4) | (fmt << 7) | (fmt << 10) | ((b_mn_major ? 1u : 0u) << 16) | ((256u >> 3) << 17) |
+         ((128u >> 4) << 24);
+}
+
+bool iter_fp16(const meq_options& o, int k) { return k < 32 && ((o.ns_fp16_mask >> k) & 1u); }
+
+// Prebuilds the GemmParams of every NS launch of one step.
+bool build_gemm_plan(meq_state* st, std::string* why) {
+  st->gemm.clear();
+  st->gemm_grid.clear();
+  const int K = st->opt.ns_steps;
+  const int ng = static_cast<int>(st->groups.size());
+  for (int k = 0; k < K; ++k) {
+    const bool f16 = iter_fp16(st->opt, k);
+    const bool next_f16 = (k + 1 < K) ? iter_fp16(st->opt, k + 1) : false;
+    const int cur = k & 1, nxt = cur ^ 1;
+    for (int mode = MODE_GRAM; mode <= MODE_XUPD; ++mode) {
+      const int real_mode = (mode == MODE_XUPD && k == K - 1) ? MODE_XLAST : mode;
+      for (int g0 = 0; g0 < ng; g0 += kMaxGroups) {
+        GemmParams P;
+        std::memset(&P, 0, sizeof(P));
+        P.mode = real_mode;
+        P.b_mn_major = (mode == MODE_XUPD) ? 1 : 0;
+        P.idesc = make_idesc(f16, P.b_mn_major);
+        P.ca = st->opt.ns_a, P.cb = st->opt.ns_b, P.cc = st->opt.ns_c;
+        P.mats = st->d_mats_bg;
+        P.u_slab = st->d_u;
+        P.err = st->d_err;
+        P.timeout_ns = static_cast<unsigned long long>(static_cast<double>(st->opt.wait_timeout_ms) * 1e6);
+        int tiles = 0;
+        P.ngroups = std::min(kMaxGroups, ng - g0);
+        for (int gi = 0; gi < P.ngroups; ++gi) {
+          Group& G = st->groups[g0 + gi];
+          GemmGroup& Q = P.g[gi];
+          const float ak = (k == 0) ? G.alpha0 : G.alpha;
+          Q.count = static_cast<int32_t>(G.count);
+          Q.mat_base = 0;
+          bool ok = true;
+          if (mode == MODE_GRAM) {
+            Q.M = (int32_t)G.s, Q.N = (int32_t)G.s, Q.K = (int32_t)G.l;
+            ok &= encode_map(&Q.tmA, G.x[cur], G.l, G.s, G.count, G.lp, 64, 128);
+            ok &= encode_map(&Q.tmB, G.x[cur], G.l, G.s, G.count, G.lp, 64, 256);
+            Q.out0 = G.a32, Q.ld0 = G.sp, Q.mstride0 = G.s * G.sp;
+            Q.out1 = G.a16, Q.ld1 = G.sp, Q.mstride1 = G.s * G.sp;
+            Q.scale = 1.0f / (ak * ak);
+            Q.out_half_is_fp16 = f16;
+          } else if (mode == MODE_POLY) {
+            Q.M = (int32_t)G.s, Q.N = (int32_t)G.s, Q.K = (int32_t)G.s;
+            ok &= encode_map(&Q.tmA, G.a16, G.s, G.s, G.count, G.sp, 64, 128);
+            ok &= encode_map(&Q.tmB, G.a16, G.s, G.s, G.count, G.sp, 64, 256);
+            Q.out0 = G.p16, Q.ld0 = G.sp, Q.mstride0 = G.s * G.sp;
+            Q.aux = G.a32, Q.ldaux = G.sp, Q.mstrideaux = G.s * G.sp;
+            Q.out_half_is_fp16 = f16;
+          } else {
+            Q.M = (int32_t)G.s, Q.N = (int32_t)G.l, Q.K = (int32_t)G.s;
+            ok &= encode_map(&Q.tmA, G.p16, G.s, G.s, G.count, G.sp, 64, 128);
+            ok &= encode_map(&Q.tmB, G.x[cur], G.l, G.s, G.count, G.lp, 64, 64);
+            if (real_mode == MODE_XUPD) {
+              Q.out0 = G.x[nxt], Q.ld0 = G.lp, Q.mstride0 = G.s * G.lp;
+              Q.scale = G.alpha / ak;
+              Q.out_half_is_fp16 = next_f16;
+            } else {
+              Q.scale = 1.0f / ak;
+              Q.mat_base = 0;
+            }
+          }
+          if (!ok) { *why = "cuTensorMapEncodeTiled failed"; return false; }
+          Q.tiles_m = (int32_t)((Q.M + 127) / 128);
+          Q.tiles_n = (int32_t)((Q.N + 255) / 256);
+          Q.tile_begin = tiles;
+          const int64_t t = int64_t(Q.tiles_m) * Q.tiles_n * Q.count;
+          if (tiles + t > (int64_t(1) << 30)) { *why = "too many GEMM tiles in one launch"; return false; }
+          tiles += static_cast<int>(t);
+        }
+        P.total_tiles = tiles;
+        st->gemm.push_back(P);
+        st->gemm_grid.push_back(std::max(1, std::min(tiles, st->num_sms)));
+      }
+    }
+  }
+  return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+void meq_default_options(meq_options* o) {
+  if (!o) return;
+  std::memset(o, 0, sizeof(*o));
+  o->rho = 0.2f;
+  o->ns_steps = 5;
+  o->ns_a = 3.4445f;
+  o->ns_b = -4.7750f;
+  o->ns_c = 2.0315f;
+  o->nesterov = 0;
+  o->ns_fp16_mask = 0xFFFFFFFFu;
+  o->tie_atol = 1e-6f;
+  o->use_graph = 1;
+  o->workspace_limit_bytes = 0;
+  o->wait_timeout_ms = 4000.f;
+}
+
+const char* meq_status_string(meq_status s) {
+  switch (s) {
+    case MEQ_OK: return "MEQ_OK";
+    case MEQ_ERR_INVALID_ARG: return "MEQ_ERR_INVALID_ARG";
+    case MEQ_ERR_OOM: return "MEQ_ERR_OOM";
+    case MEQ_ERR_CUDA: return "MEQ_ERR_CUDA";
+    case MEQ_ERR_NONFINITE: return "MEQ_ERR_NONFINITE";
+    case MEQ_ERR_TIMEOUT: return "MEQ_ERR_TIMEOUT";
+    case MEQ_ERR_UNSUPPORTED: return "MEQ_ERR_UNSUPPORTED";
+  }
+  return "MEQ_ERR_UNKNOWN";
+}
+
+const char* meq_last_error(const meq_state* st) { return st ? st->last_error.c_str() : g_init_error.c_str(); }
+
+meq_status meq_state_bytes(const meq_shape* shapes, int n, const meq_options* opt, size_t* persistent, size_t* workspace) {
+  meq_options o;
+  if (opt) o = *opt; else meq_default_options(&o);
+  std::string why;
+  if (!valid_shapes(shapes, n, &why) || !valid_options(o, &why)) return fail(nullptr, MEQ_ERR_INVALID_ARG, why);
+  meq_state tmp;
+  tmp.n = n;
+  tmp.shapes.assign(shapes, shapes + n);
+  tmp.opt = o;
+  Layout L;
+  int64_t a[14];
+  std::vector<int64_t> goffs;
+  plan(&tmp, &L, &a[0], &a[1], &a[2], &a[3], &a[4], &a[5], &a[6], &a[7], &a[8], &a[9], &a[10], &a[11], &a[12], &goffs);
+  if (persistent) *persistent = static_cast<size_t>(tmp.persistent_bytes);
+  if (workspace) *workspace = static_cast<size_t>(L.total - tmp.persistent_bytes);
+  return MEQ_OK;
+}
+
+meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt, void* cuda_stream, meq_state** out) {
+  if (!out) return fail(nullptr, MEQ_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  meq_options o;
+  if (opt) o = *opt; else meq_default_options(&o);
+  std::string why;
+  if (!valid_shapes(shapes, n, &why) || !valid_options(o, &why)) return fail(nullptr, MEQ_ERR_INVALID_ARG, why);
+
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(nullptr, MEQ_ERR_UNSUPPORTED, std::string("no CUDA device: ") + cudaGetErrorString(e));
+  cudaDeviceProp prop;
+  e = cudaGetDeviceProperties(&prop, dev);
+  if (e != cudaSuccess) return fail(nullptr, MEQ_ERR_CUDA, std::string("cudaGetDeviceProperties: ") + cudaGetErrorString(e));
+  if (prop.major != 10 || prop.minor != 3)
+    return fail(nullptr, MEQ_ERR_UNSUPPORTED,
+                "this library is built for sm_103a (GB300); device is sm_" + std::to_string(prop.major) + std::to_string(prop.minor));
+  if (prop.sharedMemPerBlockOptin < static_cast<size_t>(ns_gemm_smem_bytes()))
+    return fail(nullptr, MEQ_ERR_UNSUPPORTED, "not enough opt-in shared memory per block");
+  if (!get_encode()) return fail(nullptr, MEQ_ERR_UNSUPPORTED, "cuTensorMapEncodeTiled is not available from the driver");
+
+  e = prepare_ns_gemm();
+  if (e != cudaSuccess) return fail(nullptr, MEQ_ERR_CUDA, std::string("cudaFuncSetAttribute: ") + cudaGetErrorString(e));
+
+  meq_state* st = new meq_state();
+  st->n = n;
+  st->shapes.assign(shapes, shapes + n);
+  st->opt = o;
+  st->device = dev;
+  st->num_sms = prop.multiProcessorCount;
+
+  Layout L;
+  int64_t off_mom, off_u, off_vec4, off_cpart, off_partials, off_counters, off_x0s, off_stats, off_step, off_err, off_mats,
+      off_mats_bg, off_groups;
+  std::vector<int64_t> goffs;
+  plan(st, &L, &off_mom, &off_u, &off_vec4, &off_cpart, &off_partials, &off_counters, &off_x0s, &off_stats, &off_step,
+       &off_err, &off_mats, &off_mats_bg, &off_groups, &goffs);
+  if (o.workspace_limit_bytes > 0 && L.total > o.workspace_limit_bytes) {
+    delete st;
+    return fail(nullptr, MEQ_ERR_OOM, "state needs " + std::to_string(L.total) + " bytes, above workspace_limit_bytes");
+  }
+  e = cudaMalloc(reinterpret_cast<void**>(&st->arena), static_cast<size_t>(L.total));
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    delete st;
+    return fail(nullptr, MEQ_ERR_OOM, "cudaMalloc of " + std::to_string(L.total) + " bytes failed");
+  }
+  st->arena_bytes = L.total;
+  char* A = st->arena;
+  st->d_mom = reinterpret_cast<float*>(A + off_mom);
+  st->d_u = reinterpret_cast<float*>(A + off_u);
+  st->d_rvec = reinterpret_cast<float*>(A + off_vec4);
+  st->d_cvec = st->d_rvec + st->vec_floats;
+  st->d_svec = st->d_cvec + st->vec_floats;
+  st->d_rowss = st->d_svec + st->vec_floats;
+  st->d_cpart = reinterpret_cast<float*>(A + off_cpart);
+  st->d_partials = reinterpret_cast<float*>(A + off_partials);
+  st->d_counters = reinterpret_cast<unsigned int*>(A + off_counters);
+  st->d_x0scale = reinterpret_cast<float*>(A + off_x0s);
+  st->d_stats = reinterpret_cast<MatStats*>(A + off_stats);
+  st->d_step = A + off_step;
+  st->d_err = reinterpret_cast<int*>(A + off_err);
+  st->d_flag = st->d_err + 4;
+  st->d_mats = reinterpret_cast<MatInfo*>(A + off_mats);
+  st->d_mats_bg = reinterpret_cast<MatInfo*>(A + off_mats_bg);
+  st->d_groups = reinterpret_cast<GroupInfo*>(A + off_groups);
+  for (size_t g = 0; g < st->groups.size(); ++g) {
+    Group& G = st->groups[g];
+    G.x[0] = reinterpret_cast<uint16_t*>(A + goffs[5 * g + 0]);
+    G.x[1] = reinterpret_cast<uint16_t*>(A + goffs[5 * g + 1]);
+    G.a32 = reinterpret_cast<float*>(A + goffs[5 * g + 2]);
+    G.a16 = reinterpret_cast<uint16_t*>(A + goffs[5 * g + 3]);
+    G.p16 = reinterpret_cast<uint16_t*>(A + goffs[5 * g + 4]);
+  }
+
+  // MODE_XLAST reads mats_bg[mat_base + index in group]: a copy of the
+  // per-matrix table ordered group by group.
+  std::vector<MatInfo> by_group;
+  std::vector<int> group_base(st->groups.size(), 0);
+  for (size_t g = 0; g < st->groups.size(); ++g) {
+    group_base[g] = static_cast<int>(by_group.size());
+    for (int i : st->groups[g].mats) by_group.push_back(st->mats[i]);
+  }
+
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  std::vector<GroupInfo> gi(st->groups.size());
+  for (size_t g = 0; g < st->groups.size(); ++g) {
+    const Group& G = st->groups[g];
+    gi[g].s = G.s, gi[g].l = G.l, gi[g].lp = G.lp, gi[g].sp = G.sp, gi[g].count = G.count;
+    gi[g].x0 = G.x[0];
+    gi[g].alpha0 = G.alpha0;
+  }
+  bool ok = cudaMemsetAsync(st->arena, 0, static_cast<size_t>(L.total), s) == cudaSuccess;
+  ok = ok && cudaMemcpyAsync(st->d_mats, st->mats.data(), sizeof(MatInfo) * n, cudaMemcpyHostToDevice, s) == cudaSuccess;
+  ok = ok && cudaMemcpyAsync(st->d_groups, gi.data(), sizeof(GroupInfo) * gi.size(), cudaMemcpyHostToDevice, s) == cudaSuccess;
+  ok = ok && cudaMemcpyAsync(st->d_mats_bg, by_group.data(), sizeof(MatInfo) * by_group.size(), cudaMemcpyHostToDevice, s) ==
+                 cudaSuccess;
+  ok = ok && cudaStreamSynchronize(s) == cudaSuccess;
+  if (!ok) {
+    cudaError_t ee = cudaGetLastError();
+    cudaFree(st->arena);
+    delete st;
+    return fail(nullptr, MEQ_ERR_CUDA, std::string("initialising the state failed: ") + cudaGetErrorString(ee));
+  }
+
+  if (!build_gemm_plan(st, &why)) {
+    cudaFree(st->arena);
+    delete st;
+    return fail(nullptr, MEQ_ERR_UNSUPPORTED, why);
+  }
+  // Each launch slot covers groups g0 .. g0 + ngroups - 1, in build order.
+  {
+    const int ng = static_cast<int>(st->groups.size());
+    size_t li = 0;
+    for (int k = 0; k < o.ns_steps; ++k)
+      for (int mode = MODE_GRAM; mode <= MODE_XUPD; ++mode)
+        for (int g0 = 0; g0 < ng; g0 += kMaxGroups, ++li)
+          for (int gi2 = 0; gi2 < st->gemm[li].ngroups; ++gi2) st->gemm[li].g[gi2].mat_base = group_base[g0 + gi2];
+  }
+
+  LaunchCtx& C = st->ctx;
+  C.mats = st->d_mats;
+  C.nmat = n;
+  C.groups = st->d_groups;
+  C.mom = st->d_mom;
+  C.sc = reinterpret_cast<const StepScalars*>(st->d_step);
+  C.params = reinterpret_cast<float* const*>(st->d_step + sizeof(StepScalars));
+  C.grads = reinterpret_cast<const float* const*>(st->d_step + sizeof(StepScalars) + n * sizeof(void*));
+  C.partials = st->d_partials;
+  C.counters = st->d_counters;
+  C.x0scale = st->d_x0scale;
+  C.uslab = st->d_u;
+  C.rowss = st->d_rowss;
+  C.cpart = st->d_cpart;
+  C.rvec = st->d_rvec;
+  C.cvec = st->d_cvec;
+  C.svec = st->d_svec;
+  C.stats = st->d_stats;
+  C.total_chunks = st->total_chunks;
+  C.total_tiles = st->total_tiles;
+  C.total_slabs = st->total_slabs;
+  st->kernels_per_step = 5 + static_cast<int>(st->gemm.size());
+  st->step_host.assign(static_cast<size_t>(st->step_bytes), 0);
+  st->last_stream = s;
+  *out = st;
+  return MEQ_OK;
+}
+
+
+static void drop_profile(meq_state* st) {
+  for (auto& v : st->prof_events)
+    for (auto x : v) cudaEventDestroy(x);
+  st->prof_events.clear();
+}
+
+static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev = nullptr) {
+  const LaunchCtx& C = st->ctx;
+  auto mark = [&](int i) { if (ev) cudaEventRecord(ev[i], s); };
+  mark(0);
+  cudaError_t e = launch_momentum_norm(C, s);
+  if (e != cudaSuccess) return cuda_fail(st, e, "momentum_norm launch");
+  mark(1);
+  e = launch_cast_x0(C, iter_fp16(st->opt, 0), s);
+  if (e != cudaSuccess) return cuda_fail(st, e, "cast_x0 launch");
+  mark(2);
+  for (size_t i = 0; i < st->gemm.size(); ++i) {
+    e = launch_ns_gemm(st->gemm[i], st->gemm_grid[i], s);
+    if (e != cudaSuccess) return cuda_fail(st, e, "ns_gemm launch");
+  }
+  mark(3);
+  e = launch_stats(C, s);
+  if (e != cudaSuccess) return cuda_fail(st, e, "stats launch");
+  mark(4);
+  e = launch_apply(C, s);
+  if (e != cudaSuccess) return cuda_fail(st, e, "apply launch");
+  mark(5);
+  return MEQ_OK;
+}
+
+static meq_status capture_graph(meq_state* st) {
+  cudaStream_t cs = nullptr;
+  cudaError_t e = cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking);
+  if (e != cudaSuccess) return cuda_fail(st, e, "cudaStreamCreate");
+  e = cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal);
+  if (e != cudaSuccess) {
+    cudaStreamDestroy(cs);
+    return cuda_fail(st, e, "cudaStreamBeginCapture");
+  }
+  meq_status ms = enqueue_kernels(st, cs);
+  cudaGraph_t g = nullptr;
+  e = cudaStreamEndCapture(cs, &g);
+  cudaStreamDestroy(cs);
+  if (ms != MEQ_OK) {
+    if (g) cudaGraphDestroy(g);
+    return ms;
+  }
+  if (e != cudaSuccess) return cuda_fail(st, e, "cudaStreamEndCapture");
+  cudaGraphExec_t x = nullptr;
+  e = cudaGraphInstantiate(&x, g, 0);
+  if (e != cudaSuccess) {
+    cudaGraphDestroy(g);
+    return cuda_fail(st, e, "cudaGraphInstantiate");
+  }
+  st->graph = g;
+  st->gexec = x;
+  st->graph_ready = true;
+  return MEQ_OK;
+}
+
+meq_status meq_step(float* const* params, const float* const* grads, meq_state* st, const meq_shape* shapes, int n,
+                    float lr, float momentum, float weight_decay, float eps, void* cuda_stream) {
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  if (!params || !grads || !shapes) return fail(st, MEQ_ERR_INVALID_ARG, "params, grads and shapes must be non-NULL");
+  if (n != st->n) return fail(st, MEQ_ERR_INVALID_ARG, "n differs from the init-time shape list");
+  for (int i = 0; i < n; ++i) {
+    if (shapes[i].rows != st->shapes[i].rows || shapes[i].cols != st->shapes[i].cols)
+      return fail(st, MEQ_ERR_INVALID_ARG, "shape of matrix " + std::to_string(i) + " differs from init");
+    if (!params[i] || !grads[i]) return fail(st, MEQ_ERR_INVALID_ARG, "NULL params/grads pointer at " + std::to_string(i));
+    if ((reinterpret_cast<uintptr_t>(params[i]) & 15u) || (reinterpret_cast<uintptr_t>(grads[i]) & 15u))
+      return fail(st, MEQ_ERR_INVALID_ARG, "params/grads pointer " + std::to_string(i) + " is not 16-byte aligned");
+  }
+  if (!std::isfinite(lr) || !std::isfinite(momentum) || !std::isfinite(weight_decay) || !(eps >= 0.f) || !std::isfinite(eps))
+    return fail(st, MEQ_ERR_INVALID_ARG, "lr, momentum, weight_decay must be finite and eps >= 0");
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  StepScalars sc;
+  std::memset(&sc, 0, sizeof(sc));
+  sc.lr = lr, sc.mu = momentum, sc.wd = weight_decay, sc.eps = eps;
+  sc.rho = st->opt.rho, sc.tie_atol = st->opt.tie_atol, sc.nesterov = st->opt.nesterov;
+  char* h = st->step_host.data();
+  std::memcpy(h, &sc, sizeof(sc));
+  std::memcpy(h + sizeof(sc), params, n * sizeof(void*));
+  std::memcpy(h + sizeof(sc) + n * sizeof(void*), grads, n * sizeof(void*));
+  // Pageable source: the call returns once the bytes are staged, so the
+  // host buffer can be reused by the next step right away.
+  cudaError_t e = cudaMemcpyAsync(st->d_step, h, static_cast<size_t>(st->step_bytes), cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_fail(st, e, "step upload");
+  st->last_stream = s;
+  if (st->profiling) {
+    std::vector<cudaEvent_t> ev(6, nullptr);
+    for (auto& x : ev) {
+      e = cudaEventCreate(&x);
+      if (e != cudaSuccess) return cuda_fail(st, e, "cudaEventCreate");
+    }
+    st->prof_events.push_back(ev);
+    return enqueue_kernels(st, s, st->prof_events.back().data());
+  }
+  if (st->opt.use_graph) {
+    if (!st->graph_ready) {
+      meq_status ms = capture_graph(st);
+      if (ms != MEQ_OK) return ms;
+    }
+    e = cudaGraphLaunch(st->gexec, s);
+    if (e != cudaSuccess) return cuda_fail(st, e, "cudaGraphLaunch");
+    return MEQ_OK;
+  }
+  return enqueue_kernels(st, s);
+}
+
+meq_status meq_sync(meq_state* st) {
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  cudaError_t e = cudaStreamSynchronize(st->last_stream);
+  if (e != cudaSuccess) return cuda_fail(st, e, "cudaStreamSynchronize");
+  int err = 0;
+  e = cudaMemcpy(&err, st->d_err, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(st, e, "reading the device error word");
+  if (err != 0) {
+    int zero = 0;
+    cudaMemcpy(st->d_err, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    char buf[96];
+    std::snprintf(buf, sizeof(buf), "device-side bounded wait expired (code 0x%x)", err);
+    return fail(st, MEQ_ERR_TIMEOUT, buf);
+  }
+  return MEQ_OK;
+}
+
+meq_status meq_free(meq_state* st) {
+  if (!st) return MEQ_OK;
+  cudaStreamSynchronize(st->last_stream);
+  drop_profile(st);
+  if (st->gexec) cudaGraphExecDestroy(st->gexec);
+  if (st->graph) cudaGraphDestroy(st->graph);
+  if (st->arena) cudaFree(st->arena);
+  delete st;
+  return MEQ_OK;
+}
+
+static meq_status check_index(meq_state* st, int i) {
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  if (i < 0 || i >= st->n) return fail(st, MEQ_ERR_INVALID_ARG, "matrix index out of range");
+  cudaError_t e = cudaStreamSynchronize(st->last_stream);
+  if (e != cudaSuccess) return cuda_fail(st, e, "cudaStreamSynchronize");
+  return MEQ_OK;
+}
+
+meq_status meq_read_momentum(meq_state* st, int i, float* dst) {
+  meq_status ms = check_index(st, i);
+  if (ms != MEQ_OK) return ms;
+  if (!dst) return fail(st, MEQ_ERR_INVALID_ARG, "dst is NULL");
+  const MatInfo& M = st->mats[i];
+  cudaError_t e = cudaMemcpy(dst, st->d_mom + M.mom_off, M.m * M.n * sizeof(float), cudaMemcpyDefault);
+  return e == cudaSuccess ? MEQ_OK : cuda_fail(st, e, "cudaMemcpy");
+}
+
+meq_status meq_write_momentum(meq_state* st, int i, const float* src) {
+  meq_status ms = check_index(st, i);
+  if (ms != MEQ_OK) return ms;
+  if (!src) return fail(st, MEQ_ERR_INVALID_ARG, "src is NULL");
+  const MatInfo& M = st->mats[i];
+  cudaError_t e = cudaMemcpy(st->d_mom + M.mom_off, src, M.m * M.n * sizeof(float), cudaMemcpyDefault);
+  return e == cudaSuccess ? MEQ_OK : cuda_fail(st, e, "cudaMemcpy");
+}
+
+meq_status meq_read_ns_output(meq_state* st, int i, float* dst) {
+  meq_status ms = check_index(st, i);
+  if (ms != MEQ_OK) return ms;
+  if (!dst) return fail(st, MEQ_ERR_INVALID_ARG, "dst is NULL");
+  const MatInfo& M = st->mats[i];
+  cudaError_t e = cudaMemcpy2D(dst, M.n * sizeof(float), st->d_u + M.u_off, M.un * sizeof(float), M.n * sizeof(float),
+                               M.m, cudaMemcpyDefault);
+  return e == cudaSuccess ? MEQ_OK : cuda_fail(st, e, "cudaMemcpy2D");
+}
+
+meq_status meq_read_stats(meq_state* st, int i, float* r, float* c, double* gamma_r, double* gamma_c, int* direction) {
+  meq_status ms = check_index(st, i);
+  if (ms != MEQ_OK) return ms;
+  const MatInfo& M = st->mats[i];
+  cudaError_t e = cudaSuccess;
+  if (r) e = cudaMemcpy(r, st->d_rvec + M.vec_off, M.m * sizeof(float), cudaMemcpyDefault);
+  if (e == cudaSuccess && c) e = cudaMemcpy(c, st->d_cvec + M.vec_off, M.n * sizeof(float), cudaMemcpyDefault);
+  MatStats hs;
+  if (e == cudaSuccess) e = cudaMemcpy(&hs, st->d_stats + i, sizeof(hs), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(st, e, "cudaMemcpy");
+  if (gamma_r) *gamma_r = hs.gamma_r;
+  if (gamma_c) *gamma_c = hs.gamma_c;
+  if (direction) *direction = hs.direction;
+  return MEQ_OK;
+}
+
+meq_status meq_set_profiling(meq_state* st, int enable) {
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  cudaError_t e = cudaStreamSynchronize(st->last_stream);
+  if (e != cudaSuccess) return cuda_fail(st, e, "cudaStreamSynchronize");
+  drop_profile(st);
+  st->profiling = enable != 0;
+  return MEQ_OK;
+}
+
+meq_status meq_read_profile(meq_state* st, double* phase_ms, int64_t* steps) {
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  cudaError_t e = cudaStreamSynchronize(st->last_stream);
+  if (e != cudaSuccess) return cuda_fail(st, e, "cudaStreamSynchronize");
+  double acc[5] = {0, 0, 0, 0, 0};
+  for (auto& v : st->prof_events)
+    for (int p = 0; p < 5; ++p) {
+      float ms = 0.f;
+      e = cudaEventElapsedTime(&ms, v[p], v[p + 1]);
+      if (e != cudaSuccess) return cuda_fail(st, e, "cudaEventElapsedTime");
+      acc[p] += ms;
+    }
+  if (phase_ms)
+    for (int p = 0; p < 5; ++p) phase_ms[p] = acc[p];
+  if (steps) *steps = static_cast<int64_t>(st->prof_events.size());
+  return MEQ_OK;
+}
+
+int meq_kernels_per_step(const meq_state* st) { return st ? st->kernels_per_step : 0; }
+
+meq_status meq_debug_wait_selftest(meq_state* st, float timeout_ms) {
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  if (!(timeout_ms > 0.f) || timeout_ms > 10000.f) return fail(st, MEQ_ERR_INVALID_ARG, "timeout_ms must be in (0, 10000]");
+  cudaError_t e = cudaMemsetAsync(st->d_flag, 0, sizeof(int), st->last_stream);
+  if (e == cudaSuccess)
+    e = launch_wait_selftest(st->d_flag, st->d_err, static_cast<unsigned long long>(static_cast<double>(timeout_ms) * 1e6),
+                             st->last_stream);
+  if (e != cudaSuccess) return cuda_fail(st, e, "wait self-test launch");
+  return meq_sync(st);
+}
+
+}  // extern "C"

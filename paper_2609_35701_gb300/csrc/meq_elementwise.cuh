@@ -1,0 +1,48 @@
+// Launch interface of the bandwidth-bound kernels (internal).
+#pragma once
+
+#include "meq_internal.cuh"
+
+namespace meq {
+
+constexpr int64_t kChunk = 4096;   // elements per momentum / apply block
+constexpr int kCastTile = 64;      // X_0 cast tile (64 x 64 of W)
+constexpr int kSlab = 32;          // rows per statistics block
+constexpr int kFinThreads = 1024;  // finalize block size
+
+struct MatStats {
+  double gamma_r;
+  double gamma_c;
+  int32_t direction;  // 0 = row (N_r), 1 = column (N_c)
+  int32_t pad;
+};
+
+// Device pointers and sizes the elementwise launchers need.
+struct LaunchCtx {
+  const MatInfo* mats;
+  int nmat;
+  const GroupInfo* groups;
+  float* mom;
+  const float* const* grads;
+  float* const* params;
+  const StepScalars* sc;
+  float* partials;
+  unsigned int* counters;
+  float* x0scale;
+  float* uslab;
+  float* rowss;
+  float* cpart;
+  float* rvec;
+  float* cvec;
+  float* svec;
+  MatStats* stats;
+  int64_t total_chunks, total_tiles, total_slabs;
+};
+
+cudaError_t launch_momentum_norm(const LaunchCtx& L, cudaStream_t st);
+cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st);
+cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st);  // stats + finalize (2 kernels)
+cudaError_t launch_apply(const LaunchCtx& L, cudaStream_t st);
+cudaError_t launch_wait_selftest(const int* flag, int* err, unsigned long long timeout_ns, cudaStream_t st);
+
+}  // namespace meq

@@ -1,0 +1,98 @@
+// Internal declarations shared by the MeqMuon CUDA sources (not part of the ABI).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace meq {
+
+// ------------------------------------------------------------ error codes
+// Written (first writer wins) to the state's device error word.
+enum DevErr : int {
+  DEV_OK = 0,
+  DEV_TIMEOUT_PRODUCER = 0x101,  // TMA warp waited too long for a free stage
+  DEV_TIMEOUT_MMA_FULL = 0x102,  // MMA warp waited too long for a loaded stage
+  DEV_TIMEOUT_MMA_TMEM = 0x103,  // MMA warp waited too long for a free accumulator
+  DEV_TIMEOUT_EPI = 0x104,       // epilogue waited too long for an accumulator
+  DEV_TIMEOUT_DRAIN = 0x105,     // waiting for in-flight copies / MMAs at exit
+  DEV_TIMEOUT_TEST = 0x1FF,      // the wait-timeout self test
+};
+
+constexpr int kMaxGroups = 8;        // shape groups per GEMM launch
+
+// Per-matrix metadata (device copy built at init).
+struct MatInfo {
+  int64_t m, n;          // W layout: rows, cols
+  int64_t s, l;          // oriented NS shape: s = min(m, n), l = max(m, n)
+  int32_t trans;         // 1 when the NS layout is W^T (m > n)
+  int32_t group;         // shape group
+  int64_t gidx;          // index inside its group
+  int64_t mom_off;       // float offset of B in the momentum slab
+  int64_t u_off;         // float offset of U in the U slab (row stride un)
+  int64_t un;            // U row stride (cols rounded up to 4)
+  int64_t vec_off;       // float offset of r (m), c (n) and scale (max(m, n))
+  int64_t chunk_begin;   // first momentum chunk
+  int64_t tile_begin;    // first cast tile
+  int64_t slab_begin;    // first statistics slab
+  int64_t cpart_off;     // float offset of the column partial sums [nslabs][n]
+};
+
+// Per-group metadata for the elementwise kernels.
+struct GroupInfo {
+  int64_t s, l, lp, sp;  // shape and padded row strides (elements)
+  int64_t count;
+  void* x0;              // X-hat buffer 0: [count][s][lp] 16-bit
+  float alpha0;          // power-of-two storage scale of X_0
+};
+
+// Values that change per step (uploaded before each step).
+struct StepScalars {
+  float lr, mu, wd, eps;
+  float rho, tie_atol;
+  int32_t nesterov;
+  int32_t pad;
+};
+
+// --------------------------------------------------------------- GEMM side
+enum GemmMode : int { MODE_GRAM = 0, MODE_POLY = 1, MODE_XUPD = 2, MODE_XLAST = 3 };
+
+struct GemmGroup {
+  CUtensorMap tmA;        // A operand (K-major), box {64, 128, 1}
+  CUtensorMap tmB;        // B operand: K-major box {64, 256, 1} or MN-major box {64, 64, 1}
+  int32_t M, N, K;        // output rows, output cols, contraction
+  int32_t count;          // matrices in the group
+  int32_t tiles_m, tiles_n;
+  int32_t tile_begin;     // first tile of this group in the launch
+  int32_t mat_base;       // global index of the group's first matrix (XLAST)
+  void* out0;             // GRAM: fp32 A; POLY: 16-bit P; XUPD: 16-bit X next
+  void* out1;             // GRAM: 16-bit A
+  const float* aux;       // POLY: fp32 A
+  int64_t ld0, ld1, ldaux;          // row strides (elements)
+  int64_t mstride0, mstride1, mstrideaux;  // matrix strides (elements)
+  float scale;            // GRAM: 1/alpha^2; XUPD: alpha_next/alpha; XLAST: 1/alpha
+  int32_t out_half_is_fp16;  // output 16-bit format (1 = fp16, 0 = bf16)
+};
+
+struct GemmParams {
+  GemmGroup g[kMaxGroups];
+  int32_t ngroups;
+  int32_t total_tiles;
+  int32_t mode;
+  uint32_t idesc;          // tcgen05 instruction descriptor
+  int32_t b_mn_major;      // 1: B operand tile is MN-major (XUPD)
+  float ca, cb, cc;        // NS coefficients
+  const MatInfo* mats;     // XLAST: per-matrix info (U offsets, transposition)
+  float* u_slab;           // XLAST: U output slab
+  int* err;                // device error word
+  unsigned long long timeout_ns;
+};
+
+// Launchers (defined in the .cu files).
+cudaError_t prepare_ns_gemm();  // sets the kernel's dynamic shared-memory limit (per device)
+cudaError_t launch_ns_gemm(const GemmParams& p, int grid, cudaStream_t st);
+int ns_gemm_smem_bytes();
+
+}  // namespace meq

@@ -1,0 +1,468 @@
+// Newton-Schulz GEMMs on the sm_103a tensor cores (tcgen05 + TMA + TMEM).
+//
+// One persistent, warp-specialised kernel computes every product of the
+// quintic iteration, Eq. (5) of the paper, for a batch of same-shape groups:
+//
+//   MODE_GRAM : A   = X X^T / alpha^2           (s x s, contraction over l)
+//               epilogue writes A in fp32 and in the 16-bit operand format
+//   MODE_POLY : P   = a I + b A + c (A A)       (s x s, contraction over s)
+//               the a I + b A terms use the fp32 copy of A in the epilogue
+//   MODE_XUPD : X'  = P X * (alpha'/alpha)      (s x l, contraction over s)
+//   MODE_XLAST: U   = P X / alpha, written as fp32 in the weight's own layout
+//
+// P X equals a X + (b A + c A^2) X of Eq. (5) exactly in real arithmetic.
+// X is stored scaled by a power of two alpha so its entries stay in the
+// normal range of fp16; the epilogues undo the scale in fp32.
+//
+// Roles (192 threads, one CTA per SM):
+//   warp 0 : TMA producer (one thread), 4-stage shared-memory ring
+//   warp 1 : TMEM allocator and tcgen05.mma issuer (one thread)
+//   warps 2-5 : epilogue; warp w reads TMEM lanes 32*(w%4) .. +31
+// Two 128x256 fp32 accumulators (512 TMEM columns) let the epilogue of one
+// tile overlap the MMAs of the next.
+//
+// Every mbarrier wait is bounded (time and iteration count). On expiry the
+// waiting role records an error code, the others see it and stop, in-flight
+// TMA copies and MMAs are drained with bounded waits, TMEM is freed and the
+// CTA returns.
+#include "meq_internal.cuh"
+
+namespace meq {
+namespace {
+
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4, UK = 16;
+constexpr int A_BYTES = BM * BK * 2;                 // 16 KB
+constexpr int B_BYTES = BN * BK * 2;                 // 32 KB
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;       // 48 KB
+constexpr int NUM_THREADS = 192;
+constexpr uint32_t TMEM_COLS = 512;
+constexpr int NUM_BARS = 2 * STAGES + 4 + 1;         // full, empty, tmem full x2, tmem empty x2, drain
+constexpr int SMEM_BAR_OFF = STAGES * STAGE_BYTES;
+constexpr int SMEM_BYTES = SMEM_BAR_OFF + NUM_BARS * 8 + 16 + 1024;
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ uint32_t mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.b32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Single-thread bounded wait. Returns false when it gave up (its own timeout,
+// recorded in *err, or an error another role recorded).
+__device__ bool wait_bounded(uint32_t bar, uint32_t parity, int* err, int code, uint64_t timeout_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 127u) == 0) {
+      if (*reinterpret_cast<volatile int*>(err) != 0) return false;
+      if (global_ns() - t0 > timeout_ns || it >= (1u << 28)) {
+        atomicCAS(err, 0, code);
+        return false;
+      }
+    }
+  }
+}
+
+// Warp-uniform bounded wait (all 32 lanes call it; all get the same answer).
+__device__ bool wait_bounded_warp(uint32_t bar, uint32_t parity, int* err, int code, uint64_t timeout_ns) {
+  const unsigned FULL = 0xffffffffu;
+  if (__all_sync(FULL, mbar_try_wait(bar, parity))) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (__all_sync(FULL, mbar_try_wait(bar, parity))) return true;
+    if ((it & 127u) == 0) {
+      int stop = 0;
+      if ((threadIdx.x & 31) == 0) {
+        if (*reinterpret_cast<volatile int*>(err) != 0) {
+          stop = 1;
+        } else if (global_ns() - t0 > timeout_ns || it >= (1u << 28)) {
+          atomicCAS(err, 0, code);
+          stop = 1;
+        }
+      }
+      if (__shfl_sync(FULL, stop, 0)) return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* tm, uint32_t bar, int x, int y, int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(bar), "r"(x), "r"(y), "r"(z)
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_tmap(const CUtensorMap* tm) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tc_mma(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+// Shared-memory matrix descriptor for a 128-byte-swizzled tile (sm_100 format:
+// start >> 4 in bits 0-13, leading byte offset >> 4 in 16-29, stride byte
+// offset >> 4 in 32-45, descriptor version 1 at bit 46, swizzle mode 2
+// (128B) in bits 61-63).
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(2) << 61;
+  return d;
+}
+
+// 32 lanes x 32 consecutive fp32 columns from TMEM.
+__device__ __forceinline__ void tmem_ld_32cols(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+struct TileCoord {
+  int g, mat, tm, tn;
+};
+
+__device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
+  int g = 0;
+  while (g + 1 < p.ngroups && t >= p.g[g + 1].tile_begin) ++g;
+  const int local = t - p.g[g].tile_begin;
+  const int per_mat = p.g[g].tiles_m * p.g[g].tiles_n;
+  const int mat = local / per_mat;
+  const int r = local - mat * per_mat;
+  TileCoord c;
+  c.g = g;
+  c.mat = mat;
+  c.tm = r / p.g[g].tiles_n;
+  c.tn = r - c.tm * p.g[g].tiles_n;
+  return c;
+}
+
+__device__ __forceinline__ uint32_t pack_half2(float a, float b, int fp16) {
+  if (fp16) {
+    __half2 h = __floats2half2_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&h);
+  }
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+__device__ __forceinline__ uint16_t to_half_bits(float a, int fp16) {
+  if (fp16) {
+    __half h = __float2half_rn(a);
+    return *reinterpret_cast<uint16_t*>(&h);
+  }
+  __nv_bfloat16 h = __float2bfloat16_rn(a);
+  return *reinterpret_cast<uint16_t*>(&h);
+}
+
+// Store 32 consecutive values of one row as 16-bit (vectorised when whole).
+__device__ __forceinline__ void store_row_half(uint16_t* dst, const float* v, int valid, int fp16) {
+  if (valid >= 32) {
+    uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint4 w;
+      w.x = pack_half2(v[8 * q + 0], v[8 * q + 1], fp16);
+      w.y = pack_half2(v[8 * q + 2], v[8 * q + 3], fp16);
+      w.z = pack_half2(v[8 * q + 4], v[8 * q + 5], fp16);
+      w.w = pack_half2(v[8 * q + 6], v[8 * q + 7], fp16);
+      d4[q] = w;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < valid) dst[j] = to_half_bits(v[j], fp16);
+  }
+}
+__device__ __forceinline__ void store_row_f32(float* dst, const float* v, int valid) {
+  if (valid >= 32) {
+    float4* d4 = reinterpret_cast<float4*>(dst);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) d4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < valid) dst[j] = v[j];
+  }
+}
+
+__global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_constant__ GemmParams p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t bar0 = base + SMEM_BAR_OFF;
+  const uint32_t drain_bar = bar0 + 8 * (2 * STAGES + 4);
+  const uint32_t tmem_slot = bar0 + 8 * NUM_BARS;
+  volatile uint32_t* tmem_slot_ptr = reinterpret_cast<volatile uint32_t*>(gbase + SMEM_BAR_OFF + 8 * NUM_BARS);
+#define FULL_BAR(s) (bar0 + 8u * (s))
+#define EMPTY_BAR(s) (bar0 + 8u * (STAGES + (s)))
+#define TFULL_BAR(a) (bar0 + 8u * (2 * STAGES + (a)))
+#define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  int* err = p.err;
+  const uint64_t tmo = p.timeout_ns;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(FULL_BAR(s), 1);
+      mbar_init(EMPTY_BAR(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(TFULL_BAR(a), 1);
+      mbar_init(TEMPTY_BAR(a), 4);
+    }
+    mbar_init(drain_bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    for (int g = 0; g < p.ngroups; ++g) {
+      prefetch_tmap(&p.g[g].tmA);
+      prefetch_tmap(&p.g[g].tmB);
+    }
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(tmem_slot), "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot_ptr;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued_mask = 0, issued_parity = 0;  // bit s: stage s was filled / parity of its last fill
+      bool ok = true;
+      for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+        const TileCoord c = decode_tile(p, t);
+        const GemmGroup& G = p.g[c.g];
+        const int nk = (G.K + BK - 1) / BK;
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!wait_bounded(EMPTY_BAR(stage), phase ^ 1u, err, DEV_TIMEOUT_PRODUCER, tmo)) {
+            ok = false;
+            break;
+          }
+          const uint32_t sa = base + stage * STAGE_BYTES;
+          const uint32_t sb = sa + A_BYTES;
+          mbar_expect_tx(FULL_BAR(stage), STAGE_BYTES);
+          tma_load_3d(sa, &G.tmA, FULL_BAR(stage), kb * BK, c.tm * BM, c.mat);
+          if (!p.b_mn_major) {
+            tma_load_3d(sb, &G.tmB, FULL_BAR(stage), kb * BK, c.tn * BN, c.mat);
+          } else {
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j)
+              tma_load_3d(sb + j * (64 * BK * 2), &G.tmB, FULL_BAR(stage), c.tn * BN + j * 64, kb * BK, c.mat);
+          }
+          issued_mask |= 1u << stage;
+          issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      // Drain: every copy this thread issued has landed before the CTA exits.
+      for (int s = 0; s < STAGES; ++s)
+        if ((issued_mask >> s) & 1u) wait_bounded(FULL_BAR(s), (issued_parity >> s) & 1u, err, DEV_TIMEOUT_DRAIN, tmo);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- MMA issuer
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      const uint32_t b_lbo = p.b_mn_major ? (64u * BK * 2u) : 16u;
+      for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+        const TileCoord c = decode_tile(p, t);
+        const int nk = (p.g[c.g].K + BK - 1) / BK;
+        if (!wait_bounded(TEMPTY_BAR(acc), acc_phase ^ 1u, err, DEV_TIMEOUT_MMA_TMEM, tmo)) break;
+        tc_fence_after();
+        const uint32_t d = tmem_base + static_cast<uint32_t>(acc * BN);
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!wait_bounded(FULL_BAR(stage), phase, err, DEV_TIMEOUT_MMA_FULL, tmo)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = base + stage * STAGE_BYTES;
+          const uint32_t sb = sa + A_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / UK; ++k) {
+            const uint64_t adesc = smem_desc(sa + k * (UK * 2), 16u, 1024u);
+            const uint64_t bdesc = p.b_mn_major ? smem_desc(sb + k * (UK * 128), b_lbo, 1024u)
+                                                : smem_desc(sb + k * (UK * 2), 16u, 1024u);
+            tc_mma(d, adesc, bdesc, p.idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          }
+          tc_commit(EMPTY_BAR(stage));
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        tc_commit(TFULL_BAR(acc));
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1u;
+      }
+      // Drain: all MMAs issued by this thread are complete before TMEM is freed.
+      tc_commit(drain_bar);
+      wait_bounded(drain_bar, 0, err, DEV_TIMEOUT_DRAIN, tmo);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------------ epilogue
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
+      const TileCoord c = decode_tile(p, t);
+      const GemmGroup& G = p.g[c.g];
+      if (!wait_bounded_warp(TFULL_BAR(acc), acc_phase, err, DEV_TIMEOUT_EPI, tmo)) break;
+      tc_fence_after();
+      const int row = c.tm * BM + q * 32 + lane;
+      const bool row_ok = row < G.M;
+      const int nchunks = min(BN / 32, (G.N - c.tn * BN + 31) / 32);
+      for (int ch = 0; ch < nchunks; ++ch) {
+        float v[32];
+        tmem_ld_32cols(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN + ch * 32), v);
+        const int col0 = c.tn * BN + ch * 32;
+        const int valid = min(32, G.N - col0);
+        const int mode = p.mode;
+        if (row_ok) {
+        if (mode == MODE_GRAM) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] *= G.scale;
+          float* a32 = static_cast<float*>(G.out0) + c.mat * G.mstride0 + static_cast<int64_t>(row) * G.ld0 + col0;
+          uint16_t* a16 = static_cast<uint16_t*>(G.out1) + c.mat * G.mstride1 + static_cast<int64_t>(row) * G.ld1 + col0;
+          store_row_f32(a32, v, valid);
+          store_row_half(a16, v, valid, G.out_half_is_fp16);
+        } else if (mode == MODE_POLY) {
+          const float* ax = G.aux + c.mat * G.mstrideaux + static_cast<int64_t>(row) * G.ldaux + col0;
+          float av[32];
+          if (valid >= 32) {
+            const float4* a4 = reinterpret_cast<const float4*>(ax);
+#pragma unroll
+            for (int qq = 0; qq < 8; ++qq) {
+              const float4 f = __ldg(a4 + qq);
+              av[4 * qq] = f.x, av[4 * qq + 1] = f.y, av[4 * qq + 2] = f.z, av[4 * qq + 3] = f.w;
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) av[j] = j < valid ? __ldg(ax + j) : 0.f;
+          }
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const float diag = (col0 + j == row) ? p.ca : 0.f;
+            v[j] = fmaf(p.cc, v[j], fmaf(p.cb, av[j], diag));
+          }
+          uint16_t* po = static_cast<uint16_t*>(G.out0) + c.mat * G.mstride0 + static_cast<int64_t>(row) * G.ld0 + col0;
+          store_row_half(po, v, valid, G.out_half_is_fp16);
+        } else if (mode == MODE_XUPD) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] *= G.scale;
+          uint16_t* xo = static_cast<uint16_t*>(G.out0) + c.mat * G.mstride0 + static_cast<int64_t>(row) * G.ld0 + col0;
+          store_row_half(xo, v, valid, G.out_half_is_fp16);
+        } else {  // MODE_XLAST: U in the weight's layout
+          const MatInfo& mi = p.mats[G.mat_base + c.mat];
+          float* u = p.u_slab + mi.u_off;
+          if (!mi.trans) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] *= G.scale;
+            store_row_f32(u + static_cast<int64_t>(row) * mi.un + col0, v, valid);
+          } else {
+            // NS row `row` is weight column `row`; NS column j is weight row j.
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (j < valid) u[static_cast<int64_t>(col0 + j) * mi.un + row] = v[j] * G.scale;
+          }
+        }
+        }  // row_ok
+        __syncwarp();  // reconverge before the next warp-wide tcgen05.ld
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(TEMPTY_BAR(acc));
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+  }
+#undef FULL_BAR
+#undef EMPTY_BAR
+#undef TFULL_BAR
+#undef TEMPTY_BAR
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS) : "memory");
+  }
+}
+
+}  // namespace
+
+int ns_gemm_smem_bytes() { return SMEM_BYTES; }
+
+cudaError_t prepare_ns_gemm() {
+  return cudaFuncSetAttribute(ns_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+}
+
+cudaError_t launch_ns_gemm(const GemmParams& p, int grid, cudaStream_t st) {
+  ns_gemm_kernel<<<grid, NUM_THREADS, SMEM_BYTES, st>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace meq

@@ -1,0 +1,236 @@
+"""Thin ctypes binding of the MeqMuon C ABI (include/meq.h).
+
+Argument marshalling only: every step of the optimizer runs in the CUDA
+library. There is no fallback: if libmeq.so is missing or fails to load,
+importing this module raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libmeq.so")
+
+MEQ_OK = 0
+STATUS_NAMES = {
+    0: "MEQ_OK", 1: "MEQ_ERR_INVALID_ARG", 2: "MEQ_ERR_OOM", 3: "MEQ_ERR_CUDA",
+    4: "MEQ_ERR_NONFINITE", 5: "MEQ_ERR_TIMEOUT", 6: "MEQ_ERR_UNSUPPORTED",
+}
+ROW, COL = 0, 1
+
+
+class MeqShape(ctypes.Structure):
+    _fields_ = [("rows", ctypes.c_int64), ("cols", ctypes.c_int64)]
+
+
+class MeqOptions(ctypes.Structure):
+    _fields_ = [
+        ("rho", ctypes.c_float),
+        ("ns_steps", ctypes.c_int),
+        ("ns_a", ctypes.c_float),
+        ("ns_b", ctypes.c_float),
+        ("ns_c", ctypes.c_float),
+        ("nesterov", ctypes.c_int),
+        ("ns_fp16_mask", ctypes.c_uint32),
+        ("tie_atol", ctypes.c_float),
+        ("use_graph", ctypes.c_int),
+        ("workspace_limit_bytes", ctypes.c_int64),
+        ("wait_timeout_ms", ctypes.c_float),
+    ]
+
+
+EXPORTED = [
+    "meq_default_options", "meq_state_bytes", "meq_init_state", "meq_step", "meq_sync", "meq_free",
+    "meq_last_error", "meq_status_string", "meq_read_momentum", "meq_write_momentum",
+    "meq_read_ns_output", "meq_read_stats", "meq_kernels_per_step", "meq_debug_wait_selftest",
+    "meq_set_profiling", "meq_read_profile",
+]
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it with paper_2609_35701_gb300.build.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, I, F, D = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_double
+    lib.meq_default_options.argtypes = [ctypes.POINTER(MeqOptions)]
+    lib.meq_default_options.restype = None
+    lib.meq_state_bytes.argtypes = [ctypes.POINTER(MeqShape), I, ctypes.POINTER(MeqOptions),
+                                    ctypes.POINTER(ctypes.c_size_t), ctypes.POINTER(ctypes.c_size_t)]
+    lib.meq_state_bytes.restype = I
+    lib.meq_init_state.argtypes = [ctypes.POINTER(MeqShape), I, ctypes.POINTER(MeqOptions), P, ctypes.POINTER(P)]
+    lib.meq_init_state.restype = I
+    lib.meq_step.argtypes = [ctypes.POINTER(P), ctypes.POINTER(P), P, ctypes.POINTER(MeqShape), I, F, F, F, F, P]
+    lib.meq_step.restype = I
+    lib.meq_sync.argtypes = [P]
+    lib.meq_sync.restype = I
+    lib.meq_free.argtypes = [P]
+    lib.meq_free.restype = I
+    lib.meq_last_error.argtypes = [P]
+    lib.meq_last_error.restype = ctypes.c_char_p
+    lib.meq_status_string.argtypes = [I]
+    lib.meq_status_string.restype = ctypes.c_char_p
+    lib.meq_read_momentum.argtypes = [P, I, P]
+    lib.meq_read_momentum.restype = I
+    lib.meq_write_momentum.argtypes = [P, I, P]
+    lib.meq_write_momentum.restype = I
+    lib.meq_read_ns_output.argtypes = [P, I, P]
+    lib.meq_read_ns_output.restype = I
+    lib.meq_read_stats.argtypes = [P, I, P, P, ctypes.POINTER(D), ctypes.POINTER(D), ctypes.POINTER(I)]
+    lib.meq_read_stats.restype = I
+    lib.meq_kernels_per_step.argtypes = [P]
+    lib.meq_kernels_per_step.restype = I
+    lib.meq_debug_wait_selftest.argtypes = [P, F]
+    lib.meq_debug_wait_selftest.restype = I
+    lib.meq_set_profiling.argtypes = [P, I]
+    lib.meq_set_profiling.restype = I
+    lib.meq_read_profile.argtypes = [P, P, ctypes.POINTER(ctypes.c_int64)]
+    lib.meq_read_profile.restype = I
+    return lib
+
+
+lib = _load()
+
+
+class MeqError(RuntimeError):
+    def __init__(self, status, msg):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {msg}")
+        self.status = status
+
+
+def default_options(**overrides):
+    o = MeqOptions()
+    lib.meq_default_options(ctypes.byref(o))
+    for k, v in overrides.items():
+        if not hasattr(o, k):
+            raise KeyError(k)
+        setattr(o, k, v)
+    return o
+
+
+def _shape_array(shapes):
+    arr = (MeqShape * len(shapes))()
+    for i, (r, c) in enumerate(shapes):
+        arr[i].rows, arr[i].cols = int(r), int(c)
+    return arr
+
+
+def state_bytes(shapes, **opts):
+    """(persistent, workspace) bytes for a shape list, computed on the host."""
+    p, w = ctypes.c_size_t(), ctypes.c_size_t()
+    o = default_options(**opts)
+    st = lib.meq_state_bytes(_shape_array(shapes), len(shapes), ctypes.byref(o), ctypes.byref(p), ctypes.byref(w))
+    if st != MEQ_OK:
+        raise MeqError(st, lib.meq_last_error(None).decode())
+    return p.value, w.value
+
+
+def _stream_handle(stream):
+    if stream is None:
+        import torch
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+class MeqMuon:
+    """MeqMuon state for a fixed list of 2D hidden weights (rows, cols)."""
+
+    def __init__(self, shapes, stream=None, **opts):
+        self.shapes = [(int(r), int(c)) for r, c in shapes]
+        self._shape_arr = _shape_array(self.shapes)
+        self._opts = default_options(**opts)
+        self._st = ctypes.c_void_p()
+        s = lib.meq_init_state(self._shape_arr, len(self.shapes), ctypes.byref(self._opts), _stream_handle(stream),
+                               ctypes.byref(self._st))
+        if s != MEQ_OK:
+            raise MeqError(s, lib.meq_last_error(None).decode())
+        n = len(self.shapes)
+        self._pp = (ctypes.c_void_p * n)()
+        self._gp = (ctypes.c_void_p * n)()
+
+    def _check(self, s):
+        if s != MEQ_OK:
+            raise MeqError(s, lib.meq_last_error(self._st).decode())
+
+    @property
+    def kernels_per_step(self):
+        return lib.meq_kernels_per_step(self._st)
+
+    def step_ptrs(self, param_ptrs, grad_ptrs, lr, momentum, weight_decay, eps=1e-7, stream=None):
+        """One step given raw device pointers (ints)."""
+        for i, (p, g) in enumerate(zip(param_ptrs, grad_ptrs)):
+            self._pp[i] = p
+            self._gp[i] = g
+        self._check(lib.meq_step(self._pp, self._gp, self._st, self._shape_arr, len(self.shapes), float(lr),
+                                 float(momentum), float(weight_decay), float(eps), _stream_handle(stream)))
+
+    def step(self, params, grads, lr, momentum, weight_decay, eps=1e-7, stream=None):
+        """One step on lists of contiguous fp32 CUDA tensors (params updated in place)."""
+        if len(params) != len(self.shapes) or len(grads) != len(self.shapes):
+            raise ValueError("params / grads must have one tensor per matrix")
+        for t in list(params) + list(grads):
+            if not t.is_cuda or t.dtype.itemsize != 4 or not t.is_contiguous():
+                raise ValueError("params and grads must be contiguous fp32 CUDA tensors")
+        self.step_ptrs([p.data_ptr() for p in params], [g.data_ptr() for g in grads], lr, momentum, weight_decay,
+                       eps, stream)
+
+    def sync(self):
+        self._check(lib.meq_sync(self._st))
+
+    def read_momentum(self, i):
+        r, c = self.shapes[i]
+        out = np.empty((r, c), np.float32)
+        self._check(lib.meq_read_momentum(self._st, i, out.ctypes.data))
+        return out
+
+    def write_momentum(self, i, arr):
+        r, c = self.shapes[i]
+        a = np.ascontiguousarray(arr, dtype=np.float32)
+        assert a.shape == (r, c)
+        self._check(lib.meq_write_momentum(self._st, i, a.ctypes.data))
+
+    def read_ns_output(self, i):
+        r, c = self.shapes[i]
+        out = np.empty((r, c), np.float32)
+        self._check(lib.meq_read_ns_output(self._st, i, out.ctypes.data))
+        return out
+
+    def read_stats(self, i):
+        r, c = self.shapes[i]
+        rv = np.empty(r, np.float32)
+        cv = np.empty(c, np.float32)
+        gr, gc, d = ctypes.c_double(), ctypes.c_double(), ctypes.c_int()
+        self._check(lib.meq_read_stats(self._st, i, rv.ctypes.data, cv.ctypes.data, ctypes.byref(gr),
+                                       ctypes.byref(gc), ctypes.byref(d)))
+        return {"r": rv, "c": cv, "gamma_r": gr.value, "gamma_c": gc.value, "direction": d.value}
+
+    def set_profiling(self, enable):
+        self._check(lib.meq_set_profiling(self._st, int(bool(enable))))
+
+    PHASES = ("momentum", "cast_x0", "ns_gemm", "stats", "apply")
+
+    def read_profile(self):
+        """Summed per-phase milliseconds and the number of profiled steps."""
+        ms = (ctypes.c_double * 5)()
+        n = ctypes.c_int64()
+        self._check(lib.meq_read_profile(self._st, ms, ctypes.byref(n)))
+        return dict(zip(self.PHASES, list(ms))), n.value
+
+    def wait_selftest(self, timeout_ms=200.0):
+        """Returns the status of the bounded-wait self test (expected MEQ_ERR_TIMEOUT)."""
+        return lib.meq_debug_wait_selftest(self._st, float(timeout_ms))
+
+    def close(self):
+        if self._st:
+            lib.meq_free(self._st)
+            self._st = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,74 @@
+"""The C-ABI library builds, loads and exports every declared symbol; host-only
+entry points work without a GPU (no compute calls here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import oracle_pins as P
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_35701_gb300 import build
+
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def declared_symbols():
+    with open(os.path.join(ROOT, "include", "meq.h")) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(meq_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_symbols()
+    assert len(names) >= 14
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_binding_covers_the_header():
+    from paper_2609_35701_gb300 import meq
+
+    assert sorted(meq.EXPORTED) == declared_symbols()
+
+
+def test_default_options_are_the_papers():
+    from paper_2609_35701_gb300 import meq
+
+    o = meq.default_options()
+    g = P.golden()
+    assert abs(o.ns_a - g["ns"]["a"]) < 1e-6 and abs(o.ns_b - g["ns"]["b"]) < 1e-6 and abs(o.ns_c - g["ns"]["c"]) < 1e-6
+    assert o.ns_steps == g["ns"]["steps"] and abs(o.rho - g["rho"]) < 1e-7
+    assert o.nesterov == 0 and o.use_graph == 1
+
+
+def test_state_holds_momentum_only():
+    """Section 4 'Memory overhead': MeqMuon keeps one fp32 momentum value per
+    element of the hidden weights (no second moment, no per-row state)."""
+    from paper_2609_35701_gb300 import meq, workloads as W
+
+    g = P.golden()["architecture"]
+    for wl, arch in (("llama130m", "Llama-130M"), ("llama350m", "Llama-350M")):
+        shapes = [(r, c) for _, r, c in W.get_workload(wl).shapes]
+        persistent, workspace = meq.state_bytes(shapes)
+        Nh, _ = P.llama_hidden_counts(g[arch])
+        assert persistent == 4 * Nh
+        assert workspace > 0
+
+
+def test_host_validation_errors():
+    from paper_2609_35701_gb300 import meq
+
+    for bad in ([], [(0, 4)], [(3, -1)], [(1 << 21, 2)]):
+        with pytest.raises(meq.MeqError) as e:
+            meq.state_bytes(bad)
+        assert e.value.status == 1
+    with pytest.raises(meq.MeqError):
+        meq.state_bytes([(4, 4)], ns_steps=0)
