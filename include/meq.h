@@ -146,6 +146,37 @@ meq_status meq_read_profile(meq_state* st, double* phase_ms /* 5 */, int64_t* st
  * counterpart; this exists to test error reporting without faulting a GPU. */
 meq_status meq_debug_wait_selftest(meq_state* st, float timeout_ms);
 
+/* ---- allocation-free statistics ------------------------------------------
+ * The paper has no counterpart to this entry point; it exists for callers
+ * that cannot call cudaMalloc (code running inside a framework that owns all
+ * device memory through its own pool, or a latency-critical path that must
+ * not allocate after start-up, since cudaMalloc may synchronise the device).
+ *
+ * meq_row_col_stats_noalloc computes, for one fp32 row-major matrix U
+ * (rows x cols, device memory, read only), the statistics step of the
+ * optimizer: r (rows floats) and c (cols floats) of Eq. (7), gammas[0] =
+ * gamma_r and gammas[1] = gamma_c of Eq. (8) over entries > eps, and
+ * *direction of Eq. (11) (0 = row, 1 = column; row when gamma_r >= gamma_c -
+ * tie_atol). All outputs are caller-provided device memory. The arithmetic is
+ * that of meq_step's statistics kernels, so results agree with
+ * meq_read_stats for the same U.
+ *
+ * It allocates nothing. Its scratch is a fixed 8 MiB __device__ array inside
+ * the library, held by every GPU that loads the library until the process
+ * exits. A matrix fits when rows + ceil(rows / 32) * cols <= 2,097,152 (e.g.
+ * 4096 x 11008 and 11008 x 4096); larger ones, NULL pointers or
+ * non-positive sizes return MEQ_ERR_INVALID_ARG before anything is enqueued.
+ * The first call on a device looks up the array's device address (once per
+ * device, with that device current); make that first call before any CUDA
+ * stream capture. Every call shares the one array and overwrites all of the
+ * scratch it reads, so nothing needs clearing between calls, but calls whose
+ * kernels overlap on the GPU (different streams without ordering) race on
+ * it. Work is enqueued on cuda_stream (cudaStream_t, NULL = legacy stream);
+ * MEQ_ERR_CUDA reports a failed launch or address lookup. */
+meq_status meq_row_col_stats_noalloc(const float* U, int64_t rows, int64_t cols, float eps,
+                                     float tie_atol, float* r, float* c, double* gammas,
+                                     int* direction, void* cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1,6 +1,6 @@
 """Builds the in-tree CUDA library libmeq.so for sm_103a (GB300).
 
-The three translation units are compiled in parallel with nvcc and linked
+The translation units are compiled in parallel with nvcc and linked
 into one shared object next to this file. A rebuild happens only when a
 source or header is newer than the library.
 """
@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libmeq.so")
-SOURCES = ["ns_gemm.cu", "elementwise.cu", "meq_api.cu"]
+SOURCES = ["ns_gemm.cu", "elementwise.cu", "meq_api.cu", "noalloc.cu"]
 HEADERS = ["meq_internal.cuh", "meq_elementwise.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + INCLUDE]

@@ -1,0 +1,181 @@
+// Row / column statistics of one matrix without any device allocation.
+//
+// Some callers cannot call cudaMalloc: code that runs inside a framework
+// which owns all device memory through its own pool and forbids outside
+// allocations, and latency-critical paths that must not allocate after
+// start-up (cudaMalloc may synchronise the whole device). For them this file
+// provides meq_row_col_stats_noalloc(), the statistics step of the optimizer
+// (row / column RMS, their coefficients of variation and the chosen
+// normalisation side) for one caller-provided matrix. Its scratch lives in a
+// file-scope __device__ array of fixed size that every GPU which loads the
+// library holds until the process exits.
+//
+// The arithmetic (32-row slabs, per-slab column partial sums, warp
+// transpose-reduction of row sums, fp64 CVs) is the same as the statistics
+// kernels of the full step, so results agree with meq_read_stats.
+#include <mutex>
+
+#include "../../include/meq.h"
+#include "meq_elementwise.cuh"
+
+namespace {
+
+constexpr int kNaThreads = 256;
+constexpr int kNaSlab = 32;
+constexpr int kNaFinThreads = 1024;
+constexpr int kMaxDevices = 64;
+
+// 8 MiB of scratch: row sums of squares (rows floats) followed by the column
+// partial sums (ceil(rows / 32) x cols floats).
+constexpr long long kScratchFloats = 2ll * 1024 * 1024;
+static __device__ __align__(256) float g_stats_scratch[kScratchFloats];
+
+std::mutex g_setup_mu;
+float* g_scratch_addr[kMaxDevices] = {nullptr};
+
+__device__ __forceinline__ double na_block_sum_f64(double v, double* sh) {
+  const unsigned FULL = 0xffffffffu;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL, v, o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) sh[w] = v;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double r = 0.0;
+    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) r += sh[i];
+    sh[0] = r;
+  }
+  __syncthreads();
+  return sh[0];
+}
+
+// One block per 32-row slab: column partial sums of squares for the slab and
+// the slab's row sums of squares.
+__global__ void __launch_bounds__(kNaThreads) na_stats_kernel(const float* __restrict__ U, int64_t m, int64_t n,
+                                                              float* __restrict__ scratch) {
+  __shared__ float shr[kNaThreads / 32][32];
+  const int64_t slab = blockIdx.x;
+  const int64_t r0 = slab * kNaSlab;
+  const int nr = static_cast<int>(m - r0 < kNaSlab ? m - r0 : kNaSlab);
+  const float* Us = U + r0 * n;
+  float* rowss = scratch;
+  float* cp = scratch + m + slab * n;
+  float racc[kNaSlab];
+#pragma unroll
+  for (int r = 0; r < kNaSlab; ++r) racc[r] = 0.f;
+  for (int64_t c = threadIdx.x; c < n; c += kNaThreads) {
+    float cacc = 0.f;
+#pragma unroll
+    for (int r = 0; r < kNaSlab; ++r) {
+      if (r < nr) {
+        const float u = Us[r * n + c];
+        const float u2 = u * u;
+        cacc += u2;
+        racc[r] += u2;
+      }
+    }
+    cp[c] = cacc;
+  }
+  const unsigned FULL = 0xffffffffu;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const bool up = (lane & o) != 0;
+      const float send = up ? racc[i] : racc[i + o];
+      const float keep = up ? racc[i + o] : racc[i];
+      racc[i] = keep + __shfl_xor_sync(FULL, send, o);
+    }
+  }
+  shr[w][lane] = racc[0];
+  __syncthreads();
+  if (threadIdx.x < nr) {
+    float s = 0.f;
+    for (int i = 0; i < kNaThreads / 32; ++i) s += shr[i][threadIdx.x];
+    rowss[r0 + threadIdx.x] = s;
+  }
+}
+
+// r, c (Eq. (7)), gamma_r, gamma_c (Eq. (8), fp64) and the side (Eq. (11)).
+__global__ void __launch_bounds__(kNaFinThreads) na_finalize_kernel(int64_t m, int64_t n, float delta, float tie_atol,
+                                                                    const float* __restrict__ scratch,
+                                                                    float* __restrict__ r, float* __restrict__ c,
+                                                                    double* __restrict__ gammas,
+                                                                    int* __restrict__ direction) {
+  __shared__ double shd[32];
+  const int64_t nslabs = (m + kNaSlab - 1) / kNaSlab;
+  const float* rowss = scratch;
+  const float* cpart = scratch + m;
+  const float inv_n = 1.0f / static_cast<float>(n);
+  const float inv_m = 1.0f / static_cast<float>(m);
+  for (int64_t i = threadIdx.x; i < m; i += blockDim.x) r[i] = sqrtf(rowss[i] * inv_n);
+  for (int64_t j = threadIdx.x; j < n; j += blockDim.x) {
+    float acc = 0.f;
+    for (int64_t k = 0; k < nslabs; ++k) acc += cpart[k * n + j];
+    c[j] = sqrtf(acc * inv_m);
+  }
+  __syncthreads();
+  double gam[2];
+  for (int side = 0; side < 2; ++side) {
+    const float* v = side == 0 ? r : c;
+    const int64_t len = side == 0 ? m : n;
+    double cnt = 0.0, sum = 0.0;
+    for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
+      const float x = v[i];
+      if (x > delta) cnt += 1.0, sum += static_cast<double>(x);
+    }
+    cnt = na_block_sum_f64(cnt, shd);
+    sum = na_block_sum_f64(sum, shd);
+    const double mean = cnt > 0.0 ? sum / cnt : 0.0;
+    double var = 0.0;
+    for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
+      const double x = static_cast<double>(v[i]);
+      if (v[i] > delta) var += (x - mean) * (x - mean);
+    }
+    var = na_block_sum_f64(var, shd);
+    gam[side] = cnt > 0.0 ? sqrt(var / cnt) / mean : 0.0;
+  }
+  if (threadIdx.x == 0) {
+    gammas[0] = gam[0];
+    gammas[1] = gam[1];
+    *direction = gam[0] >= gam[1] - static_cast<double>(tie_atol) ? 0 : 1;
+  }
+}
+
+// Device address of the scratch array on the current device, looked up once
+// per device (the host-side symbol is only a stand-in, not a device address).
+meq_status scratch_address(float** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MEQ_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_setup_mu);
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_stats_scratch) != cudaSuccess || p == nullptr) return MEQ_ERR_CUDA;
+    g_scratch_addr[dev] = static_cast<float*>(p);
+  }
+  *out = g_scratch_addr[dev];
+  return MEQ_OK;
+}
+
+}  // namespace
+
+extern "C" meq_status meq_row_col_stats_noalloc(const float* U, int64_t rows, int64_t cols, float eps, float tie_atol,
+                                                float* r, float* c, double* gammas, int* direction,
+                                                void* cuda_stream) {
+  if (!U || !r || !c || !gammas || !direction) return MEQ_ERR_INVALID_ARG;
+  if (rows <= 0 || cols <= 0 || rows > (int64_t(1) << 20) || cols > (int64_t(1) << 20)) return MEQ_ERR_INVALID_ARG;
+  if (!(eps >= 0.f) || !(tie_atol >= 0.f)) return MEQ_ERR_INVALID_ARG;
+  const int64_t nslabs = (rows + kNaSlab - 1) / kNaSlab;
+  if (rows + nslabs * cols > kScratchFloats) return MEQ_ERR_INVALID_ARG;  // beyond the fixed scratch
+  float* scratch = nullptr;
+  meq_status s = scratch_address(&scratch);
+  if (s != MEQ_OK) return s;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  na_stats_kernel<<<static_cast<unsigned>(nslabs), kNaThreads, 0, st>>>(U, rows, cols, scratch);
+  if (cudaGetLastError() != cudaSuccess) return MEQ_ERR_CUDA;
+  na_finalize_kernel<<<1, kNaFinThreads, 0, st>>>(rows, cols, eps, tie_atol, scratch, r, c, gammas, direction);
+  if (cudaGetLastError() != cudaSuccess) return MEQ_ERR_CUDA;
+  return MEQ_OK;
+}

@@ -46,7 +46,7 @@ EXPORTED = [
     "meq_default_options", "meq_state_bytes", "meq_init_state", "meq_step", "meq_sync", "meq_free",
     "meq_last_error", "meq_status_string", "meq_read_momentum", "meq_write_momentum",
     "meq_read_ns_output", "meq_read_stats", "meq_kernels_per_step", "meq_debug_wait_selftest",
-    "meq_set_profiling", "meq_read_profile",
+    "meq_set_profiling", "meq_read_profile", "meq_row_col_stats_noalloc",
 ]
 
 
@@ -88,6 +88,8 @@ def _load():
     lib.meq_set_profiling.restype = I
     lib.meq_read_profile.argtypes = [P, P, ctypes.POINTER(ctypes.c_int64)]
     lib.meq_read_profile.restype = I
+    lib.meq_row_col_stats_noalloc.argtypes = [P, ctypes.c_int64, ctypes.c_int64, F, F, P, P, P, P, P]
+    lib.meq_row_col_stats_noalloc.restype = I
     return lib
 
 
@@ -125,6 +127,17 @@ def state_bytes(shapes, **opts):
     if st != MEQ_OK:
         raise MeqError(st, lib.meq_last_error(None).decode())
     return p.value, w.value
+
+
+def row_col_stats_noalloc(U, r, c, gammas, direction, eps=1e-7, tie_atol=1e-6, stream=None):
+    """Statistics of one CUDA fp32 matrix U into caller-provided CUDA tensors
+    r (rows), c (cols), gammas (2 x float64) and direction (1 x int32),
+    without any device allocation (see include/meq.h). Returns the status."""
+    rows, cols = U.shape
+    return lib.meq_row_col_stats_noalloc(ctypes.c_void_p(U.data_ptr()), rows, cols, float(eps), float(tie_atol),
+                                         ctypes.c_void_p(r.data_ptr()), ctypes.c_void_p(c.data_ptr()),
+                                         ctypes.c_void_p(gammas.data_ptr()), ctypes.c_void_p(direction.data_ptr()),
+                                         _stream_handle(stream))
 
 
 def _stream_handle(stream):
