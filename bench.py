@@ -36,6 +36,26 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 BW_BYTES_PER_ELEM = 24  # read G, B; write B; write X_0 (2 B); read U (2 B); read + write W
 
 
+def recorded_traffic(workload):
+    """dram read + write bytes per ns_gemm launch from the committed ncu
+    summary, if the kernel source is unchanged since that capture."""
+    import hashlib
+    import re
+
+    path = os.path.join(ROOT, "profiles", f"ns_gemm_{workload}.md")
+    src = os.path.join(ROOT, "paper_2609_35701_gb300", "csrc", "ns_gemm.cu")
+    try:
+        text = open(path).read()
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        m = re.search(r"sha256 prefix `([0-9a-f]+)`", text)
+        t = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+-]+)", text)
+        if m and t and m.group(1) == sha:
+            return float(t.group(1))
+    except Exception:
+        pass
+    return None
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -356,7 +376,7 @@ def main():
                 "bound": "tensor", "kernel": "ns_gemm_kernel",
                 "achieved": ns_tflops, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                 "frac": ns_tflops / peaks["bf16_tflops"], "peak_source": f"{peak_src} bf16 dense burst (fp16 rate = bf16 rate)",
-                "traffic": None,
+                "traffic": recorded_traffic(args.workload),
                 "flops_per_launch": sym / max(n_gemm_launches, 1),
                 "avg_launch_ms": ph["ns_gemm"] / max(n_gemm_launches, 1),
                 "dense_equivalent_tflops": ns_dense_tflops,
