@@ -20,6 +20,7 @@
 #include <cstdio>
 #include <cstring>
 #include <map>
+#include <tuple>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -39,9 +40,11 @@ std::string g_init_error;  // last meq_init_state failure text
 
 struct Group {
   int64_t s = 0, l = 0, lp = 0, sp = 0, count = 0;
+  int trans = 0;           // members are tall (W = X^T)
+  int64_t m = 0, n = 0, un = 0;  // weight shape of every member, U row stride
+  int64_t u_base = 0;      // float offset of the group's U block [count][m][un]
   std::vector<int> mats;
   uint16_t* x[2] = {nullptr, nullptr};
-  float* a32 = nullptr;
   uint16_t* a16 = nullptr;
   uint16_t* p16 = nullptr;
   float alpha0 = 1.f, alpha = 1.f;
@@ -73,7 +76,6 @@ struct meq_state {
   int64_t arena_bytes = 0;
   // device views
   MatInfo* d_mats = nullptr;
-  MatInfo* d_mats_bg = nullptr;
   GroupInfo* d_groups = nullptr;
   float* d_mom = nullptr;
   float* d_u = nullptr;
@@ -147,11 +149,11 @@ float pow2_round(double x) { return static_cast<float>(std::ldexp(1.0, static_ca
 // Builds the whole plan (shapes -> groups, offsets, sizes). Allocation-free.
 void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* off_vec4, int64_t* off_cpart,
           int64_t* off_partials, int64_t* off_counters, int64_t* off_x0s, int64_t* off_stats, int64_t* off_step,
-          int64_t* off_err, int64_t* off_mats, int64_t* off_mats_bg, int64_t* off_groups,
+          int64_t* off_err, int64_t* off_mats, int64_t* off_groups,
           std::vector<int64_t>* group_offs) {
   const int n = st->n;
   st->mats.assign(n, MatInfo{});
-  std::map<std::pair<int64_t, int64_t>, int> gmap;
+  std::map<std::tuple<int64_t, int64_t, int>, int> gmap;
   st->groups.clear();
   for (int i = 0; i < n; ++i) {
     const int64_t m = st->shapes[i].rows, c = st->shapes[i].cols;
@@ -159,7 +161,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
     M.m = m, M.n = c;
     M.s = std::min(m, c), M.l = std::max(m, c);
     M.trans = m > c ? 1 : 0;
-    auto key = std::make_pair(M.s, M.l);
+    auto key = std::make_tuple(M.s, M.l, M.trans);
     auto it = gmap.find(key);
     int g;
     if (it == gmap.end()) {
@@ -167,6 +169,8 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
       gmap[key] = g;
       Group G;
       G.s = M.s, G.l = M.l;
+      G.trans = M.trans;
+      G.m = m, G.n = c, G.un = round_up(c, 4);
       G.lp = round_up(M.l, 64), G.sp = round_up(M.s, 64);
       G.alpha0 = std::min(pow2_round(std::sqrt(static_cast<double>(M.s) * static_cast<double>(M.l))), 16384.f);
       G.alpha = std::min(pow2_round(std::sqrt(static_cast<double>(M.l))), 16384.f);
@@ -179,13 +183,17 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
     st->groups[g].mats.push_back(i);
   }
   int64_t mom = 0, u = 0, vec = 0, cp = 0, chunks = 0, tiles = 0, slabs = 0;
+  for (auto& G : st->groups) {  // U is stored group by group: [count][m][un]
+    G.u_base = u;
+    u += round_up(G.count * G.m * G.un, 64);
+  }
   for (int i = 0; i < n; ++i) {
     MatInfo& M = st->mats[i];
-    M.un = round_up(M.n, 4);
+    const Group& G = st->groups[M.group];
+    M.un = G.un;
     M.mom_off = mom;
     mom += round_up(M.m * M.n, 64);
-    M.u_off = u;
-    u += round_up(M.m * M.un, 64);
+    M.u_off = G.u_base + M.gidx * M.m * M.un;
     M.vec_off = vec;
     vec += round_up(std::max(M.m, M.n), 64);
     M.chunk_begin = chunks;
@@ -215,7 +223,6 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
   *off_step = L->add(st->step_bytes);
   *off_err = L->add(64);
   *off_mats = L->add(int64_t(n) * sizeof(MatInfo));
-  *off_mats_bg = L->add(int64_t(n) * sizeof(MatInfo));
   *off_groups = L->add(int64_t(st->groups.size()) * sizeof(GroupInfo));
   group_offs->clear();
   for (auto& G : st->groups) {
@@ -223,7 +230,6 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
     const int64_t sb = G.count * G.s * G.sp;
     group_offs->push_back(L->add(xb));
     group_offs->push_back(L->add(xb));
-    group_offs->push_back(L->add(sb * 4));
     group_offs->push_back(L->add(sb * 2));
     group_offs->push_back(L->add(sb * 2));
   }
@@ -242,19 +248,28 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
-// 3D map over [count][rows][row_stride] 16-bit elements, 128-byte swizzle.
-bool encode_map(CUtensorMap* m, void* base, int64_t inner, int64_t rows, int64_t count, int64_t row_stride_elems,
-                uint32_t box_inner, uint32_t box_rows) {
+// 3D tensor map over [count][rows][row_stride] elements of 2 or 4 bytes.
+bool encode_map(CUtensorMap* m, void* base, int elem_bytes, int64_t inner, int64_t rows, int64_t count,
+                int64_t row_stride_elems, uint32_t box_inner, uint32_t box_rows, CUtensorMapSwizzle swz) {
   auto enc = get_encode();
   if (!enc) return false;
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows), static_cast<cuuint64_t>(count)};
-  cuuint64_t strides[2] = {static_cast<cuuint64_t>(row_stride_elems * 2),
-                           static_cast<cuuint64_t>(rows * row_stride_elems * 2)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(row_stride_elems * elem_bytes),
+                           static_cast<cuuint64_t>(rows * row_stride_elems * elem_bytes)};
   cuuint32_t box[3] = {box_inner, box_rows, 1};
   cuuint32_t estr[3] = {1, 1, 1};
-  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT16, 3, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                   CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  const CUtensorMapDataType dt = elem_bytes == 2 ? CU_TENSOR_MAP_DATA_TYPE_UINT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+  CUresult r = enc(m, dt, 3, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+constexpr CUtensorMapSwizzle SW64 = CU_TENSOR_MAP_SWIZZLE_64B;
+constexpr CUtensorMapSwizzle SW128 = CU_TENSOR_MAP_SWIZZLE_128B;
+
+int sym_tiles(int tiles_m, int tiles_n) {
+  int t = 0;
+  for (int tn = 0; tn < tiles_n; ++tn) t += std::min(tiles_m, 2 * (tn + 1));
+  return t;
 }
 
 // tcgen05 kind::f16 instruction descriptor: D fp32, A/B fp16 (0) or bf16 (1),
@@ -286,8 +301,6 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
         P.b_mn_major = (mode == MODE_XUPD) ? 1 : 0;
         P.idesc = make_idesc(f16, P.b_mn_major);
         P.ca = st->opt.ns_a, P.cb = st->opt.ns_b, P.cc = st->opt.ns_c;
-        P.mats = st->d_mats_bg;
-        P.u_slab = st->d_u;
         P.err = st->d_err;
         P.timeout_ns = static_cast<unsigned long long>(static_cast<double>(st->opt.wait_timeout_ms) * 1e6);
         int tiles = 0;
@@ -297,41 +310,50 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
           GemmGroup& Q = P.g[gi];
           const float ak = (k == 0) ? G.alpha0 : G.alpha;
           Q.count = static_cast<int32_t>(G.count);
-          Q.mat_base = 0;
+          Q.trans = G.trans;
           bool ok = true;
           if (mode == MODE_GRAM) {
             Q.M = (int32_t)G.s, Q.N = (int32_t)G.s, Q.K = (int32_t)G.l;
-            ok &= encode_map(&Q.tmA, G.x[cur], G.l, G.s, G.count, G.lp, 64, 128);
-            ok &= encode_map(&Q.tmB, G.x[cur], G.l, G.s, G.count, G.lp, 64, 256);
-            Q.out0 = G.a32, Q.ld0 = G.sp, Q.mstride0 = G.s * G.sp;
-            Q.out1 = G.a16, Q.ld1 = G.sp, Q.mstride1 = G.s * G.sp;
+            Q.sym = 1;
+            ok &= encode_map(&Q.tmA, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 128, SW128);
+            ok &= encode_map(&Q.tmB, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 256, SW128);
+            ok &= encode_map(&Q.tmOut, G.a16, 2, G.s, G.s, G.count, G.sp, 32, 32, SW64);
             Q.scale = 1.0f / (ak * ak);
-            Q.out_half_is_fp16 = f16;
+            Q.out_fp16 = f16;
           } else if (mode == MODE_POLY) {
             Q.M = (int32_t)G.s, Q.N = (int32_t)G.s, Q.K = (int32_t)G.s;
-            ok &= encode_map(&Q.tmA, G.a16, G.s, G.s, G.count, G.sp, 64, 128);
-            ok &= encode_map(&Q.tmB, G.a16, G.s, G.s, G.count, G.sp, 64, 256);
-            Q.out0 = G.p16, Q.ld0 = G.sp, Q.mstride0 = G.s * G.sp;
-            Q.aux = G.a32, Q.ldaux = G.sp, Q.mstrideaux = G.s * G.sp;
-            Q.out_half_is_fp16 = f16;
+            Q.sym = 1;
+            ok &= encode_map(&Q.tmA, G.a16, 2, G.s, G.s, G.count, G.sp, 64, 128, SW128);
+            ok &= encode_map(&Q.tmB, G.a16, 2, G.s, G.s, G.count, G.sp, 64, 256, SW128);
+            ok &= encode_map(&Q.tmOut, G.p16, 2, G.s, G.s, G.count, G.sp, 32, 32, SW64);
+            ok &= encode_map(&Q.tmAux, G.a16, 2, G.s, G.s, G.count, G.sp, 32, 32, SW64);
+            Q.scale = 1.0f;
+            Q.out_fp16 = f16;
           } else {
             Q.M = (int32_t)G.s, Q.N = (int32_t)G.l, Q.K = (int32_t)G.s;
-            ok &= encode_map(&Q.tmA, G.p16, G.s, G.s, G.count, G.sp, 64, 128);
-            ok &= encode_map(&Q.tmB, G.x[cur], G.l, G.s, G.count, G.lp, 64, 64);
+            Q.sym = 0;
+            ok &= encode_map(&Q.tmA, G.p16, 2, G.s, G.s, G.count, G.sp, 64, 128, SW128);
+            ok &= encode_map(&Q.tmB, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 64, SW128);
             if (real_mode == MODE_XUPD) {
-              Q.out0 = G.x[nxt], Q.ld0 = G.lp, Q.mstride0 = G.s * G.lp;
+              ok &= encode_map(&Q.tmOut, G.x[nxt], 2, G.l, G.s, G.count, G.lp, 32, 32, SW64);
               Q.scale = G.alpha / ak;
-              Q.out_half_is_fp16 = next_f16;
+              Q.out_fp16 = next_f16;
             } else {
+              float* ub = st->d_u + G.u_base;
+              if (!G.trans)
+                ok &= encode_map(&Q.tmOut, ub, 4, G.n, G.m, G.count, G.un, 16, 32, SW64);
+              else
+                ok &= encode_map(&Q.tmOut, ub, 4, G.n, G.m, G.count, G.un, 32, 16, SW128);
               Q.scale = 1.0f / ak;
-              Q.mat_base = 0;
+              Q.out_fp16 = 0;
             }
           }
           if (!ok) { *why = "cuTensorMapEncodeTiled failed"; return false; }
           Q.tiles_m = (int32_t)((Q.M + 127) / 128);
           Q.tiles_n = (int32_t)((Q.N + 255) / 256);
+          Q.tiles_per_mat = Q.sym ? sym_tiles(Q.tiles_m, Q.tiles_n) : Q.tiles_m * Q.tiles_n;
           Q.tile_begin = tiles;
-          const int64_t t = int64_t(Q.tiles_m) * Q.tiles_n * Q.count;
+          const int64_t t = int64_t(Q.tiles_per_mat) * Q.count;
           if (tiles + t > (int64_t(1) << 30)) { *why = "too many GEMM tiles in one launch"; return false; }
           tiles += static_cast<int>(t);
         }
@@ -389,9 +411,9 @@ meq_status meq_state_bytes(const meq_shape* shapes, int n, const meq_options* op
   tmp.shapes.assign(shapes, shapes + n);
   tmp.opt = o;
   Layout L;
-  int64_t a[14];
+  int64_t a[13];
   std::vector<int64_t> goffs;
-  plan(&tmp, &L, &a[0], &a[1], &a[2], &a[3], &a[4], &a[5], &a[6], &a[7], &a[8], &a[9], &a[10], &a[11], &a[12], &goffs);
+  plan(&tmp, &L, &a[0], &a[1], &a[2], &a[3], &a[4], &a[5], &a[6], &a[7], &a[8], &a[9], &a[10], &a[11], &goffs);
   if (persistent) *persistent = static_cast<size_t>(tmp.persistent_bytes);
   if (workspace) *workspace = static_cast<size_t>(L.total - tmp.persistent_bytes);
   return MEQ_OK;
@@ -430,10 +452,10 @@ meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt
 
   Layout L;
   int64_t off_mom, off_u, off_vec4, off_cpart, off_partials, off_counters, off_x0s, off_stats, off_step, off_err, off_mats,
-      off_mats_bg, off_groups;
+      off_groups;
   std::vector<int64_t> goffs;
   plan(st, &L, &off_mom, &off_u, &off_vec4, &off_cpart, &off_partials, &off_counters, &off_x0s, &off_stats, &off_step,
-       &off_err, &off_mats, &off_mats_bg, &off_groups, &goffs);
+       &off_err, &off_mats, &off_groups, &goffs);
   if (o.workspace_limit_bytes > 0 && L.total > o.workspace_limit_bytes) {
     delete st;
     return fail(nullptr, MEQ_ERR_OOM, "state needs " + std::to_string(L.total) + " bytes, above workspace_limit_bytes");
@@ -461,24 +483,13 @@ meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt
   st->d_err = reinterpret_cast<int*>(A + off_err);
   st->d_flag = st->d_err + 4;
   st->d_mats = reinterpret_cast<MatInfo*>(A + off_mats);
-  st->d_mats_bg = reinterpret_cast<MatInfo*>(A + off_mats_bg);
   st->d_groups = reinterpret_cast<GroupInfo*>(A + off_groups);
   for (size_t g = 0; g < st->groups.size(); ++g) {
     Group& G = st->groups[g];
-    G.x[0] = reinterpret_cast<uint16_t*>(A + goffs[5 * g + 0]);
-    G.x[1] = reinterpret_cast<uint16_t*>(A + goffs[5 * g + 1]);
-    G.a32 = reinterpret_cast<float*>(A + goffs[5 * g + 2]);
-    G.a16 = reinterpret_cast<uint16_t*>(A + goffs[5 * g + 3]);
-    G.p16 = reinterpret_cast<uint16_t*>(A + goffs[5 * g + 4]);
-  }
-
-  // MODE_XLAST reads mats_bg[mat_base + index in group]: a copy of the
-  // per-matrix table ordered group by group.
-  std::vector<MatInfo> by_group;
-  std::vector<int> group_base(st->groups.size(), 0);
-  for (size_t g = 0; g < st->groups.size(); ++g) {
-    group_base[g] = static_cast<int>(by_group.size());
-    for (int i : st->groups[g].mats) by_group.push_back(st->mats[i]);
+    G.x[0] = reinterpret_cast<uint16_t*>(A + goffs[4 * g + 0]);
+    G.x[1] = reinterpret_cast<uint16_t*>(A + goffs[4 * g + 1]);
+    G.a16 = reinterpret_cast<uint16_t*>(A + goffs[4 * g + 2]);
+    G.p16 = reinterpret_cast<uint16_t*>(A + goffs[4 * g + 3]);
   }
 
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
@@ -492,8 +503,6 @@ meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt
   bool ok = cudaMemsetAsync(st->arena, 0, static_cast<size_t>(L.total), s) == cudaSuccess;
   ok = ok && cudaMemcpyAsync(st->d_mats, st->mats.data(), sizeof(MatInfo) * n, cudaMemcpyHostToDevice, s) == cudaSuccess;
   ok = ok && cudaMemcpyAsync(st->d_groups, gi.data(), sizeof(GroupInfo) * gi.size(), cudaMemcpyHostToDevice, s) == cudaSuccess;
-  ok = ok && cudaMemcpyAsync(st->d_mats_bg, by_group.data(), sizeof(MatInfo) * by_group.size(), cudaMemcpyHostToDevice, s) ==
-                 cudaSuccess;
   ok = ok && cudaStreamSynchronize(s) == cudaSuccess;
   if (!ok) {
     cudaError_t ee = cudaGetLastError();
@@ -507,16 +516,6 @@ meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt
     delete st;
     return fail(nullptr, MEQ_ERR_UNSUPPORTED, why);
   }
-  // Each launch slot covers groups g0 .. g0 + ngroups - 1, in build order.
-  {
-    const int ng = static_cast<int>(st->groups.size());
-    size_t li = 0;
-    for (int k = 0; k < o.ns_steps; ++k)
-      for (int mode = MODE_GRAM; mode <= MODE_XUPD; ++mode)
-        for (int g0 = 0; g0 < ng; g0 += kMaxGroups, ++li)
-          for (int gi2 = 0; gi2 < st->gemm[li].ngroups; ++gi2) st->gemm[li].g[gi2].mat_base = group_base[g0 + gi2];
-  }
-
   LaunchCtx& C = st->ctx;
   C.mats = st->d_mats;
   C.nmat = n;

@@ -62,18 +62,17 @@ enum GemmMode : int { MODE_GRAM = 0, MODE_POLY = 1, MODE_XUPD = 2, MODE_XLAST = 
 struct GemmGroup {
   CUtensorMap tmA;        // A operand (K-major), box {64, 128, 1}
   CUtensorMap tmB;        // B operand: K-major box {64, 256, 1} or MN-major box {64, 64, 1}
+  CUtensorMap tmOut;      // epilogue TMA store: 16-bit {32, 32, 1}; U fp32 {16, 32, 1} or {32, 16, 1}
+  CUtensorMap tmAux;      // POLY: 16-bit A, box {32, 32, 1}, loaded by the epilogue
   int32_t M, N, K;        // output rows, output cols, contraction
   int32_t count;          // matrices in the group
   int32_t tiles_m, tiles_n;
+  int32_t tiles_per_mat;  // tiles_m * tiles_n, or the upper-triangle count when sym
   int32_t tile_begin;     // first tile of this group in the launch
-  int32_t mat_base;       // global index of the group's first matrix (XLAST)
-  void* out0;             // GRAM: fp32 A; POLY: 16-bit P; XUPD: 16-bit X next
-  void* out1;             // GRAM: 16-bit A
-  const float* aux;       // POLY: fp32 A
-  int64_t ld0, ld1, ldaux;          // row strides (elements)
-  int64_t mstride0, mstride1, mstrideaux;  // matrix strides (elements)
+  int32_t sym;            // 1: symmetric s x s output (upper-triangle tiles, mirrored stores)
+  int32_t trans;          // XLAST: 1 when the weight is the transpose of the NS layout
   float scale;            // GRAM: 1/alpha^2; XUPD: alpha_next/alpha; XLAST: 1/alpha
-  int32_t out_half_is_fp16;  // output 16-bit format (1 = fp16, 0 = bf16)
+  int32_t out_fp16;       // 16-bit format of the output / aux operand (1 = fp16, 0 = bf16)
 };
 
 struct GemmParams {
@@ -84,8 +83,6 @@ struct GemmParams {
   uint32_t idesc;          // tcgen05 instruction descriptor
   int32_t b_mn_major;      // 1: B operand tile is MN-major (XUPD)
   float ca, cb, cc;        // NS coefficients
-  const MatInfo* mats;     // XLAST: per-matrix info (U offsets, transposition)
-  float* u_slab;           // XLAST: U output slab
   int* err;                // device error word
   unsigned long long timeout_ns;
 };

@@ -4,13 +4,16 @@
 // quintic iteration, Eq. (5) of the paper, for a batch of same-shape groups:
 //
 //   MODE_GRAM : A   = X X^T / alpha^2           (s x s, contraction over l)
-//               epilogue writes A in fp32 and in the 16-bit operand format
 //   MODE_POLY : P   = a I + b A + c (A A)       (s x s, contraction over s)
-//               the a I + b A terms use the fp32 copy of A in the epilogue
+//               a I + b A is added in fp32 from the same 16-bit A the
+//               product uses, so P is exactly a polynomial of that matrix
 //   MODE_XUPD : X'  = P X * (alpha'/alpha)      (s x l, contraction over s)
 //   MODE_XLAST: U   = P X / alpha, written as fp32 in the weight's own layout
 //
 // P X equals a X + (b A + c A^2) X of Eq. (5) exactly in real arithmetic.
+// A and P are symmetric: their launches run only the tiles that hold a 32 x 32
+// block on or above the diagonal and store each strictly-upper block twice
+// (as is, and transposed), so every element is written from one accumulator.
 // X is stored scaled by a power of two alpha so its entries stay in the
 // normal range of fp16; the epilogues undo the scale in fp32.
 //
@@ -19,7 +22,8 @@
 //   warp 1 : TMEM allocator and tcgen05.mma issuer (one thread)
 //   warps 2-5 : epilogue; warp w reads TMEM lanes 32*(w%4) .. +31
 // Two 128x256 fp32 accumulators (512 TMEM columns) let the epilogue of one
-// tile overlap the MMAs of the next.
+// tile overlap the MMAs of the next. The epilogue stages 32 x 32 blocks in
+// swizzled shared memory and writes them with TMA bulk-tensor stores.
 //
 // Every mbarrier wait is bounded (time and iteration count). On expiry the
 // waiting role records an error code, the others see it and stop, in-flight
@@ -36,9 +40,12 @@ constexpr int B_BYTES = BN * BK * 2;                 // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;       // 48 KB
 constexpr int NUM_THREADS = 192;
 constexpr uint32_t TMEM_COLS = 512;
-constexpr int NUM_BARS = 2 * STAGES + 4 + 1;         // full, empty, tmem full x2, tmem empty x2, drain
-constexpr int SMEM_BAR_OFF = STAGES * STAGE_BYTES;
+constexpr int SLOT_BYTES = 2048;                      // one 32 x 32 16-bit block (or 32 x 16 fp32)
+constexpr int NUM_BARS = 2 * STAGES + 4 + 1 + 8;     // full, empty, tmem full x2, tmem empty x2, drain, aux 4x2
+constexpr int SMEM_EPI_OFF = STAGES * STAGE_BYTES;   // 4 epilogue warps x 4 slots
+constexpr int SMEM_BAR_OFF = SMEM_EPI_OFF + 4 * 4 * SLOT_BYTES;
 constexpr int SMEM_BYTES = SMEM_BAR_OFF + NUM_BARS * 8 + 16 + 1024;
+static_assert(SMEM_BYTES <= 232448, "shared memory budget of one sm_103a CTA");
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -168,18 +175,34 @@ struct TileCoord {
   int g, mat, tm, tn;
 };
 
+// Tiles of a group are numbered matrix by matrix. Dense outputs run tm-major
+// over tiles_m x tiles_n; symmetric outputs (Gram, polynomial) run tn-major
+// over the tiles with tm < 2 (tn + 1), i.e. those holding a 32 x 32 block on
+// or above the diagonal.
 __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
   int g = 0;
   while (g + 1 < p.ngroups && t >= p.g[g + 1].tile_begin) ++g;
-  const int local = t - p.g[g].tile_begin;
-  const int per_mat = p.g[g].tiles_m * p.g[g].tiles_n;
-  const int mat = local / per_mat;
-  const int r = local - mat * per_mat;
+  const GemmGroup& G = p.g[g];
+  const int local = t - G.tile_begin;
+  const int mat = local / G.tiles_per_mat;
+  int r = local - mat * G.tiles_per_mat;
   TileCoord c;
   c.g = g;
   c.mat = mat;
-  c.tm = r / p.g[g].tiles_n;
-  c.tn = r - c.tm * p.g[g].tiles_n;
+  if (!G.sym) {
+    c.tm = r / G.tiles_n;
+    c.tn = r - c.tm * G.tiles_n;
+  } else {
+    int tn = 0;
+    for (;;) {
+      const int cnt = min(G.tiles_m, 2 * (tn + 1));
+      if (r < cnt) break;
+      r -= cnt;
+      ++tn;
+    }
+    c.tm = r;
+    c.tn = tn;
+  }
   return c;
 }
 
@@ -199,36 +222,60 @@ __device__ __forceinline__ uint16_t to_half_bits(float a, int fp16) {
   __nv_bfloat16 h = __float2bfloat16_rn(a);
   return *reinterpret_cast<uint16_t*>(&h);
 }
+__device__ __forceinline__ float2 unpack_half2(uint32_t w, int fp16) {
+  if (fp16) {
+    __half2 h = *reinterpret_cast<__half2*>(&w);
+    return __half22float2(h);
+  }
+  __nv_bfloat162 h = *reinterpret_cast<__nv_bfloat162*>(&w);
+  return __bfloat1622float2(h);
+}
 
-// Store 32 consecutive values of one row as 16-bit (vectorised when whole).
-__device__ __forceinline__ void store_row_half(uint16_t* dst, const float* v, int valid, int fp16) {
-  if (valid >= 32) {
-    uint4* d4 = reinterpret_cast<uint4*>(dst);
+// ---- TMA store / bulk-group helpers (issued by one lane) ----------------------
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* tm, uint32_t src, int x, int y, int z) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(tm)),
+               "r"(src), "r"(x), "r"(y), "r"(z)
+               : "memory");
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// Row-major 32 x 32 16-bit block, 64-byte rows, 64B swizzle (16-byte chunk k
+// of row r sits at chunk k ^ ((r >> 1) & 3)).
+__device__ __forceinline__ void fill_half_rows(uint8_t* slot, int r, const float* v, int fp16) {
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      uint4 w;
-      w.x = pack_half2(v[8 * q + 0], v[8 * q + 1], fp16);
-      w.y = pack_half2(v[8 * q + 2], v[8 * q + 3], fp16);
-      w.z = pack_half2(v[8 * q + 4], v[8 * q + 5], fp16);
-      w.w = pack_half2(v[8 * q + 6], v[8 * q + 7], fp16);
-      d4[q] = w;
-    }
-  } else {
-#pragma unroll
-    for (int j = 0; j < 32; ++j)
-      if (j < valid) dst[j] = to_half_bits(v[j], fp16);
+  for (int k = 0; k < 4; ++k) {
+    uint4 w;
+    w.x = pack_half2(v[8 * k + 0], v[8 * k + 1], fp16);
+    w.y = pack_half2(v[8 * k + 2], v[8 * k + 3], fp16);
+    w.z = pack_half2(v[8 * k + 4], v[8 * k + 5], fp16);
+    w.w = pack_half2(v[8 * k + 6], v[8 * k + 7], fp16);
+    *reinterpret_cast<uint4*>(slot + r * 64 + ((k ^ ((r >> 1) & 3)) << 4)) = w;
   }
 }
-__device__ __forceinline__ void store_row_f32(float* dst, const float* v, int valid) {
-  if (valid >= 32) {
-    float4* d4 = reinterpret_cast<float4*>(dst);
+// The transposed block: element (row j, col r) = v[j] of lane r.
+__device__ __forceinline__ void fill_half_cols(uint8_t* slot, int r, const float* v, int fp16) {
 #pragma unroll
-    for (int q = 0; q < 8; ++q) d4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-  } else {
-#pragma unroll
-    for (int j = 0; j < 32; ++j)
-      if (j < valid) dst[j] = v[j];
+  for (int j = 0; j < 32; ++j) {
+    const int off = j * 64 + ((((r >> 3) ^ ((j >> 1) & 3))) << 4) + ((r & 7) << 1);
+    *reinterpret_cast<uint16_t*>(slot + off) = to_half_bits(v[j], fp16);
   }
+}
+// fp32 16-column half of a row, 64-byte rows, 64B swizzle.
+__device__ __forceinline__ void fill_f32_rows16(uint8_t* slot, int r, const float* v) {
+#pragma unroll
+  for (int k = 0; k < 4; ++k)
+    *reinterpret_cast<float4*>(slot + r * 64 + ((k ^ ((r >> 1) & 3)) << 4)) =
+        make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+}
+// fp32 transposed: 16 rows (j) x 32 columns (r), 128-byte rows, 128B swizzle.
+__device__ __forceinline__ void fill_f32_cols16(uint8_t* slot, int r, const float* v) {
+#pragma unroll
+  for (int j = 0; j < 16; ++j)
+    *reinterpret_cast<float*>(slot + j * 128 + ((((r >> 2) ^ (j & 7))) << 4) + ((r & 3) << 2)) = v[j];
 }
 
 __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_constant__ GemmParams p) {
@@ -244,6 +291,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
 #define EMPTY_BAR(s) (bar0 + 8u * (STAGES + (s)))
 #define TFULL_BAR(a) (bar0 + 8u * (2 * STAGES + (a)))
 #define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
+#define AUX_BAR(w, b) (bar0 + 8u * (2 * STAGES + 5 + 2 * (w) + (b)))
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -260,10 +308,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       mbar_init(TEMPTY_BAR(a), 4);
     }
     mbar_init(drain_bar, 1);
+    for (int w = 0; w < 4; ++w)
+      for (int b = 0; b < 2; ++b) mbar_init(AUX_BAR(w, b), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     for (int g = 0; g < p.ngroups; ++g) {
       prefetch_tmap(&p.g[g].tmA);
       prefetch_tmap(&p.g[g].tmB);
+      prefetch_tmap(&p.g[g].tmOut);
+      if (p.mode == MODE_POLY) prefetch_tmap(&p.g[g].tmAux);
     }
   }
   if (warp == 1) {
@@ -364,72 +416,112 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     __syncwarp();
   } else {
     // ------------------------------------------------------------------ epilogue
-    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    // Warp ew (0..3) owns TMEM lanes 32*q .. +31 (q = warp % 4), i.e. rows
+    // 32q .. 32q+31 of the tile, and four 2 KB shared-memory slots: two output
+    // staging slots used in turn (a TMA store drains one while the other is
+    // filled) and two slots the polynomial epilogue TMA-loads A chunks into.
+    const int q = warp & 3;
+    const int ew = warp - 2;
+    uint8_t* slots = gbase + SMEM_EPI_OFF + ew * (4 * SLOT_BYTES);
+    const uint32_t slots_s = base + SMEM_EPI_OFF + ew * (4 * SLOT_BYTES);
+    const int mode = p.mode;
+    int out_slot = 0;
+    uint32_t aux_phase = 0;    // bit b: parity of the next completion of aux slot b
+    uint32_t aux_pending = 0;  // bit b: aux slot b has a load in flight
+    bool ok = true;
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
+
+    auto next_out_slot = [&]() -> uint32_t {
+      // The slot used two stores ago must have been read by its TMA store.
+      if (lane == 0) bulk_wait_read_1();
+      __syncwarp();
+      const uint32_t s = static_cast<uint32_t>(out_slot);
+      out_slot ^= 1;
+      return s;
+    };
+    auto issue_aux = [&](const GemmGroup& G, int b, int col0, int row0, int mat) {
+      if (lane == 0) {
+        mbar_expect_tx(AUX_BAR(ew, b), SLOT_BYTES);
+        tma_load_3d(slots_s + (2 + b) * SLOT_BYTES, &G.tmAux, AUX_BAR(ew, b), col0, row0, mat);
+      }
+      aux_pending |= 1u << b;
+    };
+
+    for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
       const TileCoord c = decode_tile(p, t);
       const GemmGroup& G = p.g[c.g];
       if (!wait_bounded_warp(TFULL_BAR(acc), acc_phase, err, DEV_TIMEOUT_EPI, tmo)) break;
       tc_fence_after();
-      const int row = c.tm * BM + q * 32 + lane;
-      const bool row_ok = row < G.M;
-      const int nchunks = min(BN / 32, (G.N - c.tn * BN + 31) / 32);
-      for (int ch = 0; ch < nchunks; ++ch) {
+      const int row0 = c.tm * BM + q * 32;
+      const int R = c.tm * 4 + q;  // 32-row block index
+      const int nch = min(BN / 32, (G.N - c.tn * BN + 31) / 32);
+      int ch0 = G.sym ? max(0, R - c.tn * 8) : 0;  // blocks strictly below the diagonal come from mirrors
+      if (row0 >= G.M) ch0 = nch;
+      if (mode == MODE_POLY && ch0 < nch) issue_aux(G, ch0 & 1, c.tn * BN + ch0 * 32, row0, c.mat);
+      for (int ch = ch0; ch < nch; ++ch) {
+        const int col0 = c.tn * BN + ch * 32;
+        const int C = c.tn * 8 + ch;
+        if (mode == MODE_POLY && ch + 1 < nch) issue_aux(G, (ch + 1) & 1, col0 + 32, row0, c.mat);
         float v[32];
         tmem_ld_32cols(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN + ch * 32), v);
-        const int col0 = c.tn * BN + ch * 32;
-        const int valid = min(32, G.N - col0);
-        const int mode = p.mode;
-        if (row_ok) {
-        if (mode == MODE_GRAM) {
+        if (mode == MODE_POLY) {
+          const int b = ch & 1;
+          if (!wait_bounded_warp(AUX_BAR(ew, b), (aux_phase >> b) & 1u, err, DEV_TIMEOUT_EPI, tmo)) {
+            ok = false;
+            break;
+          }
+          aux_phase ^= 1u << b;
+          aux_pending &= ~(1u << b);
+          const uint8_t* as = slots + (2 + b) * SLOT_BYTES;
+          const int row = row0 + lane;
 #pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] *= G.scale;
-          float* a32 = static_cast<float*>(G.out0) + c.mat * G.mstride0 + static_cast<int64_t>(row) * G.ld0 + col0;
-          uint16_t* a16 = static_cast<uint16_t*>(G.out1) + c.mat * G.mstride1 + static_cast<int64_t>(row) * G.ld1 + col0;
-          store_row_f32(a32, v, valid);
-          store_row_half(a16, v, valid, G.out_half_is_fp16);
-        } else if (mode == MODE_POLY) {
-          const float* ax = G.aux + c.mat * G.mstrideaux + static_cast<int64_t>(row) * G.ldaux + col0;
-          float av[32];
-          if (valid >= 32) {
-            const float4* a4 = reinterpret_cast<const float4*>(ax);
+          for (int k = 0; k < 4; ++k) {
+            const uint4 w = *reinterpret_cast<const uint4*>(as + lane * 64 + ((k ^ ((lane >> 1) & 3)) << 4));
+            const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-            for (int qq = 0; qq < 8; ++qq) {
-              const float4 f = __ldg(a4 + qq);
-              av[4 * qq] = f.x, av[4 * qq + 1] = f.y, av[4 * qq + 2] = f.z, av[4 * qq + 3] = f.w;
+            for (int h = 0; h < 4; ++h) {
+              const float2 a2 = unpack_half2(ws[h], G.out_fp16);
+              const int j = 8 * k + 2 * h;
+              v[j] = fmaf(p.cc, v[j], fmaf(p.cb, a2.x, (col0 + j == row) ? p.ca : 0.f));
+              v[j + 1] = fmaf(p.cc, v[j + 1], fmaf(p.cb, a2.y, (col0 + j + 1 == row) ? p.ca : 0.f));
             }
-          } else {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) av[j] = j < valid ? __ldg(ax + j) : 0.f;
           }
-#pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const float diag = (col0 + j == row) ? p.ca : 0.f;
-            v[j] = fmaf(p.cc, v[j], fmaf(p.cb, av[j], diag));
-          }
-          uint16_t* po = static_cast<uint16_t*>(G.out0) + c.mat * G.mstride0 + static_cast<int64_t>(row) * G.ld0 + col0;
-          store_row_half(po, v, valid, G.out_half_is_fp16);
-        } else if (mode == MODE_XUPD) {
+          fence_async_smem();  // generic reads of the aux slot before its next TMA fill
+        } else {
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] *= G.scale;
-          uint16_t* xo = static_cast<uint16_t*>(G.out0) + c.mat * G.mstride0 + static_cast<int64_t>(row) * G.ld0 + col0;
-          store_row_half(xo, v, valid, G.out_half_is_fp16);
-        } else {  // MODE_XLAST: U in the weight's layout
-          const MatInfo& mi = p.mats[G.mat_base + c.mat];
-          float* u = p.u_slab + mi.u_off;
-          if (!mi.trans) {
+        }
+        if (mode == MODE_XLAST) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] *= G.scale;
-            store_row_f32(u + static_cast<int64_t>(row) * mi.un + col0, v, valid);
-          } else {
-            // NS row `row` is weight column `row`; NS column j is weight row j.
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-              if (j < valid) u[static_cast<int64_t>(col0 + j) * mi.un + row] = v[j] * G.scale;
+          for (int h = 0; h < 2; ++h) {
+            const uint32_t s = next_out_slot();
+            uint8_t* sp = slots + s * SLOT_BYTES;
+            if (!G.trans) fill_f32_rows16(sp, lane, v + 16 * h);
+            else fill_f32_cols16(sp, lane, v + 16 * h);
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              if (!G.trans) tma_store_3d(&G.tmOut, slots_s + s * SLOT_BYTES, col0 + 16 * h, row0, c.mat);
+              else tma_store_3d(&G.tmOut, slots_s + s * SLOT_BYTES, row0, col0 + 16 * h, c.mat);
+            }
+          }
+        } else {
+          {
+            const uint32_t s = next_out_slot();
+            fill_half_rows(slots + s * SLOT_BYTES, lane, v, G.out_fp16);
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) tma_store_3d(&G.tmOut, slots_s + s * SLOT_BYTES, col0, row0, c.mat);
+          }
+          if (G.sym && C > R) {
+            const uint32_t s = next_out_slot();
+            fill_half_cols(slots + s * SLOT_BYTES, lane, v, G.out_fp16);
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) tma_store_3d(&G.tmOut, slots_s + s * SLOT_BYTES, row0, col0, c.mat);
           }
         }
-        }  // row_ok
         __syncwarp();  // reconverge before the next warp-wide tcgen05.ld
       }
       tc_fence_before();
@@ -438,11 +530,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
     }
+    // Drain: aux loads still in flight (only after an early exit) and every
+    // TMA store this warp issued.
+    for (int b = 0; b < 2; ++b)
+      if ((aux_pending >> b) & 1u) wait_bounded_warp(AUX_BAR(ew, b), (aux_phase >> b) & 1u, err, DEV_TIMEOUT_DRAIN, tmo);
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
   }
 #undef FULL_BAR
 #undef EMPTY_BAR
 #undef TFULL_BAR
 #undef TEMPTY_BAR
+#undef AUX_BAR
 
   tc_fence_before();
   __syncthreads();
