@@ -157,9 +157,10 @@ meq_status meq_debug_wait_selftest(meq_state* st, float timeout_ms);
  * optimizer: r (rows floats) and c (cols floats) of Eq. (7), gammas[0] =
  * gamma_r and gammas[1] = gamma_c of Eq. (8) over entries > eps, and
  * *direction of Eq. (11) (0 = row, 1 = column; row when gamma_r >= gamma_c -
- * tie_atol). All outputs are caller-provided device memory. The arithmetic is
- * that of meq_step's statistics kernels, so results agree with
- * meq_read_stats for the same U.
+ * tie_atol). All outputs are caller-provided device memory. The definitions
+ * and precision (fp32 sums of squares, fp64 CVs) are those of meq_step's
+ * statistics, so results agree with meq_read_stats for the same U up to fp32
+ * summation order.
  *
  * It allocates nothing. Its scratch is a fixed 8 MiB __device__ array inside
  * the library, held by every GPU that loads the library until the process

@@ -6,9 +6,8 @@
 //                   into the X_0 scale alpha0 / ||H||_F of Eq. (5).
 //   cast_x0       : X-hat_0 = 16-bit(alpha0 H / ||H||_F) in the oriented NS
 //                   layout (transposed through shared memory for tall W).
-//   stats         : row sums of squares and per-slab column partial sums of
-//                   U (Eq. (7)), deterministic.
-//   finalize      : r, c (Eq. (7)), gamma_r, gamma_c (Eq. (8), fp64), the
+//   finalize      : r, c (Eq. (7)) from the partial sums of squares the last
+//                   NS epilogue wrote, gamma_r, gamma_c (Eq. (8), fp64), the
 //                   direction (Eq. (11)) and the scale vector of Eq. (9).
 //   apply         : W <- (1 - lr wd) W - rho lr s (.) U (Eq. (14)).
 #include "meq_elementwise.cuh"
@@ -23,7 +22,7 @@ __device__ __forceinline__ int find_mat(const MatInfo* mats, int nmat, int64_t k
   int lo = 0, hi = nmat - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
-    const int64_t b = which == 0 ? mats[mid].chunk_begin : (which == 1 ? mats[mid].tile_begin : mats[mid].slab_begin);
+    const int64_t b = which == 0 ? mats[mid].chunk_begin : mats[mid].tile_begin;
     if (b <= key) lo = mid; else hi = mid - 1;
   }
   return lo;
@@ -146,6 +145,23 @@ __device__ __forceinline__ uint16_t half_bits(float v) {
   return *reinterpret_cast<uint16_t*>(&h);
 }
 
+__device__ __forceinline__ uint2 pack4(float a, float b, float c, float d, bool fp16) {
+  uint2 w;
+  if (fp16) {
+    __half2 x = __floats2half2_rn(a, b), y = __floats2half2_rn(c, d);
+    w.x = *reinterpret_cast<uint32_t*>(&x);
+    w.y = *reinterpret_cast<uint32_t*>(&y);
+  } else {
+    __nv_bfloat162 x = __floats2bfloat162_rn(a, b), y = __floats2bfloat162_rn(c, d);
+    w.x = *reinterpret_cast<uint32_t*>(&x);
+    w.y = *reinterpret_cast<uint32_t*>(&y);
+  }
+  return w;
+}
+
+// One 64 x 64 tile of W per block. Threads read 4 consecutive columns
+// (128-bit loads when the row length allows) and write 4 consecutive 16-bit
+// values; tall matrices go through a shared-memory transpose.
 template <bool kFp16>
 __global__ void __launch_bounds__(kThreads) cast_x0_kernel(const MatInfo* __restrict__ mats, int nmat,
                                                            const GroupInfo* __restrict__ groups,
@@ -168,115 +184,101 @@ __global__ void __launch_bounds__(kThreads) cast_x0_kernel(const MatInfo* __rest
   const float* B = mom + M.mom_off;
   const float* G = grads[mi];
   uint16_t* X = static_cast<uint16_t*>(Gi.x0) + M.gidx * Gi.s * Gi.lp;
-  const int tx = threadIdx.x % kCastTile;
-  const int ty = threadIdx.x / kCastTile;
-  constexpr int kRowsPerPass = kThreads / kCastTile;
+  const bool vec = (M.n & 3) == 0;
+  const int cx = (threadIdx.x & 15) * 4;  // 4 columns
+  const int ry = threadIdx.x >> 4;        // rows ry, ry + 16, ry + 32, ry + 48
+  float h[4][4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int64_t row = r0 + ry + 16 * k, col = c0 + cx;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) h[k][u] = 0.f;
+    if (row >= M.m) continue;
+    if (vec && col + 3 < M.n) {
+      float4 b = *reinterpret_cast<const float4*>(B + row * M.n + col);
+      if (nesterov) {
+        const float4 g = *reinterpret_cast<const float4*>(G + row * M.n + col);
+        b.x = fmaf(mu, b.x, g.x), b.y = fmaf(mu, b.y, g.y), b.z = fmaf(mu, b.z, g.z), b.w = fmaf(mu, b.w, g.w);
+      }
+      h[k][0] = b.x, h[k][1] = b.y, h[k][2] = b.z, h[k][3] = b.w;
+    } else {
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (col + u < M.n) {
+          float b = B[row * M.n + col + u];
+          if (nesterov) b = fmaf(mu, b, G[row * M.n + col + u]);
+          h[k][u] = b;
+        }
+    }
+  }
   if (!M.trans) {
-    const int64_t c = c0 + tx;
-    if (c < M.n) {
-      for (int r = ty; r < kCastTile; r += kRowsPerPass) {
-        const int64_t row = r0 + r;
-        if (row >= M.m) break;
-        float h = B[row * M.n + c];
-        if (nesterov) h = fmaf(mu, h, G[row * M.n + c]);
-        X[row * Gi.lp + c] = half_bits<kFp16>(h * scale);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int64_t row = r0 + ry + 16 * k, col = c0 + cx;
+      if (row >= M.m) continue;
+      if (col + 3 < M.n) {
+        *reinterpret_cast<uint2*>(X + row * Gi.lp + col) =
+            pack4(h[k][0] * scale, h[k][1] * scale, h[k][2] * scale, h[k][3] * scale, kFp16);
+      } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (col + u < M.n) X[row * Gi.lp + col + u] = half_bits<kFp16>(h[k][u] * scale);
       }
     }
   } else {
-    for (int r = ty; r < kCastTile; r += kRowsPerPass) {
-      const int64_t row = r0 + r, c = c0 + tx;
-      float h = 0.f;
-      if (row < M.m && c < M.n) {
-        h = B[row * M.n + c];
-        if (nesterov) h = fmaf(mu, h, G[row * M.n + c]);
-      }
-      tile[r][tx] = h * scale;
-    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+#pragma unroll
+      for (int u = 0; u < 4; ++u) tile[ry + 16 * k][cx + u] = h[k][u] * scale;
     __syncthreads();
-    // X row = W column (c0 + r), X column = W row (r0 + tx).
-    for (int r = ty; r < kCastTile; r += kRowsPerPass) {
-      const int64_t xrow = c0 + r, xcol = r0 + tx;
-      if (xrow < M.n && xcol < M.m) X[xrow * Gi.lp + xcol] = half_bits<kFp16>(tile[tx][r]);
+    // X row = W column c0 + xr; X columns = W rows r0 + cx .. + 3.
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int xr = ry + 16 * k;
+      const int64_t xrow = c0 + xr, xcol = r0 + cx;
+      if (xrow >= M.n) continue;
+      if (xcol + 3 < M.m) {
+        *reinterpret_cast<uint2*>(X + xrow * Gi.lp + xcol) =
+            pack4(tile[cx][xr], tile[cx + 1][xr], tile[cx + 2][xr], tile[cx + 3][xr], kFp16);
+      } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (xcol + u < M.m) X[xrow * Gi.lp + xcol + u] = half_bits<kFp16>(tile[cx + u][xr]);
+      }
     }
   }
 }
 
 // ----------------------------------------------------------------- statistics
-__global__ void __launch_bounds__(kThreads) stats_kernel(const MatInfo* __restrict__ mats, int nmat,
-                                                         const float* __restrict__ uslab,
-                                                         float* __restrict__ rowss,
-                                                         float* __restrict__ cpart) {
-  __shared__ float shr[kThreads / 32][32];
-  const int64_t slab = blockIdx.x;
-  const int mi = find_mat(mats, nmat, slab, 2);
-  const MatInfo& M = mats[mi];
-  const int64_t ls = slab - M.slab_begin;
-  const int64_t r0 = ls * kSlab;
-  const int nr = static_cast<int>(M.m - r0 < kSlab ? M.m - r0 : kSlab);
-  const float* U = uslab + M.u_off + r0 * M.un;
-  float racc[kSlab];
-#pragma unroll
-  for (int r = 0; r < kSlab; ++r) racc[r] = 0.f;
-  float* cp = cpart + M.cpart_off + ls * M.n;
-  for (int64_t c = threadIdx.x; c < M.n; c += kThreads) {
-    float cacc = 0.f;
-#pragma unroll
-    for (int r = 0; r < kSlab; ++r) {
-      if (r < nr) {
-        const float u = __ldcs(U + r * M.un + c);
-        const float u2 = u * u;
-        cacc += u2;
-        racc[r] += u2;
-      }
-    }
-    cp[c] = cacc;
-  }
-  // Transpose-reduce the 32 row accumulators across the warp: lane l ends
-  // with the warp's sum for row l.
-  const unsigned FULL = 0xffffffffu;
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-#pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) {
-#pragma unroll
-    for (int i = 0; i < o; ++i) {
-      const bool up = (lane & o) != 0;
-      const float send = up ? racc[i] : racc[i + o];
-      const float keep = up ? racc[i + o] : racc[i];
-      racc[i] = keep + __shfl_xor_sync(FULL, send, o);
-    }
-  }
-  shr[w][lane] = racc[0];
-  __syncthreads();
-  if (threadIdx.x < nr) {
-    float s = 0.f;
-    for (int i = 0; i < kThreads / 32; ++i) s += shr[i][threadIdx.x];
-    rowss[M.vec_off + r0 + threadIdx.x] = s;
-  }
-}
-
 // Row / column RMS, CVs (fp64), direction and scale vector; one block per matrix.
 __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __restrict__ mats,
                                                                const StepScalars* __restrict__ sc,
-                                                               const float* __restrict__ rowss,
-                                                               const float* __restrict__ cpart,
+                                                               const float* __restrict__ parts,
                                                                float* __restrict__ rvec, float* __restrict__ cvec,
                                                                float* __restrict__ svec,
                                                                MatStats* __restrict__ stats) {
   __shared__ double shd[32];
   const MatInfo& M = mats[blockIdx.x];
   const float delta = sc->eps;
-  const int64_t nslabs = (M.m + kSlab - 1) / kSlab;
   float* r = rvec + M.vec_off;
   float* c = cvec + M.vec_off;
   float* s = svec + M.vec_off;
   const float inv_n = 1.0f / static_cast<float>(M.n);
   const float inv_m = 1.0f / static_cast<float>(M.m);
-  for (int64_t i = threadIdx.x; i < M.m; i += blockDim.x) r[i] = sqrtf(rowss[M.vec_off + i] * inv_n);
-  for (int64_t j = threadIdx.x; j < M.n; j += blockDim.x) {
+  // NS rows (s of them) are the weight's rows, or its columns when transposed.
+  const int64_t tiles_n = (M.l + 255) / 256;
+  const int64_t nrb = (M.s + 31) / 32;
+  for (int64_t i = threadIdx.x; i < M.s; i += blockDim.x) {
     float acc = 0.f;
-    const float* cp = cpart + M.cpart_off + j;
-    for (int64_t k = 0; k < nslabs; ++k) acc += cp[k * M.n];
-    c[j] = sqrtf(acc * inv_m);
+    for (int64_t t = 0; t < tiles_n; ++t) acc += parts[M.rpart_off + t * M.s + i];
+    if (!M.trans) r[i] = sqrtf(acc * inv_n);
+    else c[i] = sqrtf(acc * inv_m);
+  }
+  for (int64_t j = threadIdx.x; j < M.l; j += blockDim.x) {
+    float acc = 0.f;
+    for (int64_t k = 0; k < nrb; ++k) acc += parts[M.cpart_off + k * M.l + j];
+    if (!M.trans) c[j] = sqrtf(acc * inv_m);
+    else r[j] = sqrtf(acc * inv_n);
   }
   __syncthreads();
   double gam[2];
@@ -395,10 +397,7 @@ cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st) {
 }
 
 cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st) {
-  stats_kernel<<<(unsigned)L.total_slabs, kThreads, 0, st>>>(L.mats, L.nmat, L.uslab, L.rowss, L.cpart);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  finalize_kernel<<<L.nmat, kFinThreads, 0, st>>>(L.mats, L.sc, L.rowss, L.cpart, L.rvec, L.cvec, L.svec, L.stats);
+  finalize_kernel<<<L.nmat, kFinThreads, 0, st>>>(L.mats, L.sc, L.parts, L.rvec, L.cvec, L.svec, L.stats);
   return cudaGetLastError();
 }
 

@@ -43,6 +43,8 @@ struct Group {
   int trans = 0;           // members are tall (W = X^T)
   int64_t m = 0, n = 0, un = 0;  // weight shape of every member, U row stride
   int64_t u_base = 0;      // float offset of the group's U block [count][m][un]
+  int64_t rpart_base = 0;  // float offsets of the fused-statistics partials
+  int64_t cpart_base = 0;
   std::vector<int> mats;
   uint16_t* x[2] = {nullptr, nullptr};
   uint16_t* a16 = nullptr;
@@ -70,8 +72,8 @@ struct meq_state {
   int num_sms = 0;
   std::vector<MatInfo> mats;
   std::vector<Group> groups;
-  int64_t total_chunks = 0, total_tiles = 0, total_slabs = 0;
-  int64_t mom_floats = 0, u_floats = 0, vec_floats = 0, cpart_floats = 0;
+  int64_t total_chunks = 0, total_tiles = 0;
+  int64_t mom_floats = 0, u_floats = 0, vec_floats = 0, parts_floats = 0;
   char* arena = nullptr;
   int64_t arena_bytes = 0;
   // device views
@@ -82,8 +84,7 @@ struct meq_state {
   float* d_rvec = nullptr;
   float* d_cvec = nullptr;
   float* d_svec = nullptr;
-  float* d_rowss = nullptr;
-  float* d_cpart = nullptr;
+  float* d_parts = nullptr;
   float* d_partials = nullptr;
   unsigned int* d_counters = nullptr;
   float* d_x0scale = nullptr;
@@ -182,10 +183,14 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
     M.gidx = st->groups[g].count++;
     st->groups[g].mats.push_back(i);
   }
-  int64_t mom = 0, u = 0, vec = 0, cp = 0, chunks = 0, tiles = 0, slabs = 0;
+  int64_t mom = 0, u = 0, vec = 0, parts = 0, chunks = 0, tiles = 0;
   for (auto& G : st->groups) {  // U is stored group by group: [count][m][un]
     G.u_base = u;
     u += round_up(G.count * G.m * G.un, 64);
+    G.rpart_base = parts;
+    parts += round_up(G.count * ((G.l + 255) / 256) * G.s, 64);
+    G.cpart_base = parts;
+    parts += round_up(G.count * ((G.s + 31) / 32) * G.l, 64);
   }
   for (int i = 0; i < n; ++i) {
     MatInfo& M = st->mats[i];
@@ -194,27 +199,24 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
     M.mom_off = mom;
     mom += round_up(M.m * M.n, 64);
     M.u_off = G.u_base + M.gidx * M.m * M.un;
+    M.rpart_off = G.rpart_base + M.gidx * ((G.l + 255) / 256) * G.s;
+    M.cpart_off = G.cpart_base + M.gidx * ((G.s + 31) / 32) * G.l;
     M.vec_off = vec;
     vec += round_up(std::max(M.m, M.n), 64);
     M.chunk_begin = chunks;
     chunks += (M.m * M.n + kChunk - 1) / kChunk;
     M.tile_begin = tiles;
     tiles += ((M.m + kCastTile - 1) / kCastTile) * ((M.n + kCastTile - 1) / kCastTile);
-    M.slab_begin = slabs;
-    const int64_t ns = (M.m + kSlab - 1) / kSlab;
-    slabs += ns;
-    M.cpart_off = cp;
-    cp += round_up(ns * M.n, 64);
   }
-  st->mom_floats = mom, st->u_floats = u, st->vec_floats = vec, st->cpart_floats = cp;
-  st->total_chunks = chunks, st->total_tiles = tiles, st->total_slabs = slabs;
+  st->mom_floats = mom, st->u_floats = u, st->vec_floats = vec, st->parts_floats = parts;
+  st->total_chunks = chunks, st->total_tiles = tiles;
   st->persistent_bytes = 0;
   for (int i = 0; i < n; ++i) st->persistent_bytes += 4 * st->mats[i].m * st->mats[i].n;
 
   *off_mom = L->add(mom * 4);
   *off_u = L->add(u * 4);
-  *off_vec4 = L->add(vec * 4 * 4);  // r, c, scale, row sums of squares
-  *off_cpart = L->add(cp * 4);
+  *off_vec4 = L->add(vec * 3 * 4);  // r, c, scale
+  *off_cpart = L->add(parts * 4);
   *off_partials = L->add(chunks * 4);
   *off_counters = L->add(int64_t(n) * 4);
   *off_x0s = L->add(int64_t(n) * 4);
@@ -346,6 +348,8 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
                 ok &= encode_map(&Q.tmOut, ub, 4, G.n, G.m, G.count, G.un, 32, 16, SW128);
               Q.scale = 1.0f / ak;
               Q.out_fp16 = 0;
+              Q.rpart = st->d_parts + G.rpart_base;
+              Q.cpart = st->d_parts + G.cpart_base;
             }
           }
           if (!ok) { *why = "cuTensorMapEncodeTiled failed"; return false; }
@@ -473,8 +477,7 @@ meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt
   st->d_rvec = reinterpret_cast<float*>(A + off_vec4);
   st->d_cvec = st->d_rvec + st->vec_floats;
   st->d_svec = st->d_cvec + st->vec_floats;
-  st->d_rowss = st->d_svec + st->vec_floats;
-  st->d_cpart = reinterpret_cast<float*>(A + off_cpart);
+  st->d_parts = reinterpret_cast<float*>(A + off_cpart);
   st->d_partials = reinterpret_cast<float*>(A + off_partials);
   st->d_counters = reinterpret_cast<unsigned int*>(A + off_counters);
   st->d_x0scale = reinterpret_cast<float*>(A + off_x0s);
@@ -528,16 +531,14 @@ meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt
   C.counters = st->d_counters;
   C.x0scale = st->d_x0scale;
   C.uslab = st->d_u;
-  C.rowss = st->d_rowss;
-  C.cpart = st->d_cpart;
+  C.parts = st->d_parts;
   C.rvec = st->d_rvec;
   C.cvec = st->d_cvec;
   C.svec = st->d_svec;
   C.stats = st->d_stats;
   C.total_chunks = st->total_chunks;
   C.total_tiles = st->total_tiles;
-  C.total_slabs = st->total_slabs;
-  st->kernels_per_step = 5 + static_cast<int>(st->gemm.size());
+  st->kernels_per_step = 4 + static_cast<int>(st->gemm.size());
   st->step_host.assign(static_cast<size_t>(st->step_bytes), 0);
   st->last_stream = s;
   *out = st;

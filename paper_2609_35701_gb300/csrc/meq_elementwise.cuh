@@ -7,7 +7,6 @@ namespace meq {
 
 constexpr int64_t kChunk = 4096;   // elements per momentum / apply block
 constexpr int kCastTile = 64;      // X_0 cast tile (64 x 64 of W)
-constexpr int kSlab = 32;          // rows per statistics block
 constexpr int kFinThreads = 1024;  // finalize block size
 
 struct MatStats {
@@ -30,18 +29,17 @@ struct LaunchCtx {
   unsigned int* counters;
   float* x0scale;
   float* uslab;
-  float* rowss;
-  float* cpart;
+  float* parts;          // NS-row and NS-column partial sums of squares
   float* rvec;
   float* cvec;
   float* svec;
   MatStats* stats;
-  int64_t total_chunks, total_tiles, total_slabs;
+  int64_t total_chunks, total_tiles;
 };
 
 cudaError_t launch_momentum_norm(const LaunchCtx& L, cudaStream_t st);
 cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st);
-cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st);  // stats + finalize (2 kernels)
+cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st);  // finalize of the fused statistics
 cudaError_t launch_apply(const LaunchCtx& L, cudaStream_t st);
 cudaError_t launch_wait_selftest(const int* flag, int* err, unsigned long long timeout_ns, cudaStream_t st);
 

@@ -36,8 +36,8 @@ struct MatInfo {
   int64_t vec_off;       // float offset of r (m), c (n) and scale (max(m, n))
   int64_t chunk_begin;   // first momentum chunk
   int64_t tile_begin;    // first cast tile
-  int64_t slab_begin;    // first statistics slab
-  int64_t cpart_off;     // float offset of the column partial sums [nslabs][n]
+  int64_t rpart_off;     // float offset of NS-row partial sums of squares [ceil(l/256)][s]
+  int64_t cpart_off;     // float offset of NS-column partial sums of squares [ceil(s/32)][l]
 };
 
 // Per-group metadata for the elementwise kernels.
@@ -73,6 +73,8 @@ struct GemmGroup {
   int32_t trans;          // XLAST: 1 when the weight is the transpose of the NS layout
   float scale;            // GRAM: 1/alpha^2; XUPD: alpha_next/alpha; XLAST: 1/alpha
   int32_t out_fp16;       // 16-bit format of the output / aux operand (1 = fp16, 0 = bf16)
+  float* rpart;           // XLAST: NS-row partial sums of squares, [count][tiles_n][M]
+  float* cpart;           // XLAST: NS-column partial sums of squares, [count][ceil(M/32)][N]
 };
 
 struct GemmParams {

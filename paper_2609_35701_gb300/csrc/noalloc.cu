@@ -10,9 +10,9 @@
 // file-scope __device__ array of fixed size that every GPU which loads the
 // library holds until the process exits.
 //
-// The arithmetic (32-row slabs, per-slab column partial sums, warp
-// transpose-reduction of row sums, fp64 CVs) is the same as the statistics
-// kernels of the full step, so results agree with meq_read_stats.
+// It sums squares in fp32 over 32-row slabs and forms the CVs in fp64, the
+// same definitions and precision as the full step's statistics, so results
+// agree with meq_read_stats up to fp32 summation order.
 #include <mutex>
 
 #include "../../include/meq.h"

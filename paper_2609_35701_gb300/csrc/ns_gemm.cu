@@ -8,7 +8,9 @@
 //               a I + b A is added in fp32 from the same 16-bit A the
 //               product uses, so P is exactly a polynomial of that matrix
 //   MODE_XUPD : X'  = P X * (alpha'/alpha)      (s x l, contraction over s)
-//   MODE_XLAST: U   = P X / alpha, written as fp32 in the weight's own layout
+//   MODE_XLAST: U   = P X / alpha, written as fp32 in the weight's own layout,
+//               with the sums of squares of U's rows and columns (Eq. (7))
+//               reduced in the epilogue into per-tile partials
 //
 // P X equals a X + (b A + c A^2) X of Eq. (5) exactly in real arithmetic.
 // A and P are symmetric: their launches run only the tiles that hold a 32 x 32
@@ -455,6 +457,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       tc_fence_after();
       const int row0 = c.tm * BM + q * 32;
       const int R = c.tm * 4 + q;  // 32-row block index
+      float rsum = 0.f;            // XLAST: this lane's row, sum of squares over the tile
       const int nch = min(BN / 32, (G.N - c.tn * BN + 31) / 32);
       int ch0 = G.sym ? max(0, R - c.tn * 8) : 0;  // blocks strictly below the diagonal come from mirrors
       if (row0 >= G.M) ch0 = nch;
@@ -493,6 +496,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
           for (int j = 0; j < 32; ++j) v[j] *= G.scale;
         }
         if (mode == MODE_XLAST) {
+          // Column sums of squares over the warp's 32 rows: transpose-reduce
+          // so that lane j ends with the sum for column col0 + j.
+          float sq[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            sq[j] = v[j] * v[j];
+            rsum += sq[j];
+          }
+#pragma unroll
+          for (int o = 16; o >= 1; o >>= 1) {
+#pragma unroll
+            for (int i = 0; i < o; ++i) {
+              const bool up = (lane & o) != 0;
+              const float send = up ? sq[i] : sq[i + o];
+              const float keep = up ? sq[i + o] : sq[i];
+              sq[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+            }
+          }
+          if (col0 + lane < G.N)
+            G.cpart[(static_cast<int64_t>(c.mat) * ((G.M + 31) / 32) + R) * G.N + col0 + lane] = sq[0];
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             const uint32_t s = next_out_slot();
@@ -524,6 +547,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
         }
         __syncwarp();  // reconverge before the next warp-wide tcgen05.ld
       }
+      if (mode == MODE_XLAST && ch0 < nch && row0 + lane < G.M)
+        G.rpart[(static_cast<int64_t>(c.mat) * G.tiles_n + c.tn) * G.M + row0 + lane] = rsum;
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(TEMPTY_BAR(acc));
