@@ -266,7 +266,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
   const float inv_n = 1.0f / static_cast<float>(M.n);
   const float inv_m = 1.0f / static_cast<float>(M.m);
   // NS rows (s of them) are the weight's rows, or its columns when transposed.
-  const int64_t tiles_n = (M.l + 255) / 256;
+  const int64_t tiles_n = 2 * ((M.l + 255) / 256);  // two epilogue halves per 256-column tile
   const int64_t nrb = (M.s + 31) / 32;
   for (int64_t i = threadIdx.x; i < M.s; i += blockDim.x) {
     float acc = 0.f;

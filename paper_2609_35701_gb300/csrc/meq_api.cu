@@ -188,7 +188,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
     G.u_base = u;
     u += round_up(G.count * G.m * G.un, 64);
     G.rpart_base = parts;
-    parts += round_up(G.count * ((G.l + 255) / 256) * G.s, 64);
+    parts += round_up(G.count * 2 * ((G.l + 255) / 256) * G.s, 64);
     G.cpart_base = parts;
     parts += round_up(G.count * ((G.s + 31) / 32) * G.l, 64);
   }
@@ -199,7 +199,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
     M.mom_off = mom;
     mom += round_up(M.m * M.n, 64);
     M.u_off = G.u_base + M.gidx * M.m * M.un;
-    M.rpart_off = G.rpart_base + M.gidx * ((G.l + 255) / 256) * G.s;
+    M.rpart_off = G.rpart_base + M.gidx * 2 * ((G.l + 255) / 256) * G.s;
     M.cpart_off = G.cpart_base + M.gidx * ((G.s + 31) / 32) * G.l;
     M.vec_off = vec;
     vec += round_up(std::max(M.m, M.n), 64);
@@ -265,7 +265,6 @@ bool encode_map(CUtensorMap* m, void* base, int elem_bytes, int64_t inner, int64
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
-constexpr CUtensorMapSwizzle SW64 = CU_TENSOR_MAP_SWIZZLE_64B;
 constexpr CUtensorMapSwizzle SW128 = CU_TENSOR_MAP_SWIZZLE_128B;
 
 int sym_tiles(int tiles_m, int tiles_n) {
@@ -314,12 +313,14 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
           Q.count = static_cast<int32_t>(G.count);
           Q.trans = G.trans;
           bool ok = true;
+          const int64_t x_ld = G.lp * 2, x_ms = G.s * G.lp * 2;   // 16-bit X buffers, bytes
+          const int64_t s_ld = G.sp * 2, s_ms = G.s * G.sp * 2;   // 16-bit A / P buffers, bytes
           if (mode == MODE_GRAM) {
             Q.M = (int32_t)G.s, Q.N = (int32_t)G.s, Q.K = (int32_t)G.l;
             Q.sym = 1;
             ok &= encode_map(&Q.tmA, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 128, SW128);
             ok &= encode_map(&Q.tmB, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 256, SW128);
-            ok &= encode_map(&Q.tmOut, G.a16, 2, G.s, G.s, G.count, G.sp, 32, 32, SW64);
+            Q.out = G.a16, Q.out_ld = s_ld, Q.out_mstride = s_ms;
             Q.scale = 1.0f / (ak * ak);
             Q.out_fp16 = f16;
           } else if (mode == MODE_POLY) {
@@ -327,8 +328,8 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             Q.sym = 1;
             ok &= encode_map(&Q.tmA, G.a16, 2, G.s, G.s, G.count, G.sp, 64, 128, SW128);
             ok &= encode_map(&Q.tmB, G.a16, 2, G.s, G.s, G.count, G.sp, 64, 256, SW128);
-            ok &= encode_map(&Q.tmOut, G.p16, 2, G.s, G.s, G.count, G.sp, 32, 32, SW64);
-            ok &= encode_map(&Q.tmAux, G.a16, 2, G.s, G.s, G.count, G.sp, 32, 32, SW64);
+            Q.out = G.p16, Q.out_ld = s_ld, Q.out_mstride = s_ms;
+            Q.aux = G.a16, Q.aux_ld = s_ld, Q.aux_mstride = s_ms;
             Q.scale = 1.0f;
             Q.out_fp16 = f16;
           } else {
@@ -337,15 +338,11 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             ok &= encode_map(&Q.tmA, G.p16, 2, G.s, G.s, G.count, G.sp, 64, 128, SW128);
             ok &= encode_map(&Q.tmB, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 64, SW128);
             if (real_mode == MODE_XUPD) {
-              ok &= encode_map(&Q.tmOut, G.x[nxt], 2, G.l, G.s, G.count, G.lp, 32, 32, SW64);
+              Q.out = G.x[nxt], Q.out_ld = x_ld, Q.out_mstride = x_ms;
               Q.scale = G.alpha / ak;
               Q.out_fp16 = next_f16;
             } else {
-              float* ub = st->d_u + G.u_base;
-              if (!G.trans)
-                ok &= encode_map(&Q.tmOut, ub, 4, G.n, G.m, G.count, G.un, 16, 32, SW64);
-              else
-                ok &= encode_map(&Q.tmOut, ub, 4, G.n, G.m, G.count, G.un, 32, 16, SW128);
+              Q.out = st->d_u + G.u_base, Q.out_ld = G.un * 4, Q.out_mstride = G.m * G.un * 4;
               Q.scale = 1.0f / ak;
               Q.out_fp16 = 0;
               Q.rpart = st->d_parts + G.rpart_base;
@@ -362,6 +359,10 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
           tiles += static_cast<int>(t);
         }
         P.total_tiles = tiles;
+        // Each launch walks the matrices in the opposite order of the one
+        // before it (the X_0 cast writes in forward order), so it begins with
+        // the outputs still resident in L2.
+        P.reverse = (st->gemm.size() % 2 == 0) ? 1 : 0;
         st->gemm.push_back(P);
         st->gemm_grid.push_back(std::max(1, std::min(tiles, st->num_sms)));
       }

@@ -36,7 +36,7 @@ struct MatInfo {
   int64_t vec_off;       // float offset of r (m), c (n) and scale (max(m, n))
   int64_t chunk_begin;   // first momentum chunk
   int64_t tile_begin;    // first cast tile
-  int64_t rpart_off;     // float offset of NS-row partial sums of squares [ceil(l/256)][s]
+  int64_t rpart_off;     // float offset of NS-row partial sums of squares [2 * ceil(l/256)][s]
   int64_t cpart_off;     // float offset of NS-column partial sums of squares [ceil(s/32)][l]
 };
 
@@ -62,8 +62,6 @@ enum GemmMode : int { MODE_GRAM = 0, MODE_POLY = 1, MODE_XUPD = 2, MODE_XLAST = 
 struct GemmGroup {
   CUtensorMap tmA;        // A operand (K-major), box {64, 128, 1}
   CUtensorMap tmB;        // B operand: K-major box {64, 256, 1} or MN-major box {64, 64, 1}
-  CUtensorMap tmOut;      // epilogue TMA store: 16-bit {32, 32, 1}; U fp32 {16, 32, 1} or {32, 16, 1}
-  CUtensorMap tmAux;      // POLY: 16-bit A, box {32, 32, 1}, loaded by the epilogue
   int32_t M, N, K;        // output rows, output cols, contraction
   int32_t count;          // matrices in the group
   int32_t tiles_m, tiles_n;
@@ -73,7 +71,13 @@ struct GemmGroup {
   int32_t trans;          // XLAST: 1 when the weight is the transpose of the NS layout
   float scale;            // GRAM: 1/alpha^2; XUPD: alpha_next/alpha; XLAST: 1/alpha
   int32_t out_fp16;       // 16-bit format of the output / aux operand (1 = fp16, 0 = bf16)
-  float* rpart;           // XLAST: NS-row partial sums of squares, [count][tiles_n][M]
+  void* out;              // GRAM: 16-bit A; POLY: 16-bit P; XUPD: 16-bit X next; XLAST: fp32 U (weight layout)
+  int64_t out_ld;         // output row stride in bytes
+  int64_t out_mstride;    // output matrix stride in bytes
+  const void* aux;        // POLY: 16-bit A
+  int64_t aux_ld;         // bytes
+  int64_t aux_mstride;    // bytes
+  float* rpart;           // XLAST: NS-row partial sums of squares, [count][2 * tiles_n][M]
   float* cpart;           // XLAST: NS-column partial sums of squares, [count][ceil(M/32)][N]
 };
 
@@ -84,6 +88,7 @@ struct GemmParams {
   int32_t mode;
   uint32_t idesc;          // tcgen05 instruction descriptor
   int32_t b_mn_major;      // 1: B operand tile is MN-major (XUPD)
+  int32_t reverse;         // 1: tiles are taken in reverse order (alternates between launches)
   float ca, cb, cc;        // NS coefficients
   int* err;                // device error word
   unsigned long long timeout_ns;

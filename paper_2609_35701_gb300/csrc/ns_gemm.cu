@@ -19,13 +19,17 @@
 // X is stored scaled by a power of two alpha so its entries stay in the
 // normal range of fp16; the epilogues undo the scale in fp32.
 //
-// Roles (192 threads, one CTA per SM):
+// Roles (320 threads, one CTA per SM):
 //   warp 0 : TMA producer (one thread), 4-stage shared-memory ring
 //   warp 1 : TMEM allocator and tcgen05.mma issuer (one thread)
-//   warps 2-5 : epilogue; warp w reads TMEM lanes 32*(w%4) .. +31
+//   warps 2-9 : epilogue; warp w reads TMEM lanes 32*(w%4) .. +31 and takes
+//               every other 32-column chunk (two warps per lane quarter, so
+//               each SM sub-partition can hide one warp's latencies behind
+//               the other's work)
 // Two 128x256 fp32 accumulators (512 TMEM columns) let the epilogue of one
 // tile overlap the MMAs of the next. The epilogue stages 32 x 32 blocks in
-// swizzled shared memory and writes them with TMA bulk-tensor stores.
+// swizzled shared memory and writes them with coalesced 16-byte stores (the
+// SM's TMA unit stays free for the operand loads).
 //
 // Every mbarrier wait is bounded (time and iteration count). On expiry the
 // waiting role records an error code, the others see it and stop, in-flight
@@ -40,12 +44,13 @@ constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4, UK = 16;
 constexpr int A_BYTES = BM * BK * 2;                 // 16 KB
 constexpr int B_BYTES = BN * BK * 2;                 // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;       // 48 KB
-constexpr int NUM_THREADS = 192;
+constexpr int NUM_EPI_WARPS = 8;                    // two per TMEM lane quarter
+constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int SLOT_BYTES = 2048;                      // one 32 x 32 16-bit block (or 32 x 16 fp32)
-constexpr int NUM_BARS = 2 * STAGES + 4 + 1 + 8;     // full, empty, tmem full x2, tmem empty x2, drain, aux 4x2
-constexpr int SMEM_EPI_OFF = STAGES * STAGE_BYTES;   // 4 epilogue warps x 4 slots
-constexpr int SMEM_BAR_OFF = SMEM_EPI_OFF + 4 * 4 * SLOT_BYTES;
+constexpr int NUM_BARS = 2 * STAGES + 4 + 1;         // full, empty, tmem full x2, tmem empty x2, drain
+constexpr int SMEM_EPI_OFF = STAGES * STAGE_BYTES;   // one staging slot per epilogue warp
+constexpr int SMEM_BAR_OFF = SMEM_EPI_OFF + NUM_EPI_WARPS * SLOT_BYTES;
 constexpr int SMEM_BYTES = SMEM_BAR_OFF + NUM_BARS * 8 + 16 + 1024;
 static_assert(SMEM_BYTES <= 232448, "shared memory budget of one sm_103a CTA");
 
@@ -177,11 +182,14 @@ struct TileCoord {
   int g, mat, tm, tn;
 };
 
-// Tiles of a group are numbered matrix by matrix. Dense outputs run tm-major
+// Tiles of a group are numbered matrix by matrix (walked backwards when
+// p.reverse is set, so a launch starts on the matrices its predecessor wrote
+// last, which are still in L2). Dense outputs run tm-major
 // over tiles_m x tiles_n; symmetric outputs (Gram, polynomial) run tn-major
 // over the tiles with tm < 2 (tn + 1), i.e. those holding a 32 x 32 block on
 // or above the diagonal.
 __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
+  if (p.reverse) t = p.total_tiles - 1 - t;
   int g = 0;
   while (g + 1 < p.ngroups && t >= p.g[g + 1].tile_begin) ++g;
   const GemmGroup& G = p.g[g];
@@ -233,17 +241,11 @@ __device__ __forceinline__ float2 unpack_half2(uint32_t w, int fp16) {
   return __bfloat1622float2(h);
 }
 
-// ---- TMA store / bulk-group helpers (issued by one lane) ----------------------
-__device__ __forceinline__ void tma_store_3d(const CUtensorMap* tm, uint32_t src, int x, int y, int z) {
-  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
-                   reinterpret_cast<uint64_t>(tm)),
-               "r"(src), "r"(x), "r"(y), "r"(z)
-               : "memory");
-  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-}
-__device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+// ---- epilogue block staging ----------------------------------------------------
+// A warp stages one 32-row block in its shared-memory slot with a swizzled
+// layout (conflict-free for the per-row writes below), then writes it back out
+// with coalesced 16-byte global stores: lane L takes 16-byte chunk (L % 4) of
+// rows L / 4, L / 4 + 8, ... so one warp instruction covers 8 rows x 64 bytes.
 
 // Row-major 32 x 32 16-bit block, 64-byte rows, 64B swizzle (16-byte chunk k
 // of row r sits at chunk k ^ ((r >> 1) & 3)).
@@ -280,6 +282,31 @@ __device__ __forceinline__ void fill_f32_cols16(uint8_t* slot, int r, const floa
     *reinterpret_cast<float*>(slot + j * 128 + ((((r >> 2) ^ (j & 7))) << 4) + ((r & 3) << 2)) = v[j];
 }
 
+// 32 rows x 64 bytes (16-bit 32 x 32, or fp32 32 x 16) -> global: rows
+// r < rows_valid, 16-byte chunks k < chunks_valid of each row.
+__device__ __forceinline__ void store_block64(const uint8_t* slot, int lane, uint8_t* dst, int64_t ld_bytes,
+                                              int rows_valid, int chunks_valid) {
+  const int k = lane & 3;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int r = (lane >> 2) + 8 * i;
+    const uint4 w = *reinterpret_cast<const uint4*>(slot + r * 64 + ((k ^ ((r >> 1) & 3)) << 4));
+    if (r < rows_valid && k < chunks_valid) *reinterpret_cast<uint4*>(dst + r * ld_bytes + k * 16) = w;
+  }
+}
+// 16 rows x 128 bytes (fp32 16 x 32, 128B swizzle) -> global: rows
+// r < rows_valid, 16-byte chunks k < chunks_valid of each row.
+__device__ __forceinline__ void store_block128(const uint8_t* slot, int lane, uint8_t* dst, int64_t ld_bytes,
+                                               int rows_valid, int chunks_valid) {
+  const int k = lane & 7;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int r = (lane >> 3) + 4 * i;
+    const uint4 w = *reinterpret_cast<const uint4*>(slot + r * 128 + ((k ^ (r & 7)) << 4));
+    if (r < rows_valid && k < chunks_valid) *reinterpret_cast<uint4*>(dst + r * ld_bytes + k * 16) = w;
+  }
+}
+
 __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_constant__ GemmParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -293,7 +320,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
 #define EMPTY_BAR(s) (bar0 + 8u * (STAGES + (s)))
 #define TFULL_BAR(a) (bar0 + 8u * (2 * STAGES + (a)))
 #define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
-#define AUX_BAR(w, b) (bar0 + 8u * (2 * STAGES + 5 + 2 * (w) + (b)))
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -307,17 +333,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(TFULL_BAR(a), 1);
-      mbar_init(TEMPTY_BAR(a), 4);
+      mbar_init(TEMPTY_BAR(a), NUM_EPI_WARPS);
     }
     mbar_init(drain_bar, 1);
-    for (int w = 0; w < 4; ++w)
-      for (int b = 0; b < 2; ++b) mbar_init(AUX_BAR(w, b), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     for (int g = 0; g < p.ngroups; ++g) {
       prefetch_tmap(&p.g[g].tmA);
       prefetch_tmap(&p.g[g].tmB);
-      prefetch_tmap(&p.g[g].tmOut);
-      if (p.mode == MODE_POLY) prefetch_tmap(&p.g[g].tmAux);
     }
   }
   if (warp == 1) {
@@ -418,69 +440,64 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     __syncwarp();
   } else {
     // ------------------------------------------------------------------ epilogue
-    // Warp ew (0..3) owns TMEM lanes 32*q .. +31 (q = warp % 4), i.e. rows
-    // 32q .. 32q+31 of the tile, and four 2 KB shared-memory slots: two output
-    // staging slots used in turn (a TMA store drains one while the other is
-    // filled) and two slots the polynomial epilogue TMA-loads A chunks into.
+    // Warp ew (0..7) owns TMEM lanes 32*q .. +31 (q = warp % 4), i.e. rows
+    // 32q .. 32q+31 of the tile, chunks ch with ch % 2 == half, and one 2 KB
+    // shared-memory slot, used in turn for the polynomial's A block (which is
+    // prefetched into registers one chunk ahead), the block as computed and
+    // its transpose (symmetric outputs).
     const int q = warp & 3;
     const int ew = warp - 2;
-    uint8_t* slots = gbase + SMEM_EPI_OFF + ew * (4 * SLOT_BYTES);
-    const uint32_t slots_s = base + SMEM_EPI_OFF + ew * (4 * SLOT_BYTES);
+    const int half = ew >> 2;
+    uint8_t* slot = gbase + SMEM_EPI_OFF + ew * SLOT_BYTES;
     const int mode = p.mode;
-    int out_slot = 0;
-    uint32_t aux_phase = 0;    // bit b: parity of the next completion of aux slot b
-    uint32_t aux_pending = 0;  // bit b: aux slot b has a load in flight
-    bool ok = true;
     int acc = 0;
     uint32_t acc_phase = 0;
 
-    auto next_out_slot = [&]() -> uint32_t {
-      // The slot used two stores ago must have been read by its TMA store.
-      if (lane == 0) bulk_wait_read_1();
-      __syncwarp();
-      const uint32_t s = static_cast<uint32_t>(out_slot);
-      out_slot ^= 1;
-      return s;
-    };
-    auto issue_aux = [&](const GemmGroup& G, int b, int col0, int row0, int mat) {
-      if (lane == 0) {
-        mbar_expect_tx(AUX_BAR(ew, b), SLOT_BYTES);
-        tma_load_3d(slots_s + (2 + b) * SLOT_BYTES, &G.tmAux, AUX_BAR(ew, b), col0, row0, mat);
-      }
-      aux_pending |= 1u << b;
-    };
-
-    for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+    for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
       const TileCoord c = decode_tile(p, t);
       const GemmGroup& G = p.g[c.g];
       if (!wait_bounded_warp(TFULL_BAR(acc), acc_phase, err, DEV_TIMEOUT_EPI, tmo)) break;
       tc_fence_after();
       const int row0 = c.tm * BM + q * 32;
       const int R = c.tm * 4 + q;  // 32-row block index
+      const int rows_valid = min(32, G.M - row0);
       float rsum = 0.f;            // XLAST: this lane's row, sum of squares over the tile
       const int nch = min(BN / 32, (G.N - c.tn * BN + 31) / 32);
       int ch0 = G.sym ? max(0, R - c.tn * 8) : 0;  // blocks strictly below the diagonal come from mirrors
+      if ((ch0 & 1) != half) ++ch0;                // this warp's chunks: ch % 2 == half
       if (row0 >= G.M) ch0 = nch;
-      if (mode == MODE_POLY && ch0 < nch) issue_aux(G, ch0 & 1, c.tn * BN + ch0 * 32, row0, c.mat);
-      for (int ch = ch0; ch < nch; ++ch) {
+      uint8_t* outm = static_cast<uint8_t*>(G.out) + static_cast<int64_t>(c.mat) * G.out_mstride;
+      // POLY: A block of the chunk, lane L holds 16-byte chunk (L % 4) of rows L/4 + 8i.
+      uint4 aux[4];
+      const uint8_t* auxm = reinterpret_cast<const uint8_t*>(G.aux) + static_cast<int64_t>(c.mat) * G.aux_mstride;
+      auto load_aux = [&](int col0) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int r = (lane >> 2) + 8 * i;
+          aux[i] = make_uint4(0u, 0u, 0u, 0u);
+          if (r < rows_valid)
+            aux[i] = __ldg(reinterpret_cast<const uint4*>(auxm + static_cast<int64_t>(row0 + r) * G.aux_ld +
+                                                         static_cast<int64_t>(col0) * 2 + (lane & 3) * 16));
+        }
+      };
+      if (mode == MODE_POLY && ch0 < nch) load_aux(c.tn * BN + ch0 * 32);
+      for (int ch = ch0; ch < nch; ch += 2) {
         const int col0 = c.tn * BN + ch * 32;
         const int C = c.tn * 8 + ch;
-        if (mode == MODE_POLY && ch + 1 < nch) issue_aux(G, (ch + 1) & 1, col0 + 32, row0, c.mat);
         float v[32];
         tmem_ld_32cols(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN + ch * 32), v);
         if (mode == MODE_POLY) {
-          const int b = ch & 1;
-          if (!wait_bounded_warp(AUX_BAR(ew, b), (aux_phase >> b) & 1u, err, DEV_TIMEOUT_EPI, tmo)) {
-            ok = false;
-            break;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int r = (lane >> 2) + 8 * i, k = lane & 3;
+            *reinterpret_cast<uint4*>(slot + r * 64 + ((k ^ ((r >> 1) & 3)) << 4)) = aux[i];
           }
-          aux_phase ^= 1u << b;
-          aux_pending &= ~(1u << b);
-          const uint8_t* as = slots + (2 + b) * SLOT_BYTES;
+          __syncwarp();
+          if (ch + 2 < nch) load_aux(col0 + 64);  // in flight while this chunk is processed
           const int row = row0 + lane;
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
-            const uint4 w = *reinterpret_cast<const uint4*>(as + lane * 64 + ((k ^ ((lane >> 1) & 3)) << 4));
+            const uint4 w = *reinterpret_cast<const uint4*>(slot + lane * 64 + ((k ^ ((lane >> 1) & 3)) << 4));
             const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
             for (int h = 0; h < 4; ++h) {
@@ -490,7 +507,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
               v[j + 1] = fmaf(p.cc, v[j + 1], fmaf(p.cb, a2.y, (col0 + j + 1 == row) ? p.ca : 0.f));
             }
           }
-          fence_async_smem();  // generic reads of the aux slot before its next TMA fill
+          __syncwarp();  // slot free for the output block
         } else {
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] *= G.scale;
@@ -518,55 +535,52 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
             G.cpart[(static_cast<int64_t>(c.mat) * ((G.M + 31) / 32) + R) * G.N + col0 + lane] = sq[0];
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
-            const uint32_t s = next_out_slot();
-            uint8_t* sp = slots + s * SLOT_BYTES;
-            if (!G.trans) fill_f32_rows16(sp, lane, v + 16 * h);
-            else fill_f32_cols16(sp, lane, v + 16 * h);
-            fence_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-              if (!G.trans) tma_store_3d(&G.tmOut, slots_s + s * SLOT_BYTES, col0 + 16 * h, row0, c.mat);
-              else tma_store_3d(&G.tmOut, slots_s + s * SLOT_BYTES, row0, col0 + 16 * h, c.mat);
+            if (!G.trans) {
+              // U rows = NS rows; 16 columns col0 + 16h .. of 4-float chunks
+              fill_f32_rows16(slot, lane, v + 16 * h);
+              __syncwarp();
+              // 4-float chunks starting below N stay inside the padded row (stride = N rounded up to 4)
+              if (col0 + 16 * h < G.N)
+                store_block64(slot, lane, outm + static_cast<int64_t>(row0) * G.out_ld + (col0 + 16 * h) * 4, G.out_ld,
+                              rows_valid, (G.N - (col0 + 16 * h) + 3) / 4);
+            } else {
+              // U rows = NS columns col0 + 16h + j, U columns = NS rows row0 + r
+              fill_f32_cols16(slot, lane, v + 16 * h);
+              __syncwarp();
+              if (col0 + 16 * h < G.N)
+                store_block128(slot, lane, outm + static_cast<int64_t>(col0 + 16 * h) * G.out_ld + row0 * 4, G.out_ld,
+                               min(16, G.N - (col0 + 16 * h)), (rows_valid + 3) / 4);
             }
+            __syncwarp();
           }
         } else {
-          {
-            const uint32_t s = next_out_slot();
-            fill_half_rows(slots + s * SLOT_BYTES, lane, v, G.out_fp16);
-            fence_async_smem();
-            __syncwarp();
-            if (lane == 0) tma_store_3d(&G.tmOut, slots_s + s * SLOT_BYTES, col0, row0, c.mat);
-          }
+          // 16-bit rows are padded to a multiple of 64 elements: whole 32-column blocks stay inside them
+          fill_half_rows(slot, lane, v, G.out_fp16);
+          __syncwarp();
+          store_block64(slot, lane, outm + static_cast<int64_t>(row0) * G.out_ld + col0 * 2, G.out_ld, rows_valid, 4);
           if (G.sym && C > R) {
-            const uint32_t s = next_out_slot();
-            fill_half_cols(slots + s * SLOT_BYTES, lane, v, G.out_fp16);
-            fence_async_smem();
             __syncwarp();
-            if (lane == 0) tma_store_3d(&G.tmOut, slots_s + s * SLOT_BYTES, row0, col0, c.mat);
+            fill_half_cols(slot, lane, v, G.out_fp16);
+            __syncwarp();
+            store_block64(slot, lane, outm + static_cast<int64_t>(col0) * G.out_ld + row0 * 2, G.out_ld,
+                          min(32, G.M - col0), 4);
           }
         }
-        __syncwarp();  // reconverge before the next warp-wide tcgen05.ld
+        __syncwarp();  // slots free again; reconverge before the next warp-wide tcgen05.ld
       }
-      if (mode == MODE_XLAST && ch0 < nch && row0 + lane < G.M)
-        G.rpart[(static_cast<int64_t>(c.mat) * G.tiles_n + c.tn) * G.M + row0 + lane] = rsum;
+      if (mode == MODE_XLAST && row0 < G.M && row0 + lane < G.M)  // one partial per (tile column, half)
+        G.rpart[(static_cast<int64_t>(c.mat) * G.tiles_n * 2 + c.tn * 2 + half) * G.M + row0 + lane] = rsum;
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(TEMPTY_BAR(acc));
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
     }
-    // Drain: aux loads still in flight (only after an early exit) and every
-    // TMA store this warp issued.
-    for (int b = 0; b < 2; ++b)
-      if ((aux_pending >> b) & 1u) wait_bounded_warp(AUX_BAR(ew, b), (aux_phase >> b) & 1u, err, DEV_TIMEOUT_DRAIN, tmo);
-    if (lane == 0) bulk_wait_all();
-    __syncwarp();
   }
 #undef FULL_BAR
 #undef EMPTY_BAR
 #undef TFULL_BAR
 #undef TEMPTY_BAR
-#undef AUX_BAR
 
   tc_fence_before();
   __syncthreads();
