@@ -67,6 +67,8 @@ typedef struct {
   int use_graph;          /* 1: the step's kernels are replayed from a CUDA graph (default) */
   int64_t workspace_limit_bytes; /* 0 = no limit; else init fails with MEQ_ERR_OOM above it */
   float wait_timeout_ms;  /* bound of every device-side spin wait; default 4000 */
+  int ns_cta_pair;        /* 1 (default): NS GEMMs run on CTA pairs (tcgen05 cta_group::2,
+                             256 x 256 tiles on two SMs); 0: one CTA per 128 x 256 tile */
 } meq_options;
 
 typedef struct meq_state meq_state; /* opaque */

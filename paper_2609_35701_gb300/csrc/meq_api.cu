@@ -127,6 +127,7 @@ bool valid_options(const meq_options& o, std::string* why) {
   if (!(o.tie_atol >= 0.f)) { *why = "tie_atol must be >= 0"; return false; }
   if (!(o.wait_timeout_ms > 0.f)) { *why = "wait_timeout_ms must be > 0"; return false; }
   if (o.workspace_limit_bytes < 0) { *why = "workspace_limit_bytes must be >= 0"; return false; }
+  if (o.ns_cta_pair != 0 && o.ns_cta_pair != 1) { *why = "ns_cta_pair must be 0 or 1"; return false; }
   return true;
 }
 
@@ -267,18 +268,19 @@ bool encode_map(CUtensorMap* m, void* base, int elem_bytes, int64_t inner, int64
 }
 constexpr CUtensorMapSwizzle SW128 = CU_TENSOR_MAP_SWIZZLE_128B;
 
-int sym_tiles(int tiles_m, int tiles_n) {
+// Tiles (tile_m rows x 256 columns) holding a 32 x 32 block on or above the diagonal.
+int sym_tiles(int tiles_m, int tiles_n, int tile_m) {
   int t = 0;
-  for (int tn = 0; tn < tiles_n; ++tn) t += std::min(tiles_m, 2 * (tn + 1));
+  for (int tn = 0; tn < tiles_n; ++tn) t += std::min(tiles_m, ((tn + 1) * 256) / tile_m);
   return t;
 }
 
 // tcgen05 kind::f16 instruction descriptor: D fp32, A/B fp16 (0) or bf16 (1),
-// A K-major, B K-major or MN-major, N = 256, M = 128.
-uint32_t make_idesc(bool fp16, bool b_mn_major) {
+// A K-major, B K-major or MN-major, N = 256, M = 128 (one CTA) or 256 (pair).
+uint32_t make_idesc(bool fp16, bool b_mn_major, int m) {
   const uint32_t fmt = fp16 ? 0u : 1u;
   return (1u << 4) | (fmt << 7) | (fmt << 10) | ((b_mn_major ? 1u : 0u) << 16) | ((256u >> 3) << 17) |
-         ((128u >> 4) << 24);
+         ((static_cast<uint32_t>(m) >> 4) << 24);
 }
 
 bool iter_fp16(const meq_options& o, int k) { return k < 32 && ((o.ns_fp16_mask >> k) & 1u); }
@@ -289,6 +291,9 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
   st->gemm_grid.clear();
   const int K = st->opt.ns_steps;
   const int ng = static_cast<int>(st->groups.size());
+  const int pair = st->opt.ns_cta_pair ? 2 : 1;
+  const int tile_m = 128 * pair;
+  const uint32_t b_rows = static_cast<uint32_t>(256 / pair);  // K-major B rows each CTA loads
   for (int k = 0; k < K; ++k) {
     const bool f16 = iter_fp16(st->opt, k);
     const bool next_f16 = (k + 1 < K) ? iter_fp16(st->opt, k + 1) : false;
@@ -300,7 +305,7 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
         std::memset(&P, 0, sizeof(P));
         P.mode = real_mode;
         P.b_mn_major = (mode == MODE_XUPD) ? 1 : 0;
-        P.idesc = make_idesc(f16, P.b_mn_major);
+        P.idesc = make_idesc(f16, P.b_mn_major, tile_m);
         P.ca = st->opt.ns_a, P.cb = st->opt.ns_b, P.cc = st->opt.ns_c;
         P.err = st->d_err;
         P.timeout_ns = static_cast<unsigned long long>(static_cast<double>(st->opt.wait_timeout_ms) * 1e6);
@@ -319,7 +324,7 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             Q.M = (int32_t)G.s, Q.N = (int32_t)G.s, Q.K = (int32_t)G.l;
             Q.sym = 1;
             ok &= encode_map(&Q.tmA, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 128, SW128);
-            ok &= encode_map(&Q.tmB, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 256, SW128);
+            ok &= encode_map(&Q.tmB, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, b_rows, SW128);
             Q.out = G.a16, Q.out_ld = s_ld, Q.out_mstride = s_ms;
             Q.scale = 1.0f / (ak * ak);
             Q.out_fp16 = f16;
@@ -327,7 +332,7 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             Q.M = (int32_t)G.s, Q.N = (int32_t)G.s, Q.K = (int32_t)G.s;
             Q.sym = 1;
             ok &= encode_map(&Q.tmA, G.a16, 2, G.s, G.s, G.count, G.sp, 64, 128, SW128);
-            ok &= encode_map(&Q.tmB, G.a16, 2, G.s, G.s, G.count, G.sp, 64, 256, SW128);
+            ok &= encode_map(&Q.tmB, G.a16, 2, G.s, G.s, G.count, G.sp, 64, b_rows, SW128);
             Q.out = G.p16, Q.out_ld = s_ld, Q.out_mstride = s_ms;
             Q.aux = G.a16, Q.aux_ld = s_ld, Q.aux_mstride = s_ms;
             Q.scale = 1.0f;
@@ -350,9 +355,9 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             }
           }
           if (!ok) { *why = "cuTensorMapEncodeTiled failed"; return false; }
-          Q.tiles_m = (int32_t)((Q.M + 127) / 128);
+          Q.tiles_m = (int32_t)((Q.M + tile_m - 1) / tile_m);
           Q.tiles_n = (int32_t)((Q.N + 255) / 256);
-          Q.tiles_per_mat = Q.sym ? sym_tiles(Q.tiles_m, Q.tiles_n) : Q.tiles_m * Q.tiles_n;
+          Q.tiles_per_mat = Q.sym ? sym_tiles(Q.tiles_m, Q.tiles_n, tile_m) : Q.tiles_m * Q.tiles_n;
           Q.tile_begin = tiles;
           const int64_t t = int64_t(Q.tiles_per_mat) * Q.count;
           if (tiles + t > (int64_t(1) << 30)) { *why = "too many GEMM tiles in one launch"; return false; }
@@ -364,7 +369,8 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
         // the outputs still resident in L2.
         P.reverse = (st->gemm.size() % 2 == 0) ? 1 : 0;
         st->gemm.push_back(P);
-        st->gemm_grid.push_back(std::max(1, std::min(tiles, st->num_sms)));
+        // persistent grid: one CTA (pair) per SM (pair of SMs), never more than the tiles
+        st->gemm_grid.push_back(pair * std::max(1, std::min(tiles, st->num_sms / pair)));
       }
     }
   }
@@ -389,6 +395,7 @@ void meq_default_options(meq_options* o) {
   o->use_graph = 1;
   o->workspace_limit_bytes = 0;
   o->wait_timeout_ms = 4000.f;
+  o->ns_cta_pair = 1;
 }
 
 const char* meq_status_string(meq_status s) {
@@ -441,7 +448,7 @@ meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt
   if (prop.major != 10 || prop.minor != 3)
     return fail(nullptr, MEQ_ERR_UNSUPPORTED,
                 "this library is built for sm_103a (GB300); device is sm_" + std::to_string(prop.major) + std::to_string(prop.minor));
-  if (prop.sharedMemPerBlockOptin < static_cast<size_t>(ns_gemm_smem_bytes()))
+  if (prop.sharedMemPerBlockOptin < static_cast<size_t>(ns_gemm_smem_bytes(o.ns_cta_pair ? 2 : 1)))
     return fail(nullptr, MEQ_ERR_UNSUPPORTED, "not enough opt-in shared memory per block");
   if (!get_encode()) return fail(nullptr, MEQ_ERR_UNSUPPORTED, "cuTensorMapEncodeTiled is not available from the driver");
 
@@ -564,7 +571,7 @@ static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev
   if (e != cudaSuccess) return cuda_fail(st, e, "cast_x0 launch");
   mark(2);
   for (size_t i = 0; i < st->gemm.size(); ++i) {
-    e = launch_ns_gemm(st->gemm[i], st->gemm_grid[i], s);
+    e = launch_ns_gemm(st->gemm[i], st->gemm_grid[i], st->opt.ns_cta_pair ? 2 : 1, s);
     if (e != cudaSuccess) return cuda_fail(st, e, "ns_gemm launch");
   }
   mark(3);

@@ -96,7 +96,7 @@ struct GemmParams {
 
 // Launchers (defined in the .cu files).
 cudaError_t prepare_ns_gemm();  // sets the kernel's dynamic shared-memory limit (per device)
-cudaError_t launch_ns_gemm(const GemmParams& p, int grid, cudaStream_t st);
-int ns_gemm_smem_bytes();
+cudaError_t launch_ns_gemm(const GemmParams& p, int grid, int pair, cudaStream_t st);  // pair: 1 or 2 CTAs per tile
+int ns_gemm_smem_bytes(int pair);
 
 }  // namespace meq

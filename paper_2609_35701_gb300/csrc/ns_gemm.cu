@@ -40,19 +40,31 @@
 namespace meq {
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4, UK = 16;
+constexpr int BM = 128, BN = 256, BK = 64, UK = 16;  // per-CTA rows, tile columns, k-block, MMA K
 constexpr int A_BYTES = BM * BK * 2;                 // 16 KB
-constexpr int B_BYTES = BN * BK * 2;                 // 32 KB
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;       // 48 KB
-constexpr int NUM_EPI_WARPS = 8;                    // two per TMEM lane quarter
+constexpr int NUM_EPI_WARPS = 8;                     // two per TMEM lane quarter
 constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
 constexpr uint32_t TMEM_COLS = 512;
-constexpr int SLOT_BYTES = 2048;                      // one 32 x 32 16-bit block (or 32 x 16 fp32)
-constexpr int NUM_BARS = 2 * STAGES + 4 + 1;         // full, empty, tmem full x2, tmem empty x2, drain
-constexpr int SMEM_EPI_OFF = STAGES * STAGE_BYTES;   // one staging slot per epilogue warp
-constexpr int SMEM_BAR_OFF = SMEM_EPI_OFF + NUM_EPI_WARPS * SLOT_BYTES;
-constexpr int SMEM_BYTES = SMEM_BAR_OFF + NUM_BARS * 8 + 16 + 1024;
-static_assert(SMEM_BYTES <= 232448, "shared memory budget of one sm_103a CTA");
+constexpr int SLOT_BYTES = 2048;                     // one 32 x 32 16-bit block (or 32 x 16 fp32)
+
+// kPair = 1: one CTA computes a 128 x 256 tile (tcgen05 cta_group::1).
+// kPair = 2: a cluster of two CTAs computes a 256 x 256 tile with
+// cta_group::2 MMAs: each CTA holds its own 128 rows of A and half of B
+// (128 rows / columns), so a stage is 32 KB instead of 48 KB per SM and six
+// stages fit.
+template <int kPair>
+struct Cfg {
+  static constexpr int TILE_M = BM * kPair;
+  static constexpr int BN_LOCAL = BN / kPair;
+  static constexpr int B_BYTES = BN_LOCAL * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int STAGES = kPair == 1 ? 4 : 6;
+  static constexpr int NUM_BARS = 2 * STAGES + 4 + 1;  // full, empty, tmem full x2, tmem empty x2, drain
+  static constexpr int SMEM_EPI_OFF = STAGES * STAGE_BYTES;
+  static constexpr int SMEM_BAR_OFF = SMEM_EPI_OFF + NUM_EPI_WARPS * SLOT_BYTES;
+  static constexpr int SMEM_BYTES = SMEM_BAR_OFF + NUM_BARS * 8 + 16 + 1024;
+  static_assert(SMEM_BYTES <= 232448, "shared memory budget of one sm_103a CTA");
+};
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -129,6 +141,33 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* tm,
       "l"(reinterpret_cast<uint64_t>(tm)), "r"(bar), "r"(x), "r"(y), "r"(z)
       : "memory");
 }
+// Pair variant: the copy lands in this CTA's shared memory and completes on
+// an mbarrier that may live in the peer CTA (the pair leader's).
+__device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap* tm, uint32_t bar_cluster, int x, int y,
+                                                 int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, "
+      "%5}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(bar_cluster), "r"(x), "r"(y), "r"(z)
+      : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t smem_addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* tm) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
 }
@@ -142,6 +181,24 @@ __device__ __forceinline__ void tc_mma(uint32_t d, uint64_t a, uint64_t b, uint3
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
       "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
       : "memory");
+}
+__device__ __forceinline__ void tc_mma_pair(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on the barrier at this shared-memory offset in both CTAs of the pair
+// once all prior cta_group::2 MMAs of this thread have completed.
+__device__ __forceinline__ void tc_commit_pair_both(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
+}
+__device__ __forceinline__ void tc_commit_pair_local(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
 }
 __device__ __forceinline__ void tc_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
@@ -186,8 +243,9 @@ struct TileCoord {
 // p.reverse is set, so a launch starts on the matrices its predecessor wrote
 // last, which are still in L2). Dense outputs run tm-major
 // over tiles_m x tiles_n; symmetric outputs (Gram, polynomial) run tn-major
-// over the tiles with tm < 2 (tn + 1), i.e. those holding a 32 x 32 block on
-// or above the diagonal.
+// over the tiles with tm * TILE_M < (tn + 1) * 256, i.e. those holding a
+// 32 x 32 block on or above the diagonal.
+template <int kPair>
 __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
   if (p.reverse) t = p.total_tiles - 1 - t;
   int g = 0;
@@ -205,7 +263,7 @@ __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
   } else {
     int tn = 0;
     for (;;) {
-      const int cnt = min(G.tiles_m, 2 * (tn + 1));
+      const int cnt = min(G.tiles_m, ((tn + 1) * BN) / Cfg<kPair>::TILE_M);
       if (r < cnt) break;
       r -= cnt;
       ++tn;
@@ -307,15 +365,20 @@ __device__ __forceinline__ void store_block128(const uint8_t* slot, int lane, ui
   }
 }
 
+template <int kPair>
 __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_constant__ GemmParams p) {
+  using C_ = Cfg<kPair>;
+  constexpr int STAGES = C_::STAGES;
+  constexpr int STAGE_BYTES = C_::STAGE_BYTES;
+  constexpr int TILE_M = C_::TILE_M;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
-  const uint32_t bar0 = base + SMEM_BAR_OFF;
+  const uint32_t bar0 = base + C_::SMEM_BAR_OFF;
   const uint32_t drain_bar = bar0 + 8 * (2 * STAGES + 4);
-  const uint32_t tmem_slot = bar0 + 8 * NUM_BARS;
-  volatile uint32_t* tmem_slot_ptr = reinterpret_cast<volatile uint32_t*>(gbase + SMEM_BAR_OFF + 8 * NUM_BARS);
+  const uint32_t tmem_slot = bar0 + 8 * C_::NUM_BARS;
+  volatile uint32_t* tmem_slot_ptr = reinterpret_cast<volatile uint32_t*>(gbase + C_::SMEM_BAR_OFF + 8 * C_::NUM_BARS);
 #define FULL_BAR(s) (bar0 + 8u * (s))
 #define EMPTY_BAR(s) (bar0 + 8u * (STAGES + (s)))
 #define TFULL_BAR(a) (bar0 + 8u * (2 * STAGES + (a)))
@@ -325,6 +388,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
   const int lane = threadIdx.x & 31;
   int* err = p.err;
   const uint64_t tmo = p.timeout_ns;
+  // Pair mode: rank 0 of each 2-CTA cluster issues the MMAs for both.
+  const uint32_t rank = kPair == 2 ? cluster_rank() : 0u;
+  const bool leader = rank == 0;
+  const int unit = kPair == 2 ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const int nunits = kPair == 2 ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -333,7 +401,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(TFULL_BAR(a), 1);
-      mbar_init(TEMPTY_BAR(a), NUM_EPI_WARPS);
+      mbar_init(TEMPTY_BAR(a), kPair * NUM_EPI_WARPS);
     }
     mbar_init(drain_bar, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -343,12 +411,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     }
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(tmem_slot), "r"(TMEM_COLS)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    if (kPair == 2) {
+      asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(tmem_slot), "r"(TMEM_COLS)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    } else {
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(tmem_slot), "r"(TMEM_COLS)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
   }
   tc_fence_before();
   __syncthreads();
+  if (kPair == 2) cluster_sync_all();  // both CTAs' barriers exist before either signals the other
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot_ptr;
 
@@ -359,10 +434,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       uint32_t phase = 0;
       uint32_t issued_mask = 0, issued_parity = 0;  // bit s: stage s was filled / parity of its last fill
       bool ok = true;
-      for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
-        const TileCoord c = decode_tile(p, t);
+      for (int t = unit; ok && t < p.total_tiles; t += nunits) {
+        const TileCoord c = decode_tile<kPair>(p, t);
         const GemmGroup& G = p.g[c.g];
         const int nk = (G.K + BK - 1) / BK;
+        const int arow = c.tm * TILE_M + static_cast<int>(rank) * BM;
+        const int bcol = c.tn * BN + static_cast<int>(rank) * C_::BN_LOCAL;
         for (int kb = 0; kb < nk; ++kb) {
           if (!wait_bounded(EMPTY_BAR(stage), phase ^ 1u, err, DEV_TIMEOUT_PRODUCER, tmo)) {
             ok = false;
@@ -370,14 +447,29 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
           }
           const uint32_t sa = base + stage * STAGE_BYTES;
           const uint32_t sb = sa + A_BYTES;
-          mbar_expect_tx(FULL_BAR(stage), STAGE_BYTES);
-          tma_load_3d(sa, &G.tmA, FULL_BAR(stage), kb * BK, c.tm * BM, c.mat);
-          if (!p.b_mn_major) {
-            tma_load_3d(sb, &G.tmB, FULL_BAR(stage), kb * BK, c.tn * BN, c.mat);
-          } else {
+          if (kPair == 1) {
+            mbar_expect_tx(FULL_BAR(stage), STAGE_BYTES);
+            tma_load_3d(sa, &G.tmA, FULL_BAR(stage), kb * BK, arow, c.mat);
+            if (!p.b_mn_major) {
+              tma_load_3d(sb, &G.tmB, FULL_BAR(stage), kb * BK, bcol, c.mat);
+            } else {
 #pragma unroll
-            for (int j = 0; j < BN / 64; ++j)
-              tma_load_3d(sb + j * (64 * BK * 2), &G.tmB, FULL_BAR(stage), c.tn * BN + j * 64, kb * BK, c.mat);
+              for (int j = 0; j < C_::BN_LOCAL / 64; ++j)
+                tma_load_3d(sb + j * (64 * BK * 2), &G.tmB, FULL_BAR(stage), bcol + j * 64, kb * BK, c.mat);
+            }
+          } else {
+            // Both CTAs' copies complete on the leader's full barrier, which
+            // the leader arms with the bytes of both.
+            if (leader) mbar_expect_tx(FULL_BAR(stage), 2 * STAGE_BYTES);
+            const uint32_t fb = leader ? FULL_BAR(stage) : map_to_rank(FULL_BAR(stage), 0);
+            tma_load_3d_pair(sa, &G.tmA, fb, kb * BK, arow, c.mat);
+            if (!p.b_mn_major) {
+              tma_load_3d_pair(sb, &G.tmB, fb, kb * BK, bcol, c.mat);
+            } else {
+#pragma unroll
+              for (int j = 0; j < C_::BN_LOCAL / 64; ++j)
+                tma_load_3d_pair(sb + j * (64 * BK * 2), &G.tmB, fb, bcol + j * 64, kb * BK, c.mat);
+            }
           }
           issued_mask |= 1u << stage;
           issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
@@ -387,13 +479,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
           }
         }
       }
-      // Drain: every copy this thread issued has landed before the CTA exits.
-      for (int s = 0; s < STAGES; ++s)
-        if ((issued_mask >> s) & 1u) wait_bounded(FULL_BAR(s), (issued_parity >> s) & 1u, err, DEV_TIMEOUT_DRAIN, tmo);
+      // Drain: every copy issued into this CTA has landed before it exits (for
+      // the pair, the leader's full barriers count the peer's bytes as well).
+      if (leader)
+        for (int s = 0; s < STAGES; ++s)
+          if ((issued_mask >> s) & 1u)
+            wait_bounded(FULL_BAR(s), (issued_parity >> s) & 1u, err, DEV_TIMEOUT_DRAIN, tmo);
     }
     __syncwarp();
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && leader) {
       // ---------------------------------------------------------------- MMA issuer
       int stage = 0;
       uint32_t phase = 0;
@@ -401,8 +496,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       uint32_t acc_phase = 0;
       bool ok = true;
       const uint32_t b_lbo = p.b_mn_major ? (64u * BK * 2u) : 16u;
-      for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
-        const TileCoord c = decode_tile(p, t);
+      for (int t = unit; ok && t < p.total_tiles; t += nunits) {
+        const TileCoord c = decode_tile<kPair>(p, t);
         const int nk = (p.g[c.g].K + BK - 1) / BK;
         if (!wait_bounded(TEMPTY_BAR(acc), acc_phase ^ 1u, err, DEV_TIMEOUT_MMA_TMEM, tmo)) break;
         tc_fence_after();
@@ -420,21 +515,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
             const uint64_t adesc = smem_desc(sa + k * (UK * 2), 16u, 1024u);
             const uint64_t bdesc = p.b_mn_major ? smem_desc(sb + k * (UK * 128), b_lbo, 1024u)
                                                 : smem_desc(sb + k * (UK * 2), 16u, 1024u);
-            tc_mma(d, adesc, bdesc, p.idesc, (kb > 0 || k > 0) ? 1u : 0u);
+            if (kPair == 2) tc_mma_pair(d, adesc, bdesc, p.idesc, (kb > 0 || k > 0) ? 1u : 0u);
+            else tc_mma(d, adesc, bdesc, p.idesc, (kb > 0 || k > 0) ? 1u : 0u);
           }
-          tc_commit(EMPTY_BAR(stage));
+          if (kPair == 2) tc_commit_pair_both(EMPTY_BAR(stage));
+          else tc_commit(EMPTY_BAR(stage));
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
           }
         }
         if (!ok) break;
-        tc_commit(TFULL_BAR(acc));
+        if (kPair == 2) tc_commit_pair_both(TFULL_BAR(acc));
+        else tc_commit(TFULL_BAR(acc));
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1u;
       }
       // Drain: all MMAs issued by this thread are complete before TMEM is freed.
-      tc_commit(drain_bar);
+      if (kPair == 2) tc_commit_pair_local(drain_bar);
+      else tc_commit(drain_bar);
       wait_bounded(drain_bar, 0, err, DEV_TIMEOUT_DRAIN, tmo);
     }
     __syncwarp();
@@ -448,18 +547,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     const int q = warp & 3;
     const int ew = warp - 2;
     const int half = ew >> 2;
-    uint8_t* slot = gbase + SMEM_EPI_OFF + ew * SLOT_BYTES;
+    uint8_t* slot = gbase + C_::SMEM_EPI_OFF + ew * SLOT_BYTES;
     const int mode = p.mode;
     int acc = 0;
     uint32_t acc_phase = 0;
 
-    for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
-      const TileCoord c = decode_tile(p, t);
+    // The leader's tmem-empty barrier counts the epilogue warps of both CTAs.
+    const uint32_t tempty_target0 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(0), 0) : TEMPTY_BAR(0);
+    const uint32_t tempty_target1 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(1), 0) : TEMPTY_BAR(1);
+    for (int t = unit; t < p.total_tiles; t += nunits) {
+      const TileCoord c = decode_tile<kPair>(p, t);
       const GemmGroup& G = p.g[c.g];
       if (!wait_bounded_warp(TFULL_BAR(acc), acc_phase, err, DEV_TIMEOUT_EPI, tmo)) break;
       tc_fence_after();
-      const int row0 = c.tm * BM + q * 32;
-      const int R = c.tm * 4 + q;  // 32-row block index
+      const int row0 = c.tm * TILE_M + static_cast<int>(rank) * BM + q * 32;
+      const int R = row0 / 32;  // 32-row block index
       const int rows_valid = min(32, G.M - row0);
       float rsum = 0.f;            // XLAST: this lane's row, sum of squares over the tile
       const int nch = min(BN / 32, (G.N - c.tn * BN + 31) / 32);
@@ -572,7 +674,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
         G.rpart[(static_cast<int64_t>(c.mat) * G.tiles_n * 2 + c.tn * 2 + half) * G.M + row0 + lane] = rsum;
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(TEMPTY_BAR(acc));
+      if (lane == 0) {
+        if (kPair == 2) mbar_arrive_cluster(acc == 0 ? tempty_target0 : tempty_target1);
+        else mbar_arrive(TEMPTY_BAR(acc));
+      }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
     }
@@ -582,24 +687,53 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
 #undef TFULL_BAR
 #undef TEMPTY_BAR
 
+  if (kPair == 2 && *reinterpret_cast<volatile int*>(err) != 0) {
+    // After an early exit, give copies still in flight towards either CTA
+    // time to land before the pair leaves (bounded: about 2 ms).
+    const uint64_t t0 = global_ns();
+    while (global_ns() - t0 < 2000000ull) {
+    }
+  }
   tc_fence_before();
   __syncthreads();
+  if (kPair == 2) cluster_sync_all();  // no CTA leaves while its peer may still signal it
   tc_fence_after();
   if (warp == 1) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS) : "memory");
+    if (kPair == 2)
+      asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS) : "memory");
+    else
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS) : "memory");
   }
 }
 
 }  // namespace
 
-int ns_gemm_smem_bytes() { return SMEM_BYTES; }
+int ns_gemm_smem_bytes(int pair) { return pair == 2 ? Cfg<2>::SMEM_BYTES : Cfg<1>::SMEM_BYTES; }
 
 cudaError_t prepare_ns_gemm() {
-  return cudaFuncSetAttribute(ns_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  cudaError_t e =
+      cudaFuncSetAttribute(ns_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<1>::SMEM_BYTES);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(ns_gemm_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<2>::SMEM_BYTES);
 }
 
-cudaError_t launch_ns_gemm(const GemmParams& p, int grid, cudaStream_t st) {
-  ns_gemm_kernel<<<grid, NUM_THREADS, SMEM_BYTES, st>>>(p);
+cudaError_t launch_ns_gemm(const GemmParams& p, int grid, int pair, cudaStream_t st) {
+  if (pair == 2) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
+    cfg.blockDim = dim3(NUM_THREADS, 1, 1);
+    cfg.dynamicSmemBytes = Cfg<2>::SMEM_BYTES;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, ns_gemm_kernel<2>, p);
+  }
+  ns_gemm_kernel<1><<<grid, NUM_THREADS, Cfg<1>::SMEM_BYTES, st>>>(p);
   return cudaGetLastError();
 }
 

@@ -39,6 +39,7 @@ class MeqOptions(ctypes.Structure):
         ("use_graph", ctypes.c_int),
         ("workspace_limit_bytes", ctypes.c_int64),
         ("wait_timeout_ms", ctypes.c_float),
+        ("ns_cta_pair", ctypes.c_int),
     ]
 
 

@@ -64,12 +64,14 @@ def test_single256_one_step(meq):
     [(257, 513), (513, 257), (64, 1000), (1000, 64)],
     [(384, 768), (768, 384), (768, 768), (129, 385)],
 ])
-def test_ragged_shapes_two_steps(meq, shapes):
+@pytest.mark.parametrize("pair", [1, 0], ids=["cta_pair", "single_cta"])
+def test_ragged_shapes_two_steps(meq, shapes, pair):
     """Several tiles plus ragged tails in every GEMM dimension, tiny and
-    degenerate shapes, tall / wide / square, two steps (nonzero momentum)."""
+    degenerate shapes, tall / wide / square, two steps (nonzero momentum), on
+    both NS GEMM variants (CTA-pair and single-CTA tiles)."""
     wl = W.custom_workload(shapes, pattern="both", base_sigma=0.01, seed=11)
     rep = []
-    run_staged(meq, wl, 2, report=rep)
+    run_staged(meq, wl, 2, report=rep, ns_cta_pair=pair)
     assert all(r["update"] <= PT.UPDATE_TOL for r in rep)
 
 
@@ -166,6 +168,23 @@ def test_checkpoint_resume_bitwise(meq):
         assert np.array_equal(x.cpu().numpy(), y.cpu().numpy())
     a.close()
     c.close()
+
+
+def test_single_cta_and_pair_agree(meq):
+    """The two NS GEMM variants compute the same products; their updates agree
+    to fp32 / 16-bit rounding."""
+    wl = W.custom_workload([(768, 768), (768, 2048), (2048, 768)], pattern="both", seed=6)
+    shapes = [(r, c) for _, r, c in wl.shapes]
+    outs = []
+    for pair in (1, 0):
+        o = meq.MeqMuon(shapes, ns_cta_pair=pair)
+        p = _to_dev(W.initial_weights(wl))
+        o.step(p, _to_dev(W.gradients(wl, 0)), LR, MU, WD, EPS)
+        o.sync()
+        outs.append([o.read_ns_output(i) for i in range(len(shapes))])
+        o.close()
+    for a, b in zip(*outs):
+        assert PT.rel_frob(a, b) < 2e-3
 
 
 def test_graph_and_direct_launch_bitwise(meq):
