@@ -15,8 +15,7 @@
  *
  * Everything runs in the library's own CUDA kernels, asynchronously on the
  * caller's stream. Newton-Schulz runs on the tensor cores (tcgen05, TMA, TMEM)
- * with 16-bit operands and fp32 accumulation; all other arithmetic is fp32
- * (CV statistics in fp64).
+ * with 16-bit operands and fp32 accumulation; all other arithmetic is fp32.
  *
  * Conventions shared by every call:
  *   - Matrices are fp32, row-major, contiguous, rows = output features and
@@ -160,9 +159,9 @@ meq_status meq_debug_wait_selftest(meq_state* st, float timeout_ms);
  * gamma_r and gammas[1] = gamma_c of Eq. (8) over entries > eps, and
  * *direction of Eq. (11) (0 = row, 1 = column; row when gamma_r >= gamma_c -
  * tie_atol). All outputs are caller-provided device memory. The definitions
- * and precision (fp32 sums of squares, fp64 CVs) are those of meq_step's
- * statistics, so results agree with meq_read_stats for the same U up to fp32
- * summation order.
+ * and precision (fp32 sums of squares and two-pass fp32 CVs) are those of
+ * meq_step's statistics, so results agree with meq_read_stats for the same U
+ * up to fp32 summation order.
  *
  * It allocates nothing. Its scratch is a fixed 8 MiB __device__ array inside
  * the library, held by every GPU that loads the library until the process

@@ -2,12 +2,12 @@
 //
 //   momentum_norm : B <- mu B + G (Eq. (10)) in place over every matrix, with
 //                   deterministic per-chunk partial sums of the squared NS
-//                   input; the last chunk of each matrix reduces them (fp64)
-//                   into the X_0 scale alpha0 / ||H||_F of Eq. (5).
+//                   input; the last chunk of each matrix reduces them into the
+//                   X_0 scale alpha0 / ||H||_F of Eq. (5).
 //   cast_x0       : X-hat_0 = 16-bit(alpha0 H / ||H||_F) in the oriented NS
 //                   layout (transposed through shared memory for tall W).
 //   finalize      : r, c (Eq. (7)) from the partial sums of squares the last
-//                   NS epilogue wrote, gamma_r, gamma_c (Eq. (8), fp64), the
+//                   NS epilogue wrote, gamma_r, gamma_c (Eq. (8)), the
 //                   direction (Eq. (11)) and the scale vector of Eq. (9).
 //   apply         : W <- (1 - lr wd) W - rho lr s (.) U (Eq. (14)).
 #include "meq_elementwise.cuh"
@@ -45,23 +45,6 @@ __device__ __forceinline__ float block_sum_f32(float v, float* sh) {
   return sh[0];
 }
 
-__device__ __forceinline__ double block_sum_f64(double v, double* sh) {
-  const unsigned FULL = 0xffffffffu;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL, v, o);
-  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
-  __syncthreads();
-  if (l == 0) sh[w] = v;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    double r = 0.0;
-    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) r += sh[i];
-    sh[0] = r;
-  }
-  __syncthreads();
-  return sh[0];
-}
-
 // ------------------------------------------------------------- momentum + norm
 __global__ void __launch_bounds__(kThreads) momentum_norm_kernel(const MatInfo* __restrict__ mats, int nmat,
                                                                  const GroupInfo* __restrict__ groups,
@@ -71,7 +54,8 @@ __global__ void __launch_bounds__(kThreads) momentum_norm_kernel(const MatInfo* 
                                                                  float* __restrict__ partials,
                                                                  unsigned int* __restrict__ counters,
                                                                  float* __restrict__ x0scale) {
-  __shared__ double shd[32];
+  pdl_allow_dependents();
+  pdl_wait_predecessor();
   __shared__ float shf[32];
   __shared__ int is_last;
   const int64_t chunk = blockIdx.x;
@@ -120,16 +104,16 @@ __global__ void __launch_bounds__(kThreads) momentum_norm_kernel(const MatInfo* 
   __syncthreads();
   if (!is_last) return;
   __threadfence();
-  // Last chunk of this matrix: fixed-order fp64 reduction of its partials.
+  // Last chunk of this matrix: fixed-order fp32 reduction of its partials
+  // (fp32 throughout: this GPU's fp64 rate is a small fraction of its fp32 rate).
   const int64_t nchunks = (numel + kChunk - 1) / kChunk;
-  double acc = 0.0;
-  for (int64_t c = threadIdx.x; c < nchunks; c += kThreads) acc += static_cast<double>(__ldcg(partials + M.chunk_begin + c));
-  const double total = block_sum_f64(acc, shd);
+  float acc = 0.f;
+  for (int64_t c = threadIdx.x; c < nchunks; c += kThreads) acc += __ldcg(partials + M.chunk_begin + c);
+  const float total = block_sum_f32(acc, shf);
   if (threadIdx.x == 0) {
-    const double nrm = sqrt(total);
-    const double alpha0 = static_cast<double>(groups[M.group].alpha0);
+    const float nrm = sqrtf(total);
     // Zero input: U = 0 (Eq. (5) is defined for a nonzero input only).
-    x0scale[mi] = nrm > 0.0 ? static_cast<float>(alpha0 / nrm) : 0.f;
+    x0scale[mi] = nrm > 0.f ? groups[M.group].alpha0 / nrm : 0.f;
     counters[mi] = 0u;
   }
 }
@@ -169,6 +153,8 @@ __global__ void __launch_bounds__(kThreads) cast_x0_kernel(const MatInfo* __rest
                                                            const float* const* __restrict__ grads,
                                                            const StepScalars* __restrict__ sc,
                                                            const float* __restrict__ x0scale) {
+  pdl_allow_dependents();
+  pdl_wait_predecessor();
   __shared__ float tile[kCastTile][kCastTile + 1];
   const int64_t t = blockIdx.x;
   const int mi = find_mat(mats, nmat, t, 1);
@@ -257,7 +243,9 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
                                                                float* __restrict__ rvec, float* __restrict__ cvec,
                                                                float* __restrict__ svec,
                                                                MatStats* __restrict__ stats) {
-  __shared__ double shd[32];
+  pdl_allow_dependents();
+  pdl_wait_predecessor();
+  __shared__ float shf[32];
   const MatInfo& M = mats[blockIdx.x];
   const float delta = sc->eps;
   float* r = rvec + M.vec_off;
@@ -281,27 +269,29 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
     else r[j] = sqrtf(acc * inv_n);
   }
   __syncthreads();
-  double gam[2];
+  // Eq. (8) over entries > delta: two passes (mean, then squared deviations),
+  // fp32 with fixed-order block reductions.
+  float gam[2];
   for (int side = 0; side < 2; ++side) {
     const float* v = side == 0 ? r : c;
     const int64_t len = side == 0 ? M.m : M.n;
-    double cnt = 0.0, sum = 0.0;
+    float cnt = 0.f, sum = 0.f;
     for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
       const float x = v[i];
-      if (x > delta) cnt += 1.0, sum += static_cast<double>(x);
+      if (x > delta) cnt += 1.f, sum += x;
     }
-    cnt = block_sum_f64(cnt, shd);
-    sum = block_sum_f64(sum, shd);
-    const double mean = cnt > 0.0 ? sum / cnt : 0.0;
-    double var = 0.0;
+    cnt = block_sum_f32(cnt, shf);
+    sum = block_sum_f32(sum, shf);
+    const float mean = cnt > 0.f ? sum / cnt : 0.f;
+    float var = 0.f;
     for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
-      const double x = static_cast<double>(v[i]);
-      if (v[i] > delta) var += (x - mean) * (x - mean);
+      const float x = v[i];
+      if (x > delta) var += (x - mean) * (x - mean);
     }
-    var = block_sum_f64(var, shd);
-    gam[side] = cnt > 0.0 ? sqrt(var / cnt) / mean : 0.0;
+    var = block_sum_f32(var, shf);
+    gam[side] = cnt > 0.f ? sqrtf(var / cnt) / mean : 0.f;
   }
-  const int dir = gam[0] >= gam[1] - static_cast<double>(sc->tie_atol) ? 0 : 1;
+  const int dir = gam[0] >= gam[1] - sc->tie_atol ? 0 : 1;
   const float* v = dir == 0 ? r : c;
   const int64_t len = dir == 0 ? M.m : M.n;
   for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
@@ -309,8 +299,8 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
     s[i] = x > delta ? 1.0f / x : 0.0f;   // RMS at or below delta: treated as zero
   }
   if (threadIdx.x == 0) {
-    stats[blockIdx.x].gamma_r = gam[0];
-    stats[blockIdx.x].gamma_c = gam[1];
+    stats[blockIdx.x].gamma_r = static_cast<double>(gam[0]);
+    stats[blockIdx.x].gamma_c = static_cast<double>(gam[1]);
     stats[blockIdx.x].direction = dir;
   }
 }
@@ -322,6 +312,8 @@ __global__ void __launch_bounds__(kThreads) apply_kernel(const MatInfo* __restri
                                                          const float* __restrict__ svec,
                                                          const MatStats* __restrict__ stats,
                                                          const StepScalars* __restrict__ sc) {
+  pdl_allow_dependents();
+  pdl_wait_predecessor();
   const int64_t chunk = blockIdx.x;
   const int mi = find_mat(mats, nmat, chunk, 0);
   const MatInfo& M = mats[mi];
@@ -381,29 +373,27 @@ __global__ void wait_selftest_kernel(const volatile int* flag, int* err, unsigne
 }  // namespace
 
 cudaError_t launch_momentum_norm(const LaunchCtx& L, cudaStream_t st) {
-  momentum_norm_kernel<<<(unsigned)L.total_chunks, kThreads, 0, st>>>(L.mats, L.nmat, L.groups, L.mom, L.grads, L.sc,
-                                                                    L.partials, L.counters, L.x0scale);
-  return cudaGetLastError();
+  return launch_pdl(momentum_norm_kernel, dim3((unsigned)L.total_chunks), dim3(kThreads), 0, st, 1, L.mats, L.nmat,
+                    L.groups, L.mom, L.grads, L.sc, L.partials, L.counters, L.x0scale);
 }
 
 cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st) {
   if (fp16)
-    cast_x0_kernel<true><<<(unsigned)L.total_tiles, kThreads, 0, st>>>(L.mats, L.nmat, L.groups, L.mom, L.grads, L.sc,
-                                                                      L.x0scale);
-  else
-    cast_x0_kernel<false><<<(unsigned)L.total_tiles, kThreads, 0, st>>>(L.mats, L.nmat, L.groups, L.mom, L.grads, L.sc,
-                                                                       L.x0scale);
-  return cudaGetLastError();
+    return launch_pdl(cast_x0_kernel<true>, dim3((unsigned)L.total_tiles), dim3(kThreads), 0, st, 1, L.mats, L.nmat,
+                      L.groups, static_cast<const float*>(L.mom), L.grads, L.sc, static_cast<const float*>(L.x0scale));
+  return launch_pdl(cast_x0_kernel<false>, dim3((unsigned)L.total_tiles), dim3(kThreads), 0, st, 1, L.mats, L.nmat,
+                    L.groups, static_cast<const float*>(L.mom), L.grads, L.sc, static_cast<const float*>(L.x0scale));
 }
 
 cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st) {
-  finalize_kernel<<<L.nmat, kFinThreads, 0, st>>>(L.mats, L.sc, L.parts, L.rvec, L.cvec, L.svec, L.stats);
-  return cudaGetLastError();
+  return launch_pdl(finalize_kernel, dim3(L.nmat), dim3(kFinThreads), 0, st, 1, L.mats, L.sc,
+                    static_cast<const float*>(L.parts), L.rvec, L.cvec, L.svec, L.stats);
 }
 
 cudaError_t launch_apply(const LaunchCtx& L, cudaStream_t st) {
-  apply_kernel<<<(unsigned)L.total_chunks, kThreads, 0, st>>>(L.mats, L.nmat, L.params, L.uslab, L.svec, L.stats, L.sc);
-  return cudaGetLastError();
+  return launch_pdl(apply_kernel, dim3((unsigned)L.total_chunks), dim3(kThreads), 0, st, 1, L.mats, L.nmat, L.params,
+                    static_cast<const float*>(L.uslab), static_cast<const float*>(L.svec),
+                    static_cast<const MatStats*>(L.stats), L.sc);
 }
 
 cudaError_t launch_wait_selftest(const int* flag, int* err, unsigned long long timeout_ns, cudaStream_t st) {

@@ -10,9 +10,9 @@
 // file-scope __device__ array of fixed size that every GPU which loads the
 // library holds until the process exits.
 //
-// It sums squares in fp32 over 32-row slabs and forms the CVs in fp64, the
-// same definitions and precision as the full step's statistics, so results
-// agree with meq_read_stats up to fp32 summation order.
+// It sums squares over 32-row slabs and forms the CVs in two passes, all in
+// fp32 like the full step's statistics, so results agree with meq_read_stats
+// up to fp32 summation order.
 #include <mutex>
 
 #include "../../include/meq.h"
@@ -33,7 +33,7 @@ static __device__ __align__(256) float g_stats_scratch[kScratchFloats];
 std::mutex g_setup_mu;
 float* g_scratch_addr[kMaxDevices] = {nullptr};
 
-__device__ __forceinline__ double na_block_sum_f64(double v, double* sh) {
+__device__ __forceinline__ float na_block_sum_f32(float v, float* sh) {
   const unsigned FULL = 0xffffffffu;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL, v, o);
@@ -42,7 +42,7 @@ __device__ __forceinline__ double na_block_sum_f64(double v, double* sh) {
   if (l == 0) sh[w] = v;
   __syncthreads();
   if (threadIdx.x == 0) {
-    double r = 0.0;
+    float r = 0.f;
     for (int i = 0; i < (int)(blockDim.x >> 5); ++i) r += sh[i];
     sh[0] = r;
   }
@@ -98,13 +98,13 @@ __global__ void __launch_bounds__(kNaThreads) na_stats_kernel(const float* __res
   }
 }
 
-// r, c (Eq. (7)), gamma_r, gamma_c (Eq. (8), fp64) and the side (Eq. (11)).
+// r, c (Eq. (7)), gamma_r, gamma_c (Eq. (8)) and the side (Eq. (11)), all fp32.
 __global__ void __launch_bounds__(kNaFinThreads) na_finalize_kernel(int64_t m, int64_t n, float delta, float tie_atol,
                                                                     const float* __restrict__ scratch,
                                                                     float* __restrict__ r, float* __restrict__ c,
                                                                     double* __restrict__ gammas,
                                                                     int* __restrict__ direction) {
-  __shared__ double shd[32];
+  __shared__ float shf[32];
   const int64_t nslabs = (m + kNaSlab - 1) / kNaSlab;
   const float* rowss = scratch;
   const float* cpart = scratch + m;
@@ -117,30 +117,30 @@ __global__ void __launch_bounds__(kNaFinThreads) na_finalize_kernel(int64_t m, i
     c[j] = sqrtf(acc * inv_m);
   }
   __syncthreads();
-  double gam[2];
+  float gam[2];
   for (int side = 0; side < 2; ++side) {
     const float* v = side == 0 ? r : c;
     const int64_t len = side == 0 ? m : n;
-    double cnt = 0.0, sum = 0.0;
+    float cnt = 0.f, sum = 0.f;
     for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
       const float x = v[i];
-      if (x > delta) cnt += 1.0, sum += static_cast<double>(x);
+      if (x > delta) cnt += 1.f, sum += x;
     }
-    cnt = na_block_sum_f64(cnt, shd);
-    sum = na_block_sum_f64(sum, shd);
-    const double mean = cnt > 0.0 ? sum / cnt : 0.0;
-    double var = 0.0;
+    cnt = na_block_sum_f32(cnt, shf);
+    sum = na_block_sum_f32(sum, shf);
+    const float mean = cnt > 0.f ? sum / cnt : 0.f;
+    float var = 0.f;
     for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
-      const double x = static_cast<double>(v[i]);
-      if (v[i] > delta) var += (x - mean) * (x - mean);
+      const float x = v[i];
+      if (x > delta) var += (x - mean) * (x - mean);
     }
-    var = na_block_sum_f64(var, shd);
-    gam[side] = cnt > 0.0 ? sqrt(var / cnt) / mean : 0.0;
+    var = na_block_sum_f32(var, shf);
+    gam[side] = cnt > 0.f ? sqrtf(var / cnt) / mean : 0.f;
   }
   if (threadIdx.x == 0) {
-    gammas[0] = gam[0];
-    gammas[1] = gam[1];
-    *direction = gam[0] >= gam[1] - static_cast<double>(tie_atol) ? 0 : 1;
+    gammas[0] = static_cast<double>(gam[0]);
+    gammas[1] = static_cast<double>(gam[1]);
+    *direction = gam[0] >= gam[1] - tie_atol ? 0 : 1;
   }
 }
 

@@ -426,6 +426,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
   if (kPair == 2) cluster_sync_all();  // both CTAs' barriers exist before either signals the other
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot_ptr;
+  pdl_allow_dependents();
+  pdl_wait_predecessor();  // operands come from the previous kernel of the step
 
   if (warp == 0) {
     if (lane == 0) {
@@ -718,23 +720,9 @@ cudaError_t prepare_ns_gemm() {
 }
 
 cudaError_t launch_ns_gemm(const GemmParams& p, int grid, int pair, cudaStream_t st) {
-  if (pair == 2) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
-    cfg.blockDim = dim3(NUM_THREADS, 1, 1);
-    cfg.dynamicSmemBytes = Cfg<2>::SMEM_BYTES;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, ns_gemm_kernel<2>, p);
-  }
-  ns_gemm_kernel<1><<<grid, NUM_THREADS, Cfg<1>::SMEM_BYTES, st>>>(p);
-  return cudaGetLastError();
+  if (pair == 2)
+    return launch_pdl(ns_gemm_kernel<2>, dim3(grid), dim3(NUM_THREADS), Cfg<2>::SMEM_BYTES, st, 2, p);
+  return launch_pdl(ns_gemm_kernel<1>, dim3(grid), dim3(NUM_THREADS), Cfg<1>::SMEM_BYTES, st, 1, p);
 }
 
 }  // namespace meq
