@@ -1,0 +1,116 @@
+"""Full-size model workloads on the GPU: the Llama-350M and 1B-class hidden
+sets against the fp64 oracle on sampled matrices, the 7B-class set through
+properties that hold at any size (the oracle's fp64 NS on 4096 x 11008 takes
+minutes per matrix on the host)."""
+import gc
+
+import numpy as np
+import pytest
+
+import parity as PT
+from oracle import meqmuon as O
+from paper_2609_35701_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+LR, MU, WD, EPS = 0.02, 0.95, 0.1, 1e-7
+
+
+@pytest.fixture(scope="module")
+def meq():
+    import __graft_entry__
+
+    __graft_entry__.build()
+    from paper_2609_35701_gb300 import meq as m
+
+    return m
+
+
+def _release():
+    import torch
+
+    gc.collect()
+    torch.cuda.empty_cache()
+
+
+def _run(meq, name, steps, check_steps, check_names, oracle=True):
+    import torch
+
+    wl = W.get_workload(name)
+    names = [n for n, _, _ in wl.shapes]
+    pick = [names.index(n) for n in check_names]
+    shapes = [(r, c) for _, r, c in wl.shapes]
+    opt = meq.MeqMuon(shapes)
+    params = W.initial_weights(wl, device="cuda")
+    scales = W.scale_table(wl, device="cuda")
+    B_prev = {i: np.zeros(shapes[i]) for i in pick}
+    rep = []
+    for t in range(steps):
+        grads = W.gradients(wl, t, device="cuda", scale_cache=scales)
+        checking = t in check_steps
+        if checking:
+            W0 = {i: params[i].cpu().double().numpy() for i in pick}
+            G = {i: grads[i].cpu().double().numpy() for i in pick}
+            if t > 0:
+                opt.sync()
+                B_prev = {i: opt.read_momentum(i).astype(np.float64) for i in pick}
+        opt.step(params, grads, LR, MU, WD, EPS)
+        opt.sync()
+        if checking:
+            for i in pick:
+                U = opt.read_ns_output(i)
+                st = opt.read_stats(i)
+                W1 = params[i].cpu().numpy()
+                B = opt.read_momentum(i)
+                if oracle:
+                    PT.check_step(W0[i], G[i], B_prev[i], W1, B, U, st, LR, MU, WD, EPS, report=rep)
+                else:
+                    check_properties(W0[i], G[i], B_prev[i], W1, B, U, st, rep)
+        del grads
+    opt.close()
+    del params
+    _release()
+    return rep
+
+
+def check_properties(W0, G, B_prev, W1, B, U, st, rep):
+    """What holds at any size: Eq. (10) momentum; statistics of the GPU's own U
+    (Eqs. (7), (8), (11)); unit RMS on the chosen side after Eq. (9); the
+    update applied by Eq. (14) equals the normalised U; NS output finite and
+    inside the band the quintic keeps singular values in (Frobenius bound)."""
+    out = {"momentum": PT.max_rel(B, O.momentum_update(B_prev, G, MU), floor_frac=1.0)}
+    assert out["momentum"] <= PT.MOMENTUM_TOL
+    Ug = U.astype(np.float64)
+    assert np.all(np.isfinite(Ug))
+    r, c = O.row_col_rms(Ug)
+    assert PT.max_rel(st["r"], r, 1e-6) <= PT.STATS_TOL and PT.max_rel(st["c"], c, 1e-6) <= PT.STATS_TOL
+    gr, gc_ = O.coefficient_of_variation(r), O.coefficient_of_variation(c)
+    assert abs(st["gamma_r"] - gr) <= PT.STATS_TOL * max(gr, 1e-6)
+    assert abs(st["gamma_c"] - gc_) <= PT.STATS_TOL * max(gc_, 1e-6)
+    Ut = PT.staged_update(Ug, st["direction"])
+    assert PT.max_rel(W1, O.apply_update(W0, Ut, LR, WD), floor_frac=1.0) <= PT.PARAM_TOL
+    applied = PT.gpu_update_from_params(W0, W1, LR, WD)
+    rms = np.sqrt((applied ** 2).mean(axis=1 if st["direction"] == O.ROW else 0))
+    assert np.abs(rms - 1.0).max() < 2e-4
+    # singular values of U lie in [0, 1.21] (Section 2 coefficients), so
+    # ||U||_F^2 <= 1.21^2 * min(m, n)
+    assert (Ug ** 2).sum() <= 1.21 ** 2 * min(Ug.shape) * (1 + 1e-3)
+    rep.append(out)
+
+
+def test_llama350m_full_size_sampled(meq):
+    names = [f"layers.{l}.{m}" for l in (0, 23) for m in ("q_proj", "down_proj")]
+    rep = _run(meq, "llama350m", 10, {0, 4, 9}, names)
+    assert len(rep) == 12 and max(r["update"] for r in rep) <= PT.UPDATE_TOL
+
+
+def test_llama1b_full_size_sampled(meq):
+    names = ["layers.0.q_proj", "layers.0.down_proj"]
+    rep = _run(meq, "llama1b", 10, {9}, names)
+    assert len(rep) == 2 and max(r["update"] for r in rep) <= PT.UPDATE_TOL
+
+
+def test_llama7b_full_size_properties(meq):
+    names = [f"layers.{l}.{m}" for l in (0, 31) for m in ("q_proj", "o_proj", "gate_proj", "down_proj")]
+    rep = _run(meq, "llama7b", 5, {0, 4}, names, oracle=False)
+    assert len(rep) == 16
