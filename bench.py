@@ -74,9 +74,12 @@ def ns_flops(s, l, K):
     return sym, dense
 
 
-def partition(shapes, world, K=5):
-    """Greedy flop-balanced split of matrix indices over ranks."""
-    w = [(ns_flops(min(r, c), max(r, c), K)[0], i) for i, (r, c) in enumerate(shapes)]
+def partition(shapes, world, K=5, kinds=None):
+    """Greedy flop-balanced split of matrix indices over ranks (entries that
+    are not hidden weights carry no NS work and are weighted by size)."""
+    kinds = kinds or [0] * len(shapes)
+    w = [(ns_flops(min(r, c), max(r, c), K)[0] if k == 0 else 24 * r * c, i)
+         for i, ((r, c), k) in enumerate(zip(shapes, kinds))]
     w.sort(reverse=True)
     load = [0] * world
     parts = [[] for _ in range(world)]
@@ -145,20 +148,21 @@ def oracle_sample(wl, seed_step=0, max_per_class=1):
     from paper_2609_35701_gb300 import workloads as W
 
     classes = {}
+    kinds = wl.kind_list()
     for i, (_, r, c) in enumerate(wl.shapes):
-        classes.setdefault((r, c), []).append(i)
+        classes.setdefault((r, c, kinds[i]), []).append(i)
     total_ms = 0.0
     sampled = []
-    for (r, c), idx in classes.items():
+    for (r, c, k), idx in classes.items():
         i = idx[0]
         G = W.gradient(wl, i, seed_step).double().numpy()
         W0 = np.zeros((r, c))
         Bp = np.zeros((r, c))
         t0 = time.perf_counter()
-        O.hidden_step(W0, G, Bp, LR, MU, WD, eps=EPS)
+        O.param_step(k, W0, G, Bp, LR, MU, WD, eps=EPS)
         dt = (time.perf_counter() - t0) * 1e3
         total_ms += dt * len(idx)
-        sampled.append(f"{r}x{c}")
+        sampled.append(f"{r}x{c}" + ("" if k == 0 else ("/2-sided" if k == 1 else "/vector")))
     return total_ms, sampled
 
 
@@ -236,8 +240,10 @@ def main():
     from paper_2609_35701_gb300 import workloads as W
 
     wl = W.get_workload(args.workload)
-    mine = partition([(r, c) for _, r, c in wl.shapes], world)[rank]
+    mine = partition([(r, c) for _, r, c in wl.shapes], world, kinds=wl.kind_list())[rank]
     shapes = [(wl.shapes[i][1], wl.shapes[i][2]) for i in mine]
+    all_kinds = wl.kind_list()
+    kinds = [all_kinds[i] for i in mine]
     dev = torch.device("cuda", local)
 
     # Flat, 256-byte aligned device buffers with one view per matrix.
@@ -267,7 +273,7 @@ def main():
     params = [v.view(r, c) for v, (r, c) in zip(pviews, shapes)]
     grads = [[v.view(r, c) for v, (r, c) in zip(gv, shapes)] for _, gv in gbufs]
 
-    opt = meq.MeqMuon(shapes, ns_fp16_mask=args.ns_fp16_mask)
+    opt = meq.MeqMuon(shapes, kinds=kinds, ns_fp16_mask=args.ns_fp16_mask)
     stream = torch.cuda.current_stream()
     for k in range(args.warmup):
         opt.step(params, grads[k % 2], LR, MU, WD, EPS)
@@ -309,15 +315,19 @@ def main():
     ph = {k: v / max(nprof, 1) for k, v in phases.items()}
 
     K = 5
-    sym = sum(ns_flops(min(r, c), max(r, c), K)[0] for r, c in shapes)
-    dense = sum(ns_flops(min(r, c), max(r, c), K)[1] for r, c in shapes)
-    n_gemm_launches = opt.kernels_per_step - 4  # all but momentum, cast, finalize, apply
+    hid = [sh for sh, k in zip(shapes, kinds) if k == W.HIDDEN]   # Newton-Schulz runs on hidden weights only
+    sym = sum(ns_flops(min(r, c), max(r, c), K)[0] for r, c in hid)
+    dense = sum(ns_flops(min(r, c), max(r, c), K)[1] for r, c in hid)
+    n_gemm_launches = opt.ns_gemm_launches_per_step
     peaks, peak_src = load_peaks()
     ns_tflops = sym / (ph["ns_gemm"] * 1e-3) / 1e12
     ns_dense_tflops = dense / (ph["ns_gemm"] * 1e-3) / 1e12
     numel = sum(nums)
+    # algorithmic bytes of the bandwidth phases: 24 B / element, plus the
+    # column pass over the momentum (4 B) for the remaining 2D parameters
+    bw_bytes = sum((BW_BYTES_PER_ELEM + (4 if k == W.REMAINING_2D else 0)) * r * c for (r, c), k in zip(shapes, kinds))
     bw_ms = ph["momentum"] + ph["cast_x0"] + ph["stats"] + ph["apply"]
-    bw_gbs = BW_BYTES_PER_ELEM * numel / (bw_ms * 1e-3) / 1e9
+    bw_gbs = bw_bytes / (bw_ms * 1e-3) / 1e9
 
     # ---------------- end to end through the public API with host buffers
     e2e = None
@@ -383,7 +393,7 @@ def main():
             },
             "bandwidth_kernels": {
                 "bound": "hbm", "achieved": bw_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                "frac": bw_gbs / peaks["hbm_gbs"], "bytes_per_elem": BW_BYTES_PER_ELEM,
+                "frac": bw_gbs / peaks["hbm_gbs"], "bytes_per_step": bw_bytes,
                 "phase_ms": {k: round(v, 4) for k, v in ph.items()},
             },
             "gpu_launches": opt.kernels_per_step * args.steps,

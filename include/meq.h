@@ -70,6 +70,13 @@ typedef struct {
                              256 x 256 tiles on two SMs); 0: one CTA per 128 x 256 tile */
 } meq_options;
 
+/* Parameter type, selecting the branch of Algorithm 1 applied to it. */
+typedef enum {
+  MEQ_KIND_HIDDEN = 0,       /* 2D weight in a hidden layer: NS, then Eq. (11) (default) */
+  MEQ_KIND_REMAINING_2D = 1, /* token embedding / LM head: N_c(N_r(B_t)), Eq. (12) */
+  MEQ_KIND_VECTOR = 2        /* 1D parameter, given as shape (1, d): B_t / (||B_t||/sqrt(d)), Eq. (13) */
+} meq_kind;
+
 typedef struct meq_state meq_state; /* opaque */
 
 void meq_default_options(meq_options* opt);
@@ -81,12 +88,24 @@ void meq_default_options(meq_options* opt);
 meq_status meq_state_bytes(const meq_shape* shapes, int n, const meq_options* opt,
                            size_t* persistent_bytes, size_t* workspace_bytes);
 
+/* As meq_state_bytes, with a parameter type per entry (kinds may be NULL:
+ * all MEQ_KIND_HIDDEN). MEQ_KIND_VECTOR entries must have rows == 1. */
+meq_status meq_state_bytes_kinds(const meq_shape* shapes, const int* kinds, int n, const meq_options* opt,
+                                 size_t* persistent_bytes, size_t* workspace_bytes);
+
 /* Create the state for n matrices: zeroed momentum (B_{-1} = 0, Algorithm 1)
  * and the workspace, on the current CUDA device. opt may be NULL (defaults).
  * cuda_stream (cudaStream_t, may be NULL) orders the zero-fill. The shape
  * list is copied. On success *out owns device memory until meq_free. */
 meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt,
                           void* cuda_stream, meq_state** out);
+
+/* As meq_init_state, with a parameter type (meq_kind) per entry, so one state
+ * runs Algorithm 1 over every trainable parameter of a model: hidden 2D
+ * weights, the remaining 2D parameters and 1D parameters (shape (1, d)).
+ * kinds is copied; NULL means all MEQ_KIND_HIDDEN. */
+meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n,
+                                const meq_options* opt, void* cuda_stream, meq_state** out);
 
 /* One MeqMuon step over all n matrices (Algorithm 1, hidden branch).
  *   params[i]: device fp32 W_i (rows x cols), updated in place.
@@ -120,22 +139,28 @@ meq_status meq_read_momentum(meq_state* st, int i, float* dst);
 /* Overwrite momentum B_i from src (host or device), e.g. to resume. */
 meq_status meq_write_momentum(meq_state* st, int i, const float* src);
 /* Copy the last step's Newton-Schulz output U_i (rows x cols fp32, before
- * equilibration) to dst (host or device). */
+ * equilibration) to dst (host or device). Hidden weights only. */
 meq_status meq_read_ns_output(meq_state* st, int i, float* dst);
-/* Last step's statistics of U_i: r (rows floats), c (cols floats) of Eq. (7),
- * gamma_r, gamma_c of Eq. (8) and the direction of Eq. (11) (0 = row,
- * 1 = column). Any output may be NULL; r and c are host or device memory. */
+/* Last step's statistics of entry i. Hidden weight: r (rows floats), c (cols
+ * floats) of Eq. (7) for U, gamma_r, gamma_c of Eq. (8) and the direction of
+ * Eq. (11) (0 = row, 1 = column). Remaining 2D parameter: r = row RMS of
+ * B_t, c = column RMS of N_r(B_t), their CVs, direction 2. Vector: r[0] =
+ * RMS of B_t, gammas 0, direction 3. Any output may be NULL; r and c are
+ * host or device memory. */
 meq_status meq_read_stats(meq_state* st, int i, float* r, float* c,
                           double* gamma_r, double* gamma_c, int* direction);
-/* Number of kernels one meq_step launches (for launch accounting). */
+/* Number of kernels one meq_step launches (for launch accounting), and how
+ * many of them are Newton-Schulz GEMM launches. */
 int meq_kernels_per_step(const meq_state* st);
+int meq_ns_gemm_launches_per_step(const meq_state* st);
 
 /* Per-phase timing with CUDA events on the launch stream. While enabled,
  * meq_step launches its kernels directly (not from the CUDA graph) and
  * records an event between phases. meq_read_profile synchronises and returns
  * the summed milliseconds of each phase since profiling was enabled:
- *   phase_ms[0] momentum update + norms, [1] X_0 cast, [2] all NS GEMMs,
- *   [3] statistics + direction, [4] apply; *steps = profiled steps. */
+ *   phase_ms[0] momentum update + norms (all kinds), [1] X_0 cast,
+ *   [2] all NS GEMMs, [3] statistics + direction / scales, [4] apply;
+ *   *steps = profiled steps. */
 meq_status meq_set_profiling(meq_state* st, int enable);
 meq_status meq_read_profile(meq_state* st, double* phase_ms /* 5 */, int64_t* steps);
 

@@ -20,6 +20,7 @@ Equation numbers are the paper's:
   Eq. (11) adaptive one-sided selection              (Section 3.2)
   Eq. (12) two-sided normalisation                   (Section 3.2)
   Eq. (13) 1D global-RMS normalisation               (Section 3.2)
+  Algorithm 1, all three parameter branches          (param_step)
   Eq. (14) parameter update with decoupled decay     (Section 3.2)
   Algorithm 1 (MeqMuon), hidden-weight branch        (Section 3.2)
 
@@ -193,6 +194,29 @@ def hidden_step(W, G, B_prev, lr, mu, weight_decay, eps=DELTA, rho=RHO,
     W_next = apply_update(W, Ut, lr, weight_decay, rho)
     info = dict(info, U=U, U_tilde=Ut)
     return W_next, B, info
+
+
+HIDDEN = 0          # 2D weight in a hidden layer
+REMAINING_2D = 1    # remaining 2D parameter (token embedding, LM head)
+VECTOR = 2          # 1D parameter (RMSNorm weight, bias)
+
+
+def param_step(kind, W, G, B_prev, lr, mu, weight_decay, eps=DELTA, rho=RHO, **kw):
+    """Algorithm 1 for one parameter of any type: Eq. (10) momentum, then the
+    normalised update of its branch (Eq. (11) after Eq. (5) for hidden 2D
+    weights, Eq. (12) for the remaining 2D parameters, Eq. (13) for 1D
+    parameters), then Eq. (14). Returns (W_next, B_t, U_tilde)."""
+    if kind == HIDDEN:
+        Wn, B, info = hidden_step(W, G, B_prev, lr, mu, weight_decay, eps=eps, rho=rho, **kw)
+        return Wn, B, info["U_tilde"]
+    B = momentum_update(B_prev, G, mu)
+    if kind == REMAINING_2D:
+        Ut = two_sided_normalize(B, eps)
+    elif kind == VECTOR:
+        Ut = vector_normalize(B, eps)
+    else:
+        raise ValueError(kind)
+    return apply_update(W, Ut, lr, weight_decay, rho), B, Ut
 
 
 def hidden_step_all(Ws, Gs, Bs_prev, lr, mu, weight_decay, **kw):

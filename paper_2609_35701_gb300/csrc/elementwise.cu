@@ -9,7 +9,9 @@
 //   finalize      : r, c (Eq. (7)) from the partial sums of squares the last
 //                   NS epilogue wrote, gamma_r, gamma_c (Eq. (8)), the
 //                   direction (Eq. (11)) and the scale vector of Eq. (9).
-//   apply         : W <- (1 - lr wd) W - rho lr s (.) U (Eq. (14)).
+//   rows, colpart : momentum, row and column statistics of the remaining 2D
+//                   parameters and vectors (Eqs. (12), (13)).
+//   apply         : W <- (1 - lr wd) W - rho lr U~ (Eq. (14)).
 #include "meq_elementwise.cuh"
 
 namespace meq {
@@ -17,12 +19,18 @@ namespace {
 
 constexpr int kThreads = 256;
 
+// Largest i with begin(i) <= key; begin is nondecreasing in i. Entries that
+// own no work of the enumeration share their begin with the next entry (or
+// lie past the end), so they are never selected.
 __device__ __forceinline__ int find_mat(const MatInfo* mats, int nmat, int64_t key, int which) {
-  // Largest i with begin(i) <= key; begin is nondecreasing in i.
   int lo = 0, hi = nmat - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
-    const int64_t b = which == 0 ? mats[mid].chunk_begin : mats[mid].tile_begin;
+    const int64_t b = which == 0   ? mats[mid].chunk_begin
+                      : which == 1 ? mats[mid].tile_begin
+                      : which == 2 ? mats[mid].hchunk_begin
+                      : which == 3 ? mats[mid].rblk_begin
+                                   : mats[mid].slab_begin;
     if (b <= key) lo = mid; else hi = mid - 1;
   }
   return lo;
@@ -59,10 +67,10 @@ __global__ void __launch_bounds__(kThreads) momentum_norm_kernel(const MatInfo* 
   __shared__ float shf[32];
   __shared__ int is_last;
   const int64_t chunk = blockIdx.x;
-  const int mi = find_mat(mats, nmat, chunk, 0);
+  const int mi = find_mat(mats, nmat, chunk, 2);
   const MatInfo& M = mats[mi];
   const int64_t numel = M.m * M.n;
-  const int64_t e0 = (chunk - M.chunk_begin) * kChunk;
+  const int64_t e0 = (chunk - M.hchunk_begin) * kChunk;
   const int64_t e1 = min(e0 + kChunk, numel);
   const float mu = sc->mu;
   const int nesterov = sc->nesterov;
@@ -108,13 +116,86 @@ __global__ void __launch_bounds__(kThreads) momentum_norm_kernel(const MatInfo* 
   // (fp32 throughout: this GPU's fp64 rate is a small fraction of its fp32 rate).
   const int64_t nchunks = (numel + kChunk - 1) / kChunk;
   float acc = 0.f;
-  for (int64_t c = threadIdx.x; c < nchunks; c += kThreads) acc += __ldcg(partials + M.chunk_begin + c);
+  for (int64_t c = threadIdx.x; c < nchunks; c += kThreads) acc += __ldcg(partials + M.hchunk_begin + c);
   const float total = block_sum_f32(acc, shf);
   if (threadIdx.x == 0) {
     const float nrm = sqrtf(total);
     // Zero input: U = 0 (Eq. (5) is defined for a nonzero input only).
     x0scale[mi] = nrm > 0.f ? groups[M.group].alpha0 / nrm : 0.f;
     counters[mi] = 0u;
+  }
+}
+
+// ------------------------------------------- remaining 2D parameters, vectors
+// B <- mu B + G (Eq. (10)) and the row sums of squares of B, one warp per row
+// (a vector is a single row). Row sums go to rvec.
+__global__ void __launch_bounds__(kThreads) rows_kernel(const MatInfo* __restrict__ mats, int nmat,
+                                                       float* __restrict__ mom, const float* const* __restrict__ grads,
+                                                       const StepScalars* __restrict__ sc, float* __restrict__ rvec) {
+  pdl_allow_dependents();
+  pdl_wait_predecessor();
+  const int64_t blk = blockIdx.x;
+  const int mi = find_mat(mats, nmat, blk, 3);
+  const MatInfo& M = mats[mi];
+  const int lane = threadIdx.x & 31;
+  const int64_t row = (blk - M.rblk_begin) * (kThreads / 32) + (threadIdx.x >> 5);
+  if (row >= M.m) return;  // no block-wide synchronisation below
+  const float mu = sc->mu;
+  float* B = mom + M.mom_off + row * M.n;
+  const float* G = grads[mi] + row * M.n;
+  float ss = 0.f;
+  if ((M.n & 3) == 0) {
+    for (int64_t c = 4 * lane; c < M.n; c += 128) {
+      const float4 g = __ldcs(reinterpret_cast<const float4*>(G + c));
+      float4 b = *reinterpret_cast<const float4*>(B + c);
+      b.x = fmaf(mu, b.x, g.x), b.y = fmaf(mu, b.y, g.y), b.z = fmaf(mu, b.z, g.z), b.w = fmaf(mu, b.w, g.w);
+      *reinterpret_cast<float4*>(B + c) = b;
+      ss += b.x * b.x + b.y * b.y + b.z * b.z + b.w * b.w;
+    }
+  } else {
+    for (int64_t c = lane; c < M.n; c += 32) {
+      const float b = fmaf(mu, B[c], G[c]);
+      B[c] = b;
+      ss += b * b;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if (lane == 0) rvec[M.vec_off + row] = ss;
+}
+
+// Column sums of squares of N_r(B) (Eq. (12), inner operator) per 32-row
+// slab, deterministic; rows with RMS at or below eps contribute nothing.
+__global__ void __launch_bounds__(kThreads) colpart_kernel(const MatInfo* __restrict__ mats, int nmat,
+                                                          const float* __restrict__ mom, const float* __restrict__ rvec,
+                                                          const StepScalars* __restrict__ sc, float* __restrict__ parts) {
+  pdl_allow_dependents();
+  pdl_wait_predecessor();
+  __shared__ float rinv[32];
+  const int64_t slab = blockIdx.x;
+  const int mi = find_mat(mats, nmat, slab, 4);
+  const MatInfo& M = mats[mi];
+  const int64_t ls = slab - M.slab_begin;
+  const int64_t r0 = ls * 32;
+  const int nr = static_cast<int>(M.m - r0 < 32 ? M.m - r0 : 32);
+  if (threadIdx.x < 32) {
+    float v = 0.f;
+    if (static_cast<int>(threadIdx.x) < nr) {
+      const float rms = sqrtf(rvec[M.vec_off + r0 + threadIdx.x] / static_cast<float>(M.n));
+      v = rms > sc->eps ? 1.0f / rms : 0.f;
+    }
+    rinv[threadIdx.x] = v;
+  }
+  __syncthreads();
+  const float* B = mom + M.mom_off + r0 * M.n;
+  float* cp = parts + M.cpart_off + ls * M.n;
+  for (int64_t c = threadIdx.x; c < M.n; c += kThreads) {
+    float acc = 0.f;
+    for (int r = 0; r < nr; ++r) {
+      const float x = B[r * M.n + c] * rinv[r];
+      acc += x * x;
+    }
+    cp[c] = acc;
   }
 }
 
@@ -236,12 +317,38 @@ __global__ void __launch_bounds__(kThreads) cast_x0_kernel(const MatInfo* __rest
 }
 
 // ----------------------------------------------------------------- statistics
-// Row / column RMS, CVs (fp64), direction and scale vector; one block per matrix.
+// Two-pass fp32 CV of Eq. (8) over the entries of v above delta.
+__device__ float block_cv(const float* v, int64_t len, float delta, float* shf) {
+  float cnt = 0.f, sum = 0.f;
+  for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
+    const float x = v[i];
+    if (x > delta) cnt += 1.f, sum += x;
+  }
+  cnt = block_sum_f32(cnt, shf);
+  sum = block_sum_f32(sum, shf);
+  const float mean = cnt > 0.f ? sum / cnt : 0.f;
+  float var = 0.f;
+  for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
+    const float x = v[i];
+    if (x > delta) var += (x - mean) * (x - mean);
+  }
+  var = block_sum_f32(var, shf);
+  return cnt > 0.f ? sqrtf(var / cnt) / mean : 0.f;
+}
+
+// Statistics and normalisation scales, one block per parameter.
+//   hidden     : r, c of U (Eq. (7)) from the partial sums the last NS
+//                epilogue wrote, gamma_r, gamma_c (Eq. (8)), the side of
+//                Eq. (11) and its scale vector (Eq. (9)) in svec;
+//   remaining 2D: r = row RMS of B, c = column RMS of N_r(B) (Eq. (12)),
+//                1/r in svec, 1/c in tvec, their CVs for inspection;
+//   vector     : r[0] = RMS of B, 1/r[0] in svec (Eq. (13)).
+// RMS values at or below eps are treated as zero (scale 0).
 __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __restrict__ mats,
                                                                const StepScalars* __restrict__ sc,
                                                                const float* __restrict__ parts,
                                                                float* __restrict__ rvec, float* __restrict__ cvec,
-                                                               float* __restrict__ svec,
+                                                               float* __restrict__ svec, float* __restrict__ tvec,
                                                                MatStats* __restrict__ stats) {
   pdl_allow_dependents();
   pdl_wait_predecessor();
@@ -253,6 +360,42 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
   float* s = svec + M.vec_off;
   const float inv_n = 1.0f / static_cast<float>(M.n);
   const float inv_m = 1.0f / static_cast<float>(M.m);
+  if (M.kind == KIND_VECTOR) {
+    if (threadIdx.x == 0) {
+      const float rms = sqrtf(r[0] * inv_n);  // r[0] holds the sum of squares
+      r[0] = rms;
+      s[0] = rms > delta ? 1.0f / rms : 0.f;
+      stats[blockIdx.x].gamma_r = 0.0;
+      stats[blockIdx.x].gamma_c = 0.0;
+      stats[blockIdx.x].direction = 3;
+    }
+    return;
+  }
+  if (M.kind == KIND_TWO_SIDED) {
+    float* t = tvec + M.vec_off;
+    for (int64_t i = threadIdx.x; i < M.m; i += blockDim.x) {
+      const float rms = sqrtf(r[i] * inv_n);  // r holds the row sums of squares
+      r[i] = rms;
+      s[i] = rms > delta ? 1.0f / rms : 0.f;
+    }
+    const int64_t nslabs = (M.m + 31) / 32;
+    for (int64_t j = threadIdx.x; j < M.n; j += blockDim.x) {
+      float acc = 0.f;
+      for (int64_t k = 0; k < nslabs; ++k) acc += parts[M.cpart_off + k * M.n + j];
+      const float rms = sqrtf(acc * inv_m);
+      c[j] = rms;
+      t[j] = rms > delta ? 1.0f / rms : 0.f;
+    }
+    __syncthreads();
+    const float gr = block_cv(r, M.m, delta, shf);
+    const float gc = block_cv(c, M.n, delta, shf);
+    if (threadIdx.x == 0) {
+      stats[blockIdx.x].gamma_r = static_cast<double>(gr);
+      stats[blockIdx.x].gamma_c = static_cast<double>(gc);
+      stats[blockIdx.x].direction = 2;
+    }
+    return;
+  }
   // NS rows (s of them) are the weight's rows, or its columns when transposed.
   const int64_t tiles_n = 2 * ((M.l + 255) / 256);  // two epilogue halves per 256-column tile
   const int64_t nrb = (M.s + 31) / 32;
@@ -271,27 +414,9 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
   __syncthreads();
   // Eq. (8) over entries > delta: two passes (mean, then squared deviations),
   // fp32 with fixed-order block reductions.
-  float gam[2];
-  for (int side = 0; side < 2; ++side) {
-    const float* v = side == 0 ? r : c;
-    const int64_t len = side == 0 ? M.m : M.n;
-    float cnt = 0.f, sum = 0.f;
-    for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
-      const float x = v[i];
-      if (x > delta) cnt += 1.f, sum += x;
-    }
-    cnt = block_sum_f32(cnt, shf);
-    sum = block_sum_f32(sum, shf);
-    const float mean = cnt > 0.f ? sum / cnt : 0.f;
-    float var = 0.f;
-    for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
-      const float x = v[i];
-      if (x > delta) var += (x - mean) * (x - mean);
-    }
-    var = block_sum_f32(var, shf);
-    gam[side] = cnt > 0.f ? sqrtf(var / cnt) / mean : 0.f;
-  }
-  const int dir = gam[0] >= gam[1] - sc->tie_atol ? 0 : 1;
+  const float gam0 = block_cv(r, M.m, delta, shf);
+  const float gam1 = block_cv(c, M.n, delta, shf);
+  const int dir = gam0 >= gam1 - sc->tie_atol ? 0 : 1;
   const float* v = dir == 0 ? r : c;
   const int64_t len = dir == 0 ? M.m : M.n;
   for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
@@ -299,17 +424,21 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
     s[i] = x > delta ? 1.0f / x : 0.0f;   // RMS at or below delta: treated as zero
   }
   if (threadIdx.x == 0) {
-    stats[blockIdx.x].gamma_r = static_cast<double>(gam[0]);
-    stats[blockIdx.x].gamma_c = static_cast<double>(gam[1]);
+    stats[blockIdx.x].gamma_r = static_cast<double>(gam0);
+    stats[blockIdx.x].gamma_c = static_cast<double>(gam1);
     stats[blockIdx.x].direction = dir;
   }
 }
 
 // ----------------------------------------------------------------------- apply
+// W <- (1 - lr wd) W - rho lr U~ (Eq. (14)), U~ = scaled U (hidden) or scaled
+// B (remaining 2D: s_i t_j B_ij; vector: s_0 B_j).
 __global__ void __launch_bounds__(kThreads) apply_kernel(const MatInfo* __restrict__ mats, int nmat,
                                                          float* const* __restrict__ params,
                                                          const float* __restrict__ uslab,
+                                                         const float* __restrict__ mom,
                                                          const float* __restrict__ svec,
+                                                         const float* __restrict__ tvec,
                                                          const MatStats* __restrict__ stats,
                                                          const StepScalars* __restrict__ sc) {
   pdl_allow_dependents();
@@ -322,9 +451,13 @@ __global__ void __launch_bounds__(kThreads) apply_kernel(const MatInfo* __restri
   const int64_t e1 = min(e0 + kChunk, numel);
   const float decay = 1.0f - sc->lr * sc->wd;
   const float step = sc->rho * sc->lr;
-  const int dir = stats[mi].direction;
+  const bool hidden = M.kind == KIND_HIDDEN;
+  // mode 0: per-row scale; 1: per-column scale; 2: row scale x column scale
+  const int mode = hidden ? stats[mi].direction : (M.kind == KIND_TWO_SIDED ? 2 : 0);
   const float* sv = svec + M.vec_off;
-  const float* U = uslab + M.u_off;
+  const float* tv = tvec + M.vec_off;
+  const float* U = hidden ? uslab + M.u_off : mom + M.mom_off;
+  const int64_t ustride = hidden ? M.un : M.n;
   float* W = params[mi];
   if ((M.n & 3) == 0) {
     // Rows are whole float4s and the U stride equals n.
@@ -333,11 +466,15 @@ __global__ void __launch_bounds__(kThreads) apply_kernel(const MatInfo* __restri
       float4 w = *reinterpret_cast<const float4*>(W + e);
       const float4 u = __ldcs(reinterpret_cast<const float4*>(U + e));
       float s0, s1, s2, s3;
-      if (dir == 0) {
+      if (mode == 0) {
         s0 = s1 = s2 = s3 = sv[i];
       } else {
-        const float4 s4 = *reinterpret_cast<const float4*>(sv + j);
+        const float4 s4 = *reinterpret_cast<const float4*>((mode == 1 ? sv : tv) + j);
         s0 = s4.x, s1 = s4.y, s2 = s4.z, s3 = s4.w;
+        if (mode == 2) {
+          const float si = sv[i];
+          s0 *= si, s1 *= si, s2 *= si, s3 *= si;
+        }
       }
       w.x = fmaf(decay, w.x, -step * (s0 * u.x));
       w.y = fmaf(decay, w.y, -step * (s1 * u.y));
@@ -348,8 +485,8 @@ __global__ void __launch_bounds__(kThreads) apply_kernel(const MatInfo* __restri
   } else {
     for (int64_t e = e0 + threadIdx.x; e < e1; e += kThreads) {
       const int64_t i = e / M.n, j = e - i * M.n;
-      const float u = U[i * M.un + j];
-      const float s = dir == 0 ? sv[i] : sv[j];
+      const float u = U[i * ustride + j];
+      const float s = mode == 0 ? sv[i] : (mode == 1 ? sv[j] : sv[i] * tv[j]);
       W[e] = fmaf(decay, W[e], -step * (s * u));
     }
   }
@@ -373,8 +510,18 @@ __global__ void wait_selftest_kernel(const volatile int* flag, int* err, unsigne
 }  // namespace
 
 cudaError_t launch_momentum_norm(const LaunchCtx& L, cudaStream_t st) {
-  return launch_pdl(momentum_norm_kernel, dim3((unsigned)L.total_chunks), dim3(kThreads), 0, st, 1, L.mats, L.nmat,
+  return launch_pdl(momentum_norm_kernel, dim3((unsigned)L.total_hchunks), dim3(kThreads), 0, st, 1, L.mats, L.nmat,
                     L.groups, L.mom, L.grads, L.sc, L.partials, L.counters, L.x0scale);
+}
+
+cudaError_t launch_rows(const LaunchCtx& L, cudaStream_t st) {
+  return launch_pdl(rows_kernel, dim3((unsigned)L.total_rblks), dim3(kThreads), 0, st, 1, L.mats, L.nmat, L.mom,
+                    L.grads, L.sc, L.rvec);
+}
+
+cudaError_t launch_colpart(const LaunchCtx& L, cudaStream_t st) {
+  return launch_pdl(colpart_kernel, dim3((unsigned)L.total_slabs), dim3(kThreads), 0, st, 1, L.mats, L.nmat,
+                    static_cast<const float*>(L.mom), static_cast<const float*>(L.rvec), L.sc, L.parts);
 }
 
 cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st) {
@@ -387,12 +534,13 @@ cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st) {
 
 cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st) {
   return launch_pdl(finalize_kernel, dim3(L.nmat), dim3(kFinThreads), 0, st, 1, L.mats, L.sc,
-                    static_cast<const float*>(L.parts), L.rvec, L.cvec, L.svec, L.stats);
+                    static_cast<const float*>(L.parts), L.rvec, L.cvec, L.svec, L.tvec, L.stats);
 }
 
 cudaError_t launch_apply(const LaunchCtx& L, cudaStream_t st) {
   return launch_pdl(apply_kernel, dim3((unsigned)L.total_chunks), dim3(kThreads), 0, st, 1, L.mats, L.nmat, L.params,
-                    static_cast<const float*>(L.uslab), static_cast<const float*>(L.svec),
+                    static_cast<const float*>(L.uslab), static_cast<const float*>(L.mom),
+                    static_cast<const float*>(L.svec), static_cast<const float*>(L.tvec),
                     static_cast<const MatStats*>(L.stats), L.sc);
 }
 

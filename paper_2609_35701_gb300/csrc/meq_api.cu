@@ -67,12 +67,14 @@ struct Layout {
 struct meq_state {
   int n = 0;
   std::vector<meq_shape> shapes;
+  std::vector<int> kinds;                     // meq_kind per entry
+  int n_hidden = 0, n_rows = 0, n_two = 0;    // hidden / row-pass (remaining 2D + vectors) / two-sided
   meq_options opt{};
   int device = 0;
   int num_sms = 0;
   std::vector<MatInfo> mats;
   std::vector<Group> groups;
-  int64_t total_chunks = 0, total_tiles = 0;
+  int64_t total_chunks = 0, total_hchunks = 0, total_tiles = 0, total_rblks = 0, total_slabs = 0;
   int64_t mom_floats = 0, u_floats = 0, vec_floats = 0, parts_floats = 0;
   char* arena = nullptr;
   int64_t arena_bytes = 0;
@@ -84,6 +86,7 @@ struct meq_state {
   float* d_rvec = nullptr;
   float* d_cvec = nullptr;
   float* d_svec = nullptr;
+  float* d_tvec = nullptr;
   float* d_parts = nullptr;
   float* d_partials = nullptr;
   unsigned int* d_counters = nullptr;
@@ -131,6 +134,18 @@ bool valid_options(const meq_options& o, std::string* why) {
   return true;
 }
 
+bool valid_kinds(const meq_shape* shapes, const int* kinds, int n, std::string* why) {
+  if (!kinds) return true;
+  for (int i = 0; i < n; ++i) {
+    if (kinds[i] < 0 || kinds[i] > 2) { *why = "kind of entry " + std::to_string(i) + " is not a meq_kind"; return false; }
+    if (kinds[i] == KIND_VECTOR && shapes[i].rows != 1) {
+      *why = "vector entry " + std::to_string(i) + " must have shape (1, d)";
+      return false;
+    }
+  }
+  return true;
+}
+
 bool valid_shapes(const meq_shape* shapes, int n, std::string* why) {
   if (n <= 0) { *why = "n must be positive"; return false; }
   if (!shapes) { *why = "shapes is NULL"; return false; }
@@ -157,12 +172,21 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
   st->mats.assign(n, MatInfo{});
   std::map<std::tuple<int64_t, int64_t, int>, int> gmap;
   st->groups.clear();
+  st->n_hidden = st->n_rows = st->n_two = 0;
   for (int i = 0; i < n; ++i) {
     const int64_t m = st->shapes[i].rows, c = st->shapes[i].cols;
     MatInfo& M = st->mats[i];
     M.m = m, M.n = c;
     M.s = std::min(m, c), M.l = std::max(m, c);
     M.trans = m > c ? 1 : 0;
+    M.kind = st->kinds[i];
+    M.group = -1;
+    if (M.kind != KIND_HIDDEN) {
+      ++st->n_rows;
+      if (M.kind == KIND_TWO_SIDED) ++st->n_two;
+      continue;
+    }
+    ++st->n_hidden;
     auto key = std::make_tuple(M.s, M.l, M.trans);
     auto it = gmap.find(key);
     int g;
@@ -184,7 +208,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
     M.gidx = st->groups[g].count++;
     st->groups[g].mats.push_back(i);
   }
-  int64_t mom = 0, u = 0, vec = 0, parts = 0, chunks = 0, tiles = 0;
+  int64_t mom = 0, u = 0, vec = 0, parts = 0, chunks = 0, hchunks = 0, tiles = 0, rblks = 0, slabs = 0;
   for (auto& G : st->groups) {  // U is stored group by group: [count][m][un]
     G.u_base = u;
     u += round_up(G.count * G.m * G.un, 64);
@@ -195,30 +219,46 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
   }
   for (int i = 0; i < n; ++i) {
     MatInfo& M = st->mats[i];
-    const Group& G = st->groups[M.group];
-    M.un = G.un;
     M.mom_off = mom;
     mom += round_up(M.m * M.n, 64);
-    M.u_off = G.u_base + M.gidx * M.m * M.un;
-    M.rpart_off = G.rpart_base + M.gidx * 2 * ((G.l + 255) / 256) * G.s;
-    M.cpart_off = G.cpart_base + M.gidx * ((G.s + 31) / 32) * G.l;
     M.vec_off = vec;
     vec += round_up(std::max(M.m, M.n), 64);
-    M.chunk_begin = chunks;
+    M.chunk_begin = chunks;  // apply: every kind
     chunks += (M.m * M.n + kChunk - 1) / kChunk;
+    M.hchunk_begin = hchunks;
     M.tile_begin = tiles;
-    tiles += ((M.m + kCastTile - 1) / kCastTile) * ((M.n + kCastTile - 1) / kCastTile);
+    M.rblk_begin = rblks;
+    M.slab_begin = slabs;
+    if (M.kind == KIND_HIDDEN) {
+      const Group& G = st->groups[M.group];
+      M.un = G.un;
+      M.u_off = G.u_base + M.gidx * M.m * M.un;
+      M.rpart_off = G.rpart_base + M.gidx * 2 * ((G.l + 255) / 256) * G.s;
+      M.cpart_off = G.cpart_base + M.gidx * ((G.s + 31) / 32) * G.l;
+      hchunks += (M.m * M.n + kChunk - 1) / kChunk;
+      tiles += ((M.m + kCastTile - 1) / kCastTile) * ((M.n + kCastTile - 1) / kCastTile);
+    } else {
+      M.un = M.n;
+      rblks += (M.m + 7) / 8;  // 8 rows (warps) per block
+      if (M.kind == KIND_TWO_SIDED) {
+        const int64_t ns = (M.m + 31) / 32;
+        M.cpart_off = parts;
+        parts += round_up(ns * M.n, 64);
+        slabs += ns;
+      }
+    }
   }
   st->mom_floats = mom, st->u_floats = u, st->vec_floats = vec, st->parts_floats = parts;
-  st->total_chunks = chunks, st->total_tiles = tiles;
+  st->total_chunks = chunks, st->total_hchunks = hchunks, st->total_tiles = tiles;
+  st->total_rblks = rblks, st->total_slabs = slabs;
   st->persistent_bytes = 0;
   for (int i = 0; i < n; ++i) st->persistent_bytes += 4 * st->mats[i].m * st->mats[i].n;
 
   *off_mom = L->add(mom * 4);
   *off_u = L->add(u * 4);
-  *off_vec4 = L->add(vec * 3 * 4);  // r, c, scale
+  *off_vec4 = L->add(vec * 4 * 4);  // r, c, s, t
   *off_cpart = L->add(parts * 4);
-  *off_partials = L->add(chunks * 4);
+  *off_partials = L->add(hchunks * 4);
   *off_counters = L->add(int64_t(n) * 4);
   *off_x0s = L->add(int64_t(n) * 4);
   *off_stats = L->add(int64_t(n) * sizeof(MatStats));
@@ -414,13 +454,21 @@ const char* meq_status_string(meq_status s) {
 const char* meq_last_error(const meq_state* st) { return st ? st->last_error.c_str() : g_init_error.c_str(); }
 
 meq_status meq_state_bytes(const meq_shape* shapes, int n, const meq_options* opt, size_t* persistent, size_t* workspace) {
+  return meq_state_bytes_kinds(shapes, nullptr, n, opt, persistent, workspace);
+}
+
+meq_status meq_state_bytes_kinds(const meq_shape* shapes, const int* kinds, int n, const meq_options* opt,
+                                 size_t* persistent, size_t* workspace) {
   meq_options o;
   if (opt) o = *opt; else meq_default_options(&o);
   std::string why;
-  if (!valid_shapes(shapes, n, &why) || !valid_options(o, &why)) return fail(nullptr, MEQ_ERR_INVALID_ARG, why);
+  if (!valid_shapes(shapes, n, &why) || !valid_kinds(shapes, kinds, n, &why) || !valid_options(o, &why))
+    return fail(nullptr, MEQ_ERR_INVALID_ARG, why);
   meq_state tmp;
   tmp.n = n;
   tmp.shapes.assign(shapes, shapes + n);
+  tmp.kinds.assign(n, KIND_HIDDEN);
+  if (kinds) tmp.kinds.assign(kinds, kinds + n);
   tmp.opt = o;
   Layout L;
   int64_t a[13];
@@ -432,12 +480,18 @@ meq_status meq_state_bytes(const meq_shape* shapes, int n, const meq_options* op
 }
 
 meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt, void* cuda_stream, meq_state** out) {
+  return meq_init_state_kinds(shapes, nullptr, n, opt, cuda_stream, out);
+}
+
+meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n, const meq_options* opt,
+                                void* cuda_stream, meq_state** out) {
   if (!out) return fail(nullptr, MEQ_ERR_INVALID_ARG, "out is NULL");
   *out = nullptr;
   meq_options o;
   if (opt) o = *opt; else meq_default_options(&o);
   std::string why;
-  if (!valid_shapes(shapes, n, &why) || !valid_options(o, &why)) return fail(nullptr, MEQ_ERR_INVALID_ARG, why);
+  if (!valid_shapes(shapes, n, &why) || !valid_kinds(shapes, kinds, n, &why) || !valid_options(o, &why))
+    return fail(nullptr, MEQ_ERR_INVALID_ARG, why);
 
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -458,6 +512,8 @@ meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt
   meq_state* st = new meq_state();
   st->n = n;
   st->shapes.assign(shapes, shapes + n);
+  st->kinds.assign(n, KIND_HIDDEN);
+  if (kinds) st->kinds.assign(kinds, kinds + n);
   st->opt = o;
   st->device = dev;
   st->num_sms = prop.multiProcessorCount;
@@ -485,6 +541,7 @@ meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt
   st->d_rvec = reinterpret_cast<float*>(A + off_vec4);
   st->d_cvec = st->d_rvec + st->vec_floats;
   st->d_svec = st->d_cvec + st->vec_floats;
+  st->d_tvec = st->d_svec + st->vec_floats;
   st->d_parts = reinterpret_cast<float*>(A + off_cpart);
   st->d_partials = reinterpret_cast<float*>(A + off_partials);
   st->d_counters = reinterpret_cast<unsigned int*>(A + off_counters);
@@ -543,10 +600,15 @@ meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt
   C.rvec = st->d_rvec;
   C.cvec = st->d_cvec;
   C.svec = st->d_svec;
+  C.tvec = st->d_tvec;
   C.stats = st->d_stats;
   C.total_chunks = st->total_chunks;
+  C.total_hchunks = st->total_hchunks;
   C.total_tiles = st->total_tiles;
-  st->kernels_per_step = 4 + static_cast<int>(st->gemm.size());
+  C.total_rblks = st->total_rblks;
+  C.total_slabs = st->total_slabs;
+  st->kernels_per_step = (st->n_hidden ? 2 : 0) + (st->n_rows ? 1 : 0) + (st->n_two ? 1 : 0) + 2 +
+                         static_cast<int>(st->gemm.size());
   st->step_host.assign(static_cast<size_t>(st->step_bytes), 0);
   st->last_stream = s;
   *out = st;
@@ -563,20 +625,33 @@ static void drop_profile(meq_state* st) {
 static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev = nullptr) {
   const LaunchCtx& C = st->ctx;
   auto mark = [&](int i) { if (ev) cudaEventRecord(ev[i], s); };
+  cudaError_t e = cudaSuccess;
   mark(0);
-  cudaError_t e = launch_momentum_norm(C, s);
-  if (e != cudaSuccess) return cuda_fail(st, e, "momentum_norm launch");
+  if (st->n_hidden) {
+    e = launch_momentum_norm(C, s);
+    if (e != cudaSuccess) return cuda_fail(st, e, "momentum_norm launch");
+  }
+  if (st->n_rows) {
+    e = launch_rows(C, s);
+    if (e != cudaSuccess) return cuda_fail(st, e, "rows launch");
+  }
   mark(1);
-  e = launch_cast_x0(C, iter_fp16(st->opt, 0), s);
-  if (e != cudaSuccess) return cuda_fail(st, e, "cast_x0 launch");
+  if (st->n_hidden) {
+    e = launch_cast_x0(C, iter_fp16(st->opt, 0), s);
+    if (e != cudaSuccess) return cuda_fail(st, e, "cast_x0 launch");
+  }
   mark(2);
   for (size_t i = 0; i < st->gemm.size(); ++i) {
     e = launch_ns_gemm(st->gemm[i], st->gemm_grid[i], st->opt.ns_cta_pair ? 2 : 1, s);
     if (e != cudaSuccess) return cuda_fail(st, e, "ns_gemm launch");
   }
   mark(3);
+  if (st->n_two) {
+    e = launch_colpart(C, s);
+    if (e != cudaSuccess) return cuda_fail(st, e, "colpart launch");
+  }
   e = launch_stats(C, s);
-  if (e != cudaSuccess) return cuda_fail(st, e, "stats launch");
+  if (e != cudaSuccess) return cuda_fail(st, e, "finalize launch");
   mark(4);
   e = launch_apply(C, s);
   if (e != cudaSuccess) return cuda_fail(st, e, "apply launch");
@@ -721,6 +796,7 @@ meq_status meq_read_ns_output(meq_state* st, int i, float* dst) {
   meq_status ms = check_index(st, i);
   if (ms != MEQ_OK) return ms;
   if (!dst) return fail(st, MEQ_ERR_INVALID_ARG, "dst is NULL");
+  if (st->kinds[i] != KIND_HIDDEN) return fail(st, MEQ_ERR_INVALID_ARG, "entry has no Newton-Schulz output (not hidden)");
   const MatInfo& M = st->mats[i];
   cudaError_t e = cudaMemcpy2D(dst, M.n * sizeof(float), st->d_u + M.u_off, M.un * sizeof(float), M.n * sizeof(float),
                                M.m, cudaMemcpyDefault);
@@ -771,6 +847,8 @@ meq_status meq_read_profile(meq_state* st, double* phase_ms, int64_t* steps) {
 }
 
 int meq_kernels_per_step(const meq_state* st) { return st ? st->kernels_per_step : 0; }
+
+int meq_ns_gemm_launches_per_step(const meq_state* st) { return st ? static_cast<int>(st->gemm.size()) : 0; }
 
 meq_status meq_debug_wait_selftest(meq_state* st, float timeout_ms) {
   if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");

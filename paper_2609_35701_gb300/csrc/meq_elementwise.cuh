@@ -32,12 +32,17 @@ struct LaunchCtx {
   float* parts;          // NS-row and NS-column partial sums of squares
   float* rvec;
   float* cvec;
-  float* svec;
+  float* svec;           // hidden: scale of the chosen side; others: 1 / row RMS
+  float* tvec;           // remaining 2D: 1 / column RMS of the row-normalised momentum
   MatStats* stats;
-  int64_t total_chunks, total_tiles;
+  int64_t total_chunks, total_hchunks, total_tiles, total_rblks, total_slabs;
 };
 
+constexpr int KIND_HIDDEN = 0, KIND_TWO_SIDED = 1, KIND_VECTOR = 2;
+
 cudaError_t launch_momentum_norm(const LaunchCtx& L, cudaStream_t st);
+cudaError_t launch_rows(const LaunchCtx& L, cudaStream_t st);      // remaining 2D + vectors
+cudaError_t launch_colpart(const LaunchCtx& L, cudaStream_t st);   // remaining 2D
 cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st);
 cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st);  // finalize of the fused statistics
 cudaError_t launch_apply(const LaunchCtx& L, cudaStream_t st);

@@ -30,16 +30,22 @@ struct MatInfo {
   int64_t m, n;          // W layout: rows, cols
   int64_t s, l;          // oriented NS shape: s = min(m, n), l = max(m, n)
   int32_t trans;         // 1 when the NS layout is W^T (m > n)
-  int32_t group;         // shape group
+  int32_t group;         // shape group (hidden weights)
+  int32_t kind;          // 0 hidden, 1 remaining 2D (two-sided), 2 vector
+  int32_t pad_;
   int64_t gidx;          // index inside its group
   int64_t mom_off;       // float offset of B in the momentum slab
   int64_t u_off;         // float offset of U in the U slab (row stride un)
   int64_t un;            // U row stride (cols rounded up to 4)
   int64_t vec_off;       // float offset of r (m), c (n) and scale (max(m, n))
-  int64_t chunk_begin;   // first momentum chunk
-  int64_t tile_begin;    // first cast tile
+  int64_t chunk_begin;   // first apply chunk (all kinds)
+  int64_t hchunk_begin;  // first momentum-and-norm chunk (hidden weights only)
+  int64_t rblk_begin;    // first 8-row block of the row pass (remaining 2D and vectors)
+  int64_t slab_begin;    // first 32-row slab of the column pass (remaining 2D only)
+  int64_t tile_begin;    // first cast tile (hidden weights only)
   int64_t rpart_off;     // float offset of NS-row partial sums of squares [2 * ceil(l/256)][s]
-  int64_t cpart_off;     // float offset of NS-column partial sums of squares [ceil(s/32)][l]
+  int64_t cpart_off;     // float offset of column partial sums of squares: NS columns
+                         // [ceil(s/32)][l] (hidden) or normalised columns [ceil(m/32)][n] (remaining 2D)
 };
 
 // Per-group metadata for the elementwise kernels.

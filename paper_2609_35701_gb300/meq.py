@@ -48,7 +48,9 @@ EXPORTED = [
     "meq_last_error", "meq_status_string", "meq_read_momentum", "meq_write_momentum",
     "meq_read_ns_output", "meq_read_stats", "meq_kernels_per_step", "meq_debug_wait_selftest",
     "meq_set_profiling", "meq_read_profile", "meq_row_col_stats_noalloc",
+    "meq_init_state_kinds", "meq_state_bytes_kinds", "meq_ns_gemm_launches_per_step",
 ]
+HIDDEN, REMAINING_2D, VECTOR = 0, 1, 2  # meq_kind
 
 
 def _load():
@@ -91,6 +93,14 @@ def _load():
     lib.meq_read_profile.restype = I
     lib.meq_row_col_stats_noalloc.argtypes = [P, ctypes.c_int64, ctypes.c_int64, F, F, P, P, P, P, P]
     lib.meq_row_col_stats_noalloc.restype = I
+    lib.meq_init_state_kinds.argtypes = [ctypes.POINTER(MeqShape), P, I, ctypes.POINTER(MeqOptions), P,
+                                         ctypes.POINTER(P)]
+    lib.meq_init_state_kinds.restype = I
+    lib.meq_state_bytes_kinds.argtypes = [ctypes.POINTER(MeqShape), P, I, ctypes.POINTER(MeqOptions),
+                                          ctypes.POINTER(ctypes.c_size_t), ctypes.POINTER(ctypes.c_size_t)]
+    lib.meq_state_bytes_kinds.restype = I
+    lib.meq_ns_gemm_launches_per_step.argtypes = [P]
+    lib.meq_ns_gemm_launches_per_step.restype = I
     return lib
 
 
@@ -120,11 +130,20 @@ def _shape_array(shapes):
     return arr
 
 
-def state_bytes(shapes, **opts):
+def _kind_array(kinds, n):
+    if kinds is None:
+        return None
+    if len(kinds) != n:
+        raise ValueError("one kind per shape")
+    return (ctypes.c_int * n)(*[int(k) for k in kinds])
+
+
+def state_bytes(shapes, kinds=None, **opts):
     """(persistent, workspace) bytes for a shape list, computed on the host."""
     p, w = ctypes.c_size_t(), ctypes.c_size_t()
     o = default_options(**opts)
-    st = lib.meq_state_bytes(_shape_array(shapes), len(shapes), ctypes.byref(o), ctypes.byref(p), ctypes.byref(w))
+    st = lib.meq_state_bytes_kinds(_shape_array(shapes), _kind_array(kinds, len(shapes)), len(shapes), ctypes.byref(o),
+                                   ctypes.byref(p), ctypes.byref(w))
     if st != MEQ_OK:
         raise MeqError(st, lib.meq_last_error(None).decode())
     return p.value, w.value
@@ -151,15 +170,17 @@ def _stream_handle(stream):
 
 
 class MeqMuon:
-    """MeqMuon state for a fixed list of 2D hidden weights (rows, cols)."""
+    """MeqMuon state for a fixed list of parameters (rows, cols); kinds (one
+    meq_kind per entry, default all HIDDEN) select the branch of Algorithm 1."""
 
-    def __init__(self, shapes, stream=None, **opts):
+    def __init__(self, shapes, stream=None, kinds=None, **opts):
         self.shapes = [(int(r), int(c)) for r, c in shapes]
+        self.kinds = [HIDDEN] * len(self.shapes) if kinds is None else [int(k) for k in kinds]
         self._shape_arr = _shape_array(self.shapes)
         self._opts = default_options(**opts)
         self._st = ctypes.c_void_p()
-        s = lib.meq_init_state(self._shape_arr, len(self.shapes), ctypes.byref(self._opts), _stream_handle(stream),
-                               ctypes.byref(self._st))
+        s = lib.meq_init_state_kinds(self._shape_arr, _kind_array(self.kinds, len(self.shapes)), len(self.shapes),
+                                     ctypes.byref(self._opts), _stream_handle(stream), ctypes.byref(self._st))
         if s != MEQ_OK:
             raise MeqError(s, lib.meq_last_error(None).decode())
         n = len(self.shapes)
@@ -173,6 +194,10 @@ class MeqMuon:
     @property
     def kernels_per_step(self):
         return lib.meq_kernels_per_step(self._st)
+
+    @property
+    def ns_gemm_launches_per_step(self):
+        return lib.meq_ns_gemm_launches_per_step(self._st)
 
     def step_ptrs(self, param_ptrs, grad_ptrs, lr, momentum, weight_decay, eps=1e-7, stream=None):
         """One step given raw device pointers (ints)."""

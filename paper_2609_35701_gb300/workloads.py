@@ -24,6 +24,10 @@ gradients stand in for its Llama pretraining gradients):
              column scales (Student-t, nu = 3).
   llama7b    32 layers, d 4096, ffn 11008; base N(0, 0.005^2); per-matrix
              row / column / both imbalance, log-uniform [0.05, 20].
+  llama60m_full / llama130m_full
+             every trainable parameter of Llama-60M / Llama-130M (hidden 2D
+             weights, 32000 x d token embedding and LM head, RMSNorm weights),
+             the llama130m recipe on each.
 Imbalance scales are fixed per (seed, matrix); base noise is drawn per
 (seed, step, matrix). Initial weights are N(0, 0.02^2) per (seed, matrix).
 """
@@ -54,6 +58,30 @@ def hidden_shapes(layers, hidden, ffn, q_heads=None, kv_heads=None, head_dim=64)
     return out
 
 
+HIDDEN, REMAINING_2D, VECTOR = 0, 1, 2   # parameter types of Algorithm 1
+
+
+def full_model_params(layers, hidden, ffn, vocab, q_heads, kv_heads, head_dim=64, tied=False, qkv_bias=False):
+    """(name, rows, cols, kind) of every trainable parameter of a
+    pre-norm SwiGLU decoder (Table 8 architectures): the hidden 2D weights,
+    the token embedding and LM head (one matrix when tied), two RMSNorm
+    weights per layer and a final one, and q/k/v biases when present
+    (Qwen2). 1D parameters are given as (1, d)."""
+    out = [(n, r, c, HIDDEN) for n, r, c in hidden_shapes(layers, hidden, ffn, q_heads, kv_heads, head_dim)]
+    out.append(("embed_tokens", vocab, hidden, REMAINING_2D))
+    if not tied:
+        out.append(("lm_head", vocab, hidden, REMAINING_2D))
+    q, kv = q_heads * head_dim, kv_heads * head_dim
+    for l in range(layers):
+        out.append((f"layers.{l}.input_layernorm", 1, hidden, VECTOR))
+        out.append((f"layers.{l}.post_attention_layernorm", 1, hidden, VECTOR))
+        if qkv_bias:
+            out += [(f"layers.{l}.q_proj.bias", 1, q, VECTOR), (f"layers.{l}.k_proj.bias", 1, kv, VECTOR),
+                    (f"layers.{l}.v_proj.bias", 1, kv, VECTOR)]
+    out.append(("norm", 1, hidden, VECTOR))
+    return out
+
+
 @dataclass
 class Workload:
     name: str
@@ -70,9 +98,14 @@ class Workload:
     seed: int = 0
     extra: dict = field(default_factory=dict)
 
+    kinds: list = None                # one parameter type per shape (None: all hidden)
+
     @property
     def numel(self):
         return sum(r * c for _, r, c in self.shapes)
+
+    def kind_list(self):
+        return [HIDDEN] * len(self.shapes) if self.kinds is None else list(self.kinds)
 
 
 def _llama(layers, hidden, ffn):
@@ -87,6 +120,18 @@ WORKLOADS = {
     "llama7b": Workload("llama7b", _llama(32, 4096, 11008), 0.005, "row_col_both",
                         scale_lo=0.05, scale_hi=20.0, steps=5),
 }
+
+
+def _full(name, layers, hidden, ffn, vocab, heads, steps=10):
+    params = full_model_params(layers, hidden, ffn, vocab, heads, heads)
+    return Workload(name, [(n, r, c) for n, r, c, _ in params], 0.01, "half_row_half_col", steps=steps,
+                    kinds=[k for _, _, _, k in params])
+
+
+# Every trainable parameter of Llama-60M / Llama-130M (Table 8), as one
+# optimizer state (Algorithm 1 over all three parameter types).
+WORKLOADS["llama60m_full"] = _full("llama60m_full", 8, 512, 1376, 32000, 8)
+WORKLOADS["llama130m_full"] = _full("llama130m_full", 12, 768, 2048, 32000, 12)
 
 
 def get_workload(name):
@@ -111,7 +156,7 @@ def _gen(device, *key):
 def _pattern_of(w: Workload, i: int, layer: int):
     p = w.pattern
     if p == "half_row_half_col":
-        n_layers = max(1, len(w.shapes) // 7)
+        n_layers = max(1, sum(1 for n, _, _ in w.shapes if n.endswith("q_proj")))
         return "row" if layer < n_layers // 2 else "col"
     if p in ("row_col_none", "row_col_both"):
         choices = ("row", "col", "none") if p == "row_col_none" else ("row", "col", "both")

@@ -337,6 +337,24 @@ def check_two_sided_and_vector(O):
     assert abs(w[3] - v[3] / math.sqrt((v ** 2).mean())) < 1e-14
 
 
+def check_param_step_branches(O):
+    """Algorithm 1's three branches: a vector's update has RMS 1 (Eq. (13));
+    a remaining 2D parameter's update has unit-RMS columns (Eq. (12)); a
+    hidden weight goes through NS (its Hadamard case gives H_8)."""
+    rng = np.random.default_rng(21)
+    lr, mu, wd = 0.02, 0.95, 0.1
+    v = rng.standard_normal(40) * 3.0
+    Wn, B, Ut = O.param_step(O.VECTOR, np.zeros(40), v, np.zeros(40), lr, mu, wd)
+    assert np.abs(B - v).max() == 0.0 and abs(math.sqrt((Ut ** 2).mean()) - 1.0) < 1e-14
+    assert np.abs(Wn + 0.2 * lr * v / math.sqrt((v ** 2).mean())).max() < 1e-15
+    M = rng.standard_normal((30, 12)) * np.exp(rng.uniform(-2, 2, 30))[:, None]
+    Wn, B, Ut = O.param_step(O.REMAINING_2D, np.zeros((30, 12)), M, np.zeros((30, 12)), lr, mu, wd)
+    assert np.allclose(np.sqrt((Ut ** 2).sum(0) / 30), 1.0, atol=1e-14)
+    H = _sylvester_hadamard(8)
+    _, _, Ut = O.param_step(O.HIDDEN, np.zeros((8, 8)), H, np.zeros((8, 8)), lr, mu, wd)
+    assert np.abs(Ut - H).max() < 1e-12
+
+
 # ------------------------------------------------------------- momentum / apply
 def check_momentum_closed_form(O):
     """Eq. (10) with a constant gradient: B_t = G (1 - mu^(t+1)) / (1 - mu)."""
@@ -414,5 +432,5 @@ ALL_CHECKS = [
     check_ns_zero_rows_cols, check_ns_exact_integer, check_row_col_rms_rank_one,
     check_cv_hand_values, check_selection_rule, check_equilibration_invariants,
     check_orthogonality_constraint, check_two_sided_and_vector, check_momentum_closed_form,
-    check_apply_closed_form, check_hidden_step_composition,
+    check_apply_closed_form, check_hidden_step_composition, check_param_step_branches,
 ]

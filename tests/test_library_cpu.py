@@ -63,6 +63,31 @@ def test_state_holds_momentum_only():
         assert workspace > 0
 
 
+def test_full_model_state_reproduces_table5():
+    """Algorithm 1 over every trainable parameter keeps one fp32 momentum value
+    per parameter: the library's persistent bytes for the full Table 8 models
+    equal the MeqMuon column of Table 5 (Section 4, 'Memory overhead')."""
+    from paper_2609_35701_gb300 import meq, workloads as W
+
+    g = P.golden()
+    for name, a in g["architecture"].items():
+        params = W.full_model_params(a["layers"], a["hidden"], a["ffn"], a["vocab"], a["q_heads"], a["kv_heads"],
+                                     a["head_dim"], tied=a["tied"], qkv_bias=name.startswith("Qwen2"))
+        assert abs(sum(r * c for _, r, c, _ in params) / 1e6 - a["params_m"]) < 5e-4, name
+        persistent, _ = meq.state_bytes([(r, c) for _, r, c, _ in params], kinds=[k for _, _, _, k in params])
+        assert round(persistent / 2 ** 20, 2) == g["state_mib"]["MeqMuon"][name], name
+
+
+def test_kind_validation():
+    from paper_2609_35701_gb300 import meq
+
+    with pytest.raises(meq.MeqError) as e:
+        meq.state_bytes([(2, 8)], kinds=[meq.VECTOR])   # vectors are (1, d)
+    assert e.value.status == 1
+    with pytest.raises(meq.MeqError):
+        meq.state_bytes([(2, 8)], kinds=[7])
+
+
 def test_host_validation_errors():
     from paper_2609_35701_gb300 import meq
 

@@ -100,7 +100,16 @@ MUTATIONS = {
     "momentum_damped": ("momentum_update", lambda Bp, G, mu: mu * np.asarray(Bp) + (1 - mu) * np.asarray(G)),
     "momentum_no_mu": ("momentum_update", lambda Bp, G, mu: np.asarray(Bp) + np.asarray(G)),
     "nesterov_wrong": ("ns_input", lambda B, G, mu, nesterov=False: np.asarray(B) + (mu * np.asarray(G) if nesterov else 0)),
+    "two_sided_order_swapped": ("two_sided_normalize", lambda B, delta=1e-7: _col_then_row(B)),
+    "vector_uses_l2": ("vector_normalize", lambda b, delta=1e-7: np.asarray(b) / np.linalg.norm(b)),
 }
+
+
+def _col_then_row(B):
+    B = np.asarray(B, np.float64)
+    m, n = B.shape
+    X = B / np.sqrt((B * B).sum(0, keepdims=True) / m)
+    return X / np.sqrt((X * X).sum(1, keepdims=True) / n)
 
 
 @pytest.mark.parametrize("name", sorted(MUTATIONS))
