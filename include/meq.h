@@ -68,6 +68,10 @@ typedef struct {
   float wait_timeout_ms;  /* bound of every device-side spin wait; default 4000 */
   int ns_cta_pair;        /* 1 (default): NS GEMMs run on CTA pairs (tcgen05 cta_group::2,
                              256 x 256 tiles on two SMs); 0: one CTA per 128 x 256 tile */
+  int ns_x0_fused;        /* 1 (default): the momentum pass also writes X_0, unnormalised in
+                             bf16, and the first NS products apply 1/||B||_F; iteration 0
+                             then runs its X and P operands in bf16. 0: a separate pass
+                             writes the normalised X_0 in the format ns_fp16_mask gives it. */
 } meq_options;
 
 /* Parameter type, selecting the branch of Algorithm 1 applied to it. */

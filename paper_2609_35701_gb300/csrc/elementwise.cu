@@ -126,6 +126,141 @@ __global__ void __launch_bounds__(kThreads) momentum_norm_kernel(const MatInfo* 
   }
 }
 
+__device__ __forceinline__ uint2 pack4_bf16(float a, float b, float c, float d) {
+  uint2 w;
+  __nv_bfloat162 x = __floats2bfloat162_rn(a, b), y = __floats2bfloat162_rn(c, d);
+  w.x = *reinterpret_cast<uint32_t*>(&x);
+  w.y = *reinterpret_cast<uint32_t*>(&y);
+  return w;
+}
+__device__ __forceinline__ uint16_t bf16_bits(float v) {
+  __nv_bfloat16 h = __float2bfloat16_rn(v);
+  return *reinterpret_cast<uint16_t*>(&h);
+}
+
+// Hidden weights, one 64 x 64 tile of W per block: B <- mu B + G (Eq. (10))
+// and X_0 = bf16(H) in the oriented NS layout (tall W transposed through
+// shared memory), H being the NS input (B, or G + mu B for Nesterov). X_0 is
+// left unnormalised: bf16 has the exponent range of fp32, and the first NS
+// products apply 1 / ||H||_F (Eq. (5)) in their epilogues. The squared norm
+// is reduced per tile in fixed order; the last tile of a matrix writes
+// 1 / ||H||_F (0 for a zero input) to ginv.
+__global__ void __launch_bounds__(kThreads) momentum_x0_kernel(const MatInfo* __restrict__ mats, int nmat,
+                                                              const GroupInfo* __restrict__ groups,
+                                                              float* __restrict__ mom,
+                                                              const float* const* __restrict__ grads,
+                                                              const StepScalars* __restrict__ sc,
+                                                              float* __restrict__ partials,
+                                                              unsigned int* __restrict__ counters,
+                                                              float* __restrict__ ginv) {
+  pdl_allow_dependents();
+  pdl_wait_predecessor();
+  __shared__ float tile[kCastTile][kCastTile + 1];
+  __shared__ float shf[32];
+  __shared__ int is_last;
+  const int64_t t = blockIdx.x;
+  const int mi = find_mat(mats, nmat, t, 1);
+  const MatInfo& M = mats[mi];
+  const GroupInfo& Gi = groups[M.group];
+  const int64_t tiles_n = (M.n + kCastTile - 1) / kCastTile;
+  const int64_t ntiles = ((M.m + kCastTile - 1) / kCastTile) * tiles_n;
+  const int64_t lt = t - M.tile_begin;
+  const int64_t r0 = (lt / tiles_n) * kCastTile;
+  const int64_t c0 = (lt % tiles_n) * kCastTile;
+  const float mu = sc->mu;
+  const int nesterov = sc->nesterov;
+  float* B = mom + M.mom_off;
+  const float* G = grads[mi];
+  uint16_t* X = static_cast<uint16_t*>(Gi.x0) + M.gidx * Gi.s * Gi.lp;
+  const bool vec = (M.n & 3) == 0;
+  const int cx = (threadIdx.x & 15) * 4;  // 4 columns
+  const int ry = threadIdx.x >> 4;        // rows ry, ry + 16, ry + 32, ry + 48
+  float h[4][4];
+  float ss = 0.f;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int64_t row = r0 + ry + 16 * k, col = c0 + cx;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) h[k][u] = 0.f;
+    if (row >= M.m) continue;
+    if (vec && col + 3 < M.n) {
+      const float4 g = __ldcs(reinterpret_cast<const float4*>(G + row * M.n + col));
+      float4 b = *reinterpret_cast<const float4*>(B + row * M.n + col);
+      b.x = fmaf(mu, b.x, g.x), b.y = fmaf(mu, b.y, g.y), b.z = fmaf(mu, b.z, g.z), b.w = fmaf(mu, b.w, g.w);
+      *reinterpret_cast<float4*>(B + row * M.n + col) = b;
+      if (nesterov) {
+        h[k][0] = fmaf(mu, b.x, g.x), h[k][1] = fmaf(mu, b.y, g.y), h[k][2] = fmaf(mu, b.z, g.z);
+        h[k][3] = fmaf(mu, b.w, g.w);
+      } else {
+        h[k][0] = b.x, h[k][1] = b.y, h[k][2] = b.z, h[k][3] = b.w;
+      }
+    } else {
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (col + u < M.n) {
+          const float g = G[row * M.n + col + u];
+          const float b = fmaf(mu, B[row * M.n + col + u], g);
+          B[row * M.n + col + u] = b;
+          h[k][u] = nesterov ? fmaf(mu, b, g) : b;
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) ss += h[k][u] * h[k][u];
+  }
+  if (!M.trans) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int64_t row = r0 + ry + 16 * k, col = c0 + cx;
+      if (row >= M.m) continue;
+      if (col + 3 < M.n) {
+        *reinterpret_cast<uint2*>(X + row * Gi.lp + col) = pack4_bf16(h[k][0], h[k][1], h[k][2], h[k][3]);
+      } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (col + u < M.n) X[row * Gi.lp + col + u] = bf16_bits(h[k][u]);
+      }
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+#pragma unroll
+      for (int u = 0; u < 4; ++u) tile[ry + 16 * k][cx + u] = h[k][u];
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int xr = ry + 16 * k;
+      const int64_t xrow = c0 + xr, xcol = r0 + cx;
+      if (xrow >= M.n) continue;
+      if (xcol + 3 < M.m) {
+        *reinterpret_cast<uint2*>(X + xrow * Gi.lp + xcol) =
+            pack4_bf16(tile[cx][xr], tile[cx + 1][xr], tile[cx + 2][xr], tile[cx + 3][xr]);
+      } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (xcol + u < M.m) X[xrow * Gi.lp + xcol + u] = bf16_bits(tile[cx + u][xr]);
+      }
+    }
+  }
+  const float part = block_sum_f32(ss, shf);
+  if (threadIdx.x == 0) {
+    partials[t] = part;
+    __threadfence();
+    const unsigned int prev = atomicAdd(&counters[mi], 1u);
+    is_last = (prev + 1 == static_cast<unsigned int>(ntiles));
+  }
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  float acc = 0.f;
+  for (int64_t c = threadIdx.x; c < ntiles; c += kThreads) acc += __ldcg(partials + M.tile_begin + c);
+  const float total = block_sum_f32(acc, shf);
+  if (threadIdx.x == 0) {
+    const float nrm = sqrtf(total);
+    ginv[Gi.mbase + M.gidx] = nrm > 0.f ? 1.0f / nrm : 0.f;  // zero input: U = 0
+    counters[mi] = 0u;
+  }
+}
+
 // ------------------------------------------- remaining 2D parameters, vectors
 // B <- mu B + G (Eq. (10)) and the row sums of squares of B, one warp per row
 // (a vector is a single row). Row sums go to rvec.
@@ -164,27 +299,28 @@ __global__ void __launch_bounds__(kThreads) rows_kernel(const MatInfo* __restric
   if (lane == 0) rvec[M.vec_off + row] = ss;
 }
 
-// Column sums of squares of N_r(B) (Eq. (12), inner operator) per 32-row
-// slab, deterministic; rows with RMS at or below eps contribute nothing.
+// Column sums of squares of N_r(B) (Eq. (12), inner operator) per slab of
+// kColSlab rows, deterministic; rows with RMS at or below eps contribute
+// nothing.
 __global__ void __launch_bounds__(kThreads) colpart_kernel(const MatInfo* __restrict__ mats, int nmat,
                                                           const float* __restrict__ mom, const float* __restrict__ rvec,
                                                           const StepScalars* __restrict__ sc, float* __restrict__ parts) {
   pdl_allow_dependents();
   pdl_wait_predecessor();
-  __shared__ float rinv[32];
+  __shared__ float rinv[kColSlab];
   const int64_t slab = blockIdx.x;
   const int mi = find_mat(mats, nmat, slab, 4);
   const MatInfo& M = mats[mi];
   const int64_t ls = slab - M.slab_begin;
-  const int64_t r0 = ls * 32;
-  const int nr = static_cast<int>(M.m - r0 < 32 ? M.m - r0 : 32);
-  if (threadIdx.x < 32) {
+  const int64_t r0 = ls * kColSlab;
+  const int nr = static_cast<int>(M.m - r0 < kColSlab ? M.m - r0 : kColSlab);
+  for (int r = threadIdx.x; r < kColSlab; r += kThreads) {
     float v = 0.f;
-    if (static_cast<int>(threadIdx.x) < nr) {
-      const float rms = sqrtf(rvec[M.vec_off + r0 + threadIdx.x] / static_cast<float>(M.n));
+    if (r < nr) {
+      const float rms = sqrtf(rvec[M.vec_off + r0 + r] / static_cast<float>(M.n));
       v = rms > sc->eps ? 1.0f / rms : 0.f;
     }
-    rinv[threadIdx.x] = v;
+    rinv[r] = v;
   }
   __syncthreads();
   const float* B = mom + M.mom_off + r0 * M.n;
@@ -378,7 +514,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
       r[i] = rms;
       s[i] = rms > delta ? 1.0f / rms : 0.f;
     }
-    const int64_t nslabs = (M.m + 31) / 32;
+    const int64_t nslabs = (M.m + kColSlab - 1) / kColSlab;
     for (int64_t j = threadIdx.x; j < M.n; j += blockDim.x) {
       float acc = 0.f;
       for (int64_t k = 0; k < nslabs; ++k) acc += parts[M.cpart_off + k * M.n + j];
@@ -512,6 +648,11 @@ __global__ void wait_selftest_kernel(const volatile int* flag, int* err, unsigne
 cudaError_t launch_momentum_norm(const LaunchCtx& L, cudaStream_t st) {
   return launch_pdl(momentum_norm_kernel, dim3((unsigned)L.total_hchunks), dim3(kThreads), 0, st, 1, L.mats, L.nmat,
                     L.groups, L.mom, L.grads, L.sc, L.partials, L.counters, L.x0scale);
+}
+
+cudaError_t launch_momentum_x0(const LaunchCtx& L, cudaStream_t st) {
+  return launch_pdl(momentum_x0_kernel, dim3((unsigned)L.total_tiles), dim3(kThreads), 0, st, 1, L.mats, L.nmat,
+                    L.groups, L.mom, L.grads, L.sc, L.partials, L.counters, L.ginv);
 }
 
 cudaError_t launch_rows(const LaunchCtx& L, cudaStream_t st) {

@@ -43,6 +43,7 @@ struct Group {
   int trans = 0;           // members are tall (W = X^T)
   int64_t m = 0, n = 0, un = 0;  // weight shape of every member, U row stride
   int64_t u_base = 0;      // float offset of the group's U block [count][m][un]
+  int64_t mbase = 0;       // first slot of the group in the per-matrix inverse-norm array
   int64_t rpart_base = 0;  // float offsets of the fused-statistics partials
   int64_t cpart_base = 0;
   std::vector<int> mats;
@@ -91,6 +92,7 @@ struct meq_state {
   float* d_partials = nullptr;
   unsigned int* d_counters = nullptr;
   float* d_x0scale = nullptr;
+  float* d_ginv = nullptr;
   MatStats* d_stats = nullptr;
   char* d_step = nullptr;  // StepScalars, params[n], grads[n]
   int* d_err = nullptr;
@@ -131,6 +133,7 @@ bool valid_options(const meq_options& o, std::string* why) {
   if (!(o.wait_timeout_ms > 0.f)) { *why = "wait_timeout_ms must be > 0"; return false; }
   if (o.workspace_limit_bytes < 0) { *why = "workspace_limit_bytes must be >= 0"; return false; }
   if (o.ns_cta_pair != 0 && o.ns_cta_pair != 1) { *why = "ns_cta_pair must be 0 or 1"; return false; }
+  if (o.ns_x0_fused != 0 && o.ns_x0_fused != 1) { *why = "ns_x0_fused must be 0 or 1"; return false; }
   return true;
 }
 
@@ -209,6 +212,11 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
     st->groups[g].mats.push_back(i);
   }
   int64_t mom = 0, u = 0, vec = 0, parts = 0, chunks = 0, hchunks = 0, tiles = 0, rblks = 0, slabs = 0;
+  int64_t mslots = 0;
+  for (auto& G : st->groups) {
+    G.mbase = mslots;
+    mslots += G.count;
+  }
   for (auto& G : st->groups) {  // U is stored group by group: [count][m][un]
     G.u_base = u;
     u += round_up(G.count * G.m * G.un, 64);
@@ -241,7 +249,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
       M.un = M.n;
       rblks += (M.m + 7) / 8;  // 8 rows (warps) per block
       if (M.kind == KIND_TWO_SIDED) {
-        const int64_t ns = (M.m + 31) / 32;
+        const int64_t ns = (M.m + kColSlab - 1) / kColSlab;
         M.cpart_off = parts;
         parts += round_up(ns * M.n, 64);
         slabs += ns;
@@ -258,9 +266,9 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
   *off_u = L->add(u * 4);
   *off_vec4 = L->add(vec * 4 * 4);  // r, c, s, t
   *off_cpart = L->add(parts * 4);
-  *off_partials = L->add(hchunks * 4);
+  *off_partials = L->add(std::max(hchunks, tiles) * 4);  // per momentum chunk or fused tile
   *off_counters = L->add(int64_t(n) * 4);
-  *off_x0s = L->add(int64_t(n) * 4);
+  *off_x0s = L->add(int64_t(n) * 4 * 2);  // x0scale (cast pass) and the inverse norms (fused)
   *off_stats = L->add(int64_t(n) * sizeof(MatStats));
   st->step_bytes = sizeof(StepScalars) + 2 * int64_t(n) * sizeof(void*);
   *off_step = L->add(st->step_bytes);
@@ -334,18 +342,23 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
   const int pair = st->opt.ns_cta_pair ? 2 : 1;
   const int tile_m = 128 * pair;
   const uint32_t b_rows = static_cast<uint32_t>(256 / pair);  // K-major B rows each CTA loads
+  const bool fused = st->opt.ns_x0_fused != 0;
+  // 16-bit formats: dA(k) of A_k (and of the polynomial's operands) is the
+  // iteration's format; dX(k) of X_k (and of P_k, which multiplies it) too,
+  // except that a fused X_0 is bf16 (written unnormalised by the momentum pass).
+  auto dA = [&](int k) { return iter_fp16(st->opt, k); };
+  auto dX = [&](int k) { return (fused && k == 0) ? false : iter_fp16(st->opt, k); };
   for (int k = 0; k < K; ++k) {
-    const bool f16 = iter_fp16(st->opt, k);
-    const bool next_f16 = (k + 1 < K) ? iter_fp16(st->opt, k + 1) : false;
     const int cur = k & 1, nxt = cur ^ 1;
     for (int mode = MODE_GRAM; mode <= MODE_XUPD; ++mode) {
       const int real_mode = (mode == MODE_XUPD && k == K - 1) ? MODE_XLAST : mode;
+      const bool in16 = mode == MODE_POLY ? dA(k) : dX(k);  // operand format of this launch
       for (int g0 = 0; g0 < ng; g0 += kMaxGroups) {
         GemmParams P;
         std::memset(&P, 0, sizeof(P));
         P.mode = real_mode;
         P.b_mn_major = (mode == MODE_XUPD) ? 1 : 0;
-        P.idesc = make_idesc(f16, P.b_mn_major, tile_m);
+        P.idesc = make_idesc(in16, P.b_mn_major, tile_m);
         P.ca = st->opt.ns_a, P.cb = st->opt.ns_b, P.cc = st->opt.ns_c;
         P.err = st->d_err;
         P.timeout_ns = static_cast<unsigned long long>(static_cast<double>(st->opt.wait_timeout_ms) * 1e6);
@@ -354,7 +367,9 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
         for (int gi = 0; gi < P.ngroups; ++gi) {
           Group& G = st->groups[g0 + gi];
           GemmGroup& Q = P.g[gi];
-          const float ak = (k == 0) ? G.alpha0 : G.alpha;
+          // storage scale of X_k; a fused X_0 is unscaled and its 1/||H||_F is applied per matrix
+          const float ak = (k == 0) ? (fused ? 1.0f : G.alpha0) : G.alpha;
+          const bool per_matrix = fused && k == 0;
           Q.count = static_cast<int32_t>(G.count);
           Q.trans = G.trans;
           bool ok = true;
@@ -367,7 +382,8 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             ok &= encode_map(&Q.tmB, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, b_rows, SW128);
             Q.out = G.a16, Q.out_ld = s_ld, Q.out_mstride = s_ms;
             Q.scale = 1.0f / (ak * ak);
-            Q.out_fp16 = f16;
+            if (per_matrix) Q.minv = st->d_ginv + G.mbase, Q.minv_pow = 2;
+            Q.out_fp16 = dA(k);
           } else if (mode == MODE_POLY) {
             Q.M = (int32_t)G.s, Q.N = (int32_t)G.s, Q.K = (int32_t)G.s;
             Q.sym = 1;
@@ -376,7 +392,8 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             Q.out = G.p16, Q.out_ld = s_ld, Q.out_mstride = s_ms;
             Q.aux = G.a16, Q.aux_ld = s_ld, Q.aux_mstride = s_ms;
             Q.scale = 1.0f;
-            Q.out_fp16 = f16;
+            Q.out_fp16 = dX(k);
+            Q.aux_fp16 = dA(k);
           } else {
             Q.M = (int32_t)G.s, Q.N = (int32_t)G.l, Q.K = (int32_t)G.s;
             Q.sym = 0;
@@ -385,10 +402,12 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             if (real_mode == MODE_XUPD) {
               Q.out = G.x[nxt], Q.out_ld = x_ld, Q.out_mstride = x_ms;
               Q.scale = G.alpha / ak;
-              Q.out_fp16 = next_f16;
+              if (per_matrix) Q.minv = st->d_ginv + G.mbase, Q.minv_pow = 1;
+              Q.out_fp16 = dX(k + 1);
             } else {
               Q.out = st->d_u + G.u_base, Q.out_ld = G.un * 4, Q.out_mstride = G.m * G.un * 4;
               Q.scale = 1.0f / ak;
+              if (per_matrix) Q.minv = st->d_ginv + G.mbase, Q.minv_pow = 1;
               Q.out_fp16 = 0;
               Q.rpart = st->d_parts + G.rpart_base;
               Q.cpart = st->d_parts + G.cpart_base;
@@ -436,6 +455,7 @@ void meq_default_options(meq_options* o) {
   o->workspace_limit_bytes = 0;
   o->wait_timeout_ms = 4000.f;
   o->ns_cta_pair = 1;
+  o->ns_x0_fused = 1;
 }
 
 const char* meq_status_string(meq_status s) {
@@ -546,6 +566,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   st->d_partials = reinterpret_cast<float*>(A + off_partials);
   st->d_counters = reinterpret_cast<unsigned int*>(A + off_counters);
   st->d_x0scale = reinterpret_cast<float*>(A + off_x0s);
+  st->d_ginv = st->d_x0scale + n;
   st->d_stats = reinterpret_cast<MatStats*>(A + off_stats);
   st->d_step = A + off_step;
   st->d_err = reinterpret_cast<int*>(A + off_err);
@@ -567,6 +588,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
     gi[g].s = G.s, gi[g].l = G.l, gi[g].lp = G.lp, gi[g].sp = G.sp, gi[g].count = G.count;
     gi[g].x0 = G.x[0];
     gi[g].alpha0 = G.alpha0;
+    gi[g].mbase = G.mbase;
   }
   bool ok = cudaMemsetAsync(st->arena, 0, static_cast<size_t>(L.total), s) == cudaSuccess;
   ok = ok && cudaMemcpyAsync(st->d_mats, st->mats.data(), sizeof(MatInfo) * n, cudaMemcpyHostToDevice, s) == cudaSuccess;
@@ -595,6 +617,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   C.partials = st->d_partials;
   C.counters = st->d_counters;
   C.x0scale = st->d_x0scale;
+  C.ginv = st->d_ginv;
   C.uslab = st->d_u;
   C.parts = st->d_parts;
   C.rvec = st->d_rvec;
@@ -607,7 +630,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   C.total_tiles = st->total_tiles;
   C.total_rblks = st->total_rblks;
   C.total_slabs = st->total_slabs;
-  st->kernels_per_step = (st->n_hidden ? 2 : 0) + (st->n_rows ? 1 : 0) + (st->n_two ? 1 : 0) + 2 +
+  st->kernels_per_step = (st->n_hidden ? (o.ns_x0_fused ? 1 : 2) : 0) + (st->n_rows ? 1 : 0) + (st->n_two ? 1 : 0) + 2 +
                          static_cast<int>(st->gemm.size());
   st->step_host.assign(static_cast<size_t>(st->step_bytes), 0);
   st->last_stream = s;
@@ -627,16 +650,17 @@ static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev
   auto mark = [&](int i) { if (ev) cudaEventRecord(ev[i], s); };
   cudaError_t e = cudaSuccess;
   mark(0);
+  const bool fused = st->opt.ns_x0_fused != 0;
   if (st->n_hidden) {
-    e = launch_momentum_norm(C, s);
-    if (e != cudaSuccess) return cuda_fail(st, e, "momentum_norm launch");
+    e = fused ? launch_momentum_x0(C, s) : launch_momentum_norm(C, s);
+    if (e != cudaSuccess) return cuda_fail(st, e, "momentum launch");
   }
   if (st->n_rows) {
     e = launch_rows(C, s);
     if (e != cudaSuccess) return cuda_fail(st, e, "rows launch");
   }
   mark(1);
-  if (st->n_hidden) {
+  if (st->n_hidden && !fused) {
     e = launch_cast_x0(C, iter_fp16(st->opt, 0), s);
     if (e != cudaSuccess) return cuda_fail(st, e, "cast_x0 launch");
   }

@@ -8,6 +8,7 @@ namespace meq {
 constexpr int64_t kChunk = 4096;   // elements per momentum / apply block
 constexpr int kCastTile = 64;      // X_0 cast tile (64 x 64 of W)
 constexpr int kFinThreads = 1024;  // finalize block size
+constexpr int kColSlab = 256;      // rows per block of the remaining-2D column pass
 
 struct MatStats {
   double gamma_r;
@@ -28,6 +29,7 @@ struct LaunchCtx {
   float* partials;
   unsigned int* counters;
   float* x0scale;
+  float* ginv;           // 1 / ||H||_F per hidden matrix, ordered group by group
   float* uslab;
   float* parts;          // NS-row and NS-column partial sums of squares
   float* rvec;
@@ -41,6 +43,7 @@ struct LaunchCtx {
 constexpr int KIND_HIDDEN = 0, KIND_TWO_SIDED = 1, KIND_VECTOR = 2;
 
 cudaError_t launch_momentum_norm(const LaunchCtx& L, cudaStream_t st);
+cudaError_t launch_momentum_x0(const LaunchCtx& L, cudaStream_t st);  // fused momentum + bf16 X_0
 cudaError_t launch_rows(const LaunchCtx& L, cudaStream_t st);      // remaining 2D + vectors
 cudaError_t launch_colpart(const LaunchCtx& L, cudaStream_t st);   // remaining 2D
 cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st);

@@ -41,11 +41,11 @@ struct MatInfo {
   int64_t chunk_begin;   // first apply chunk (all kinds)
   int64_t hchunk_begin;  // first momentum-and-norm chunk (hidden weights only)
   int64_t rblk_begin;    // first 8-row block of the row pass (remaining 2D and vectors)
-  int64_t slab_begin;    // first 32-row slab of the column pass (remaining 2D only)
+  int64_t slab_begin;    // first row slab of the column pass (remaining 2D only)
   int64_t tile_begin;    // first cast tile (hidden weights only)
   int64_t rpart_off;     // float offset of NS-row partial sums of squares [2 * ceil(l/256)][s]
   int64_t cpart_off;     // float offset of column partial sums of squares: NS columns
-                         // [ceil(s/32)][l] (hidden) or normalised columns [ceil(m/32)][n] (remaining 2D)
+                         // [ceil(s/32)][l] (hidden) or normalised columns [slabs][n] (remaining 2D)
 };
 
 // Per-group metadata for the elementwise kernels.
@@ -53,7 +53,8 @@ struct GroupInfo {
   int64_t s, l, lp, sp;  // shape and padded row strides (elements)
   int64_t count;
   void* x0;              // X-hat buffer 0: [count][s][lp] 16-bit
-  float alpha0;          // power-of-two storage scale of X_0
+  float alpha0;          // power-of-two storage scale of X_0 (separate cast pass)
+  int64_t mbase;         // offset of the group's matrices in the inverse-norm array
 };
 
 // Values that change per step (uploaded before each step).
@@ -78,7 +79,10 @@ struct GemmGroup {
   int32_t sym;            // 1: symmetric s x s output (upper-triangle tiles, mirrored stores)
   int32_t trans;          // XLAST: 1 when the weight is the transpose of the NS layout
   float scale;            // GRAM: 1/alpha^2; XUPD: alpha_next/alpha; XLAST: 1/alpha
-  int32_t out_fp16;       // 16-bit format of the output / aux operand (1 = fp16, 0 = bf16)
+  const float* minv;      // iteration 0 with X_0 unnormalised: 1/||H||_F per matrix of the group
+  int32_t minv_pow;       // epilogue scale *= minv^minv_pow (0, 1 or 2)
+  int32_t out_fp16;       // 16-bit format of the output (1 = fp16, 0 = bf16)
+  int32_t aux_fp16;       // POLY: 16-bit format of the A it reads in the epilogue
   void* out;              // GRAM: 16-bit A; POLY: 16-bit P; XUPD: 16-bit X next; XLAST: fp32 U (weight layout)
   int64_t out_ld;         // output row stride in bytes
   int64_t out_mstride;    // output matrix stride in bytes

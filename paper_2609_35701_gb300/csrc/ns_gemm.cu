@@ -605,7 +605,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
             const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
             for (int h = 0; h < 4; ++h) {
-              const float2 a2 = unpack_half2(ws[h], G.out_fp16);
+              const float2 a2 = unpack_half2(ws[h], G.aux_fp16);
               const int j = 8 * k + 2 * h;
               v[j] = fmaf(p.cc, v[j], fmaf(p.cb, a2.x, (col0 + j == row) ? p.ca : 0.f));
               v[j + 1] = fmaf(p.cc, v[j + 1], fmaf(p.cb, a2.y, (col0 + j + 1 == row) ? p.ca : 0.f));
@@ -613,8 +613,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
           }
           __syncwarp();  // slot free for the output block
         } else {
+          float sc = G.scale;
+          if (G.minv_pow) {
+            const float iv = G.minv[c.mat];
+            sc *= G.minv_pow == 2 ? iv * iv : iv;
+          }
 #pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] *= G.scale;
+          for (int j = 0; j < 32; ++j) v[j] *= sc;
         }
         if (mode == MODE_XLAST) {
           // Column sums of squares over the warp's 32 rows: transpose-reduce

@@ -40,6 +40,7 @@ class MeqOptions(ctypes.Structure):
         ("workspace_limit_bytes", ctypes.c_int64),
         ("wait_timeout_ms", ctypes.c_float),
         ("ns_cta_pair", ctypes.c_int),
+        ("ns_x0_fused", ctypes.c_int),
     ]
 
 
