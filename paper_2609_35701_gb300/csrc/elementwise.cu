@@ -299,40 +299,49 @@ __global__ void __launch_bounds__(kThreads) rows_kernel(const MatInfo* __restric
   if (lane == 0) rvec[M.vec_off + row] = ss;
 }
 
-// Column sums of squares of N_r(B) (Eq. (12), inner operator) per slab of
-// kColSlab rows, deterministic; rows with RMS at or below eps contribute
-// nothing.
+// Column sums of squares of N_r(B) (Eq. (12), inner operator): one block per
+// kColSlab rows x 256 columns, deterministic; rows with RMS at or below eps
+// contribute nothing.
 __global__ void __launch_bounds__(kThreads) colpart_kernel(const MatInfo* __restrict__ mats, int nmat,
                                                           const float* __restrict__ mom, const float* __restrict__ rvec,
                                                           const StepScalars* __restrict__ sc, float* __restrict__ parts) {
   pdl_allow_dependents();
   pdl_wait_predecessor();
   __shared__ float rinv[kColSlab];
-  const int64_t slab = blockIdx.x;
-  const int mi = find_mat(mats, nmat, slab, 4);
+  const int64_t blk = blockIdx.x;
+  const int mi = find_mat(mats, nmat, blk, 4);
   const MatInfo& M = mats[mi];
-  const int64_t ls = slab - M.slab_begin;
+  const int64_t ncc = (M.n + kThreads - 1) / kThreads;  // column chunks
+  const int64_t lb = blk - M.slab_begin;
+  const int64_t ls = lb / ncc;
+  const int64_t c = (lb - ls * ncc) * kThreads + threadIdx.x;
   const int64_t r0 = ls * kColSlab;
   const int nr = static_cast<int>(M.m - r0 < kColSlab ? M.m - r0 : kColSlab);
-  for (int r = threadIdx.x; r < kColSlab; r += kThreads) {
+  for (int rr = threadIdx.x; rr < kColSlab; rr += kThreads) {
     float v = 0.f;
-    if (r < nr) {
-      const float rms = sqrtf(rvec[M.vec_off + r0 + r] / static_cast<float>(M.n));
+    if (rr < nr) {
+      const float rms = sqrtf(rvec[M.vec_off + r0 + rr] / static_cast<float>(M.n));
       v = rms > sc->eps ? 1.0f / rms : 0.f;
     }
-    rinv[r] = v;
+    rinv[rr] = v;
   }
   __syncthreads();
-  const float* B = mom + M.mom_off + r0 * M.n;
-  float* cp = parts + M.cpart_off + ls * M.n;
-  for (int64_t c = threadIdx.x; c < M.n; c += kThreads) {
-    float acc = 0.f;
-    for (int r = 0; r < nr; ++r) {
-      const float x = B[r * M.n + c] * rinv[r];
-      acc += x * x;
+  if (c >= M.n) return;
+  const float* B = mom + M.mom_off + r0 * M.n + c;
+  float a4[4] = {0.f, 0.f, 0.f, 0.f};
+  int r = 0;
+  for (; r + 8 <= nr; r += 8) {
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const float x = B[(r + u) * M.n] * rinv[r + u];
+      a4[u & 3] += x * x;
     }
-    cp[c] = acc;
   }
+  for (; r < nr; ++r) {
+    const float x = B[r * M.n] * rinv[r];
+    a4[r & 3] += x * x;
+  }
+  parts[M.cpart_off + ls * M.n + c] = (a4[0] + a4[1]) + (a4[2] + a4[3]);
 }
 
 // ------------------------------------------------------------------ X_0 cast
@@ -514,11 +523,20 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
       r[i] = rms;
       s[i] = rms > delta ? 1.0f / rms : 0.f;
     }
+    // Column sums over the slabs, eight independent partial sums per thread
+    // (slab k goes to accumulator k % 8) so loads overlap; fixed order.
     const int64_t nslabs = (M.m + kColSlab - 1) / kColSlab;
     for (int64_t j = threadIdx.x; j < M.n; j += blockDim.x) {
-      float acc = 0.f;
-      for (int64_t k = 0; k < nslabs; ++k) acc += parts[M.cpart_off + k * M.n + j];
-      const float rms = sqrtf(acc * inv_m);
+      const float* pj = parts + M.cpart_off + j;
+      float a8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      int64_t k = 0;
+      for (; k + 8 <= nslabs; k += 8) {
+#pragma unroll
+        for (int u = 0; u < 8; ++u) a8[u] += pj[(k + u) * M.n];
+      }
+      for (; k < nslabs; ++k) a8[k & 7] += pj[k * M.n];
+      const float tot = ((a8[0] + a8[1]) + (a8[2] + a8[3])) + ((a8[4] + a8[5]) + (a8[6] + a8[7]));
+      const float rms = sqrtf(tot * inv_m);
       c[j] = rms;
       t[j] = rms > delta ? 1.0f / rms : 0.f;
     }

@@ -252,7 +252,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
         const int64_t ns = (M.m + kColSlab - 1) / kColSlab;
         M.cpart_off = parts;
         parts += round_up(ns * M.n, 64);
-        slabs += ns;
+        slabs += ns * ((M.n + 255) / 256);  // blocks: slab x 256-column chunk
       }
     }
   }

@@ -8,7 +8,7 @@ namespace meq {
 constexpr int64_t kChunk = 4096;   // elements per momentum / apply block
 constexpr int kCastTile = 64;      // X_0 cast tile (64 x 64 of W)
 constexpr int kFinThreads = 1024;  // finalize block size
-constexpr int kColSlab = 256;      // rows per block of the remaining-2D column pass
+constexpr int kColSlab = 128;      // rows per block of the remaining-2D column pass
 
 struct MatStats {
   double gamma_r;
