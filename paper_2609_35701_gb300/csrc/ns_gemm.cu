@@ -76,9 +76,6 @@ __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
 __device__ __forceinline__ uint32_t mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -165,8 +162,12 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t smem_addr, uint32_t ran
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+// Accumulator release by the epilogue. Only the warp's tcgen05.ld reads must
+// precede it, and tcgen05.wait::ld has already completed them; a release
+// would also hold the warp until its earlier global stores are visible to
+// the cluster, which the MMA issuer does not need.
+__device__ __forceinline__ void mbar_arrive_relaxed_cluster(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* tm) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
@@ -682,8 +683,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
-        if (kPair == 2) mbar_arrive_cluster(acc == 0 ? tempty_target0 : tempty_target1);
-        else mbar_arrive(TEMPTY_BAR(acc));
+        mbar_arrive_relaxed_cluster(kPair == 2 ? (acc == 0 ? tempty_target0 : tempty_target1) : TEMPTY_BAR(acc));
       }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
