@@ -143,7 +143,10 @@ meq_status meq_read_momentum(meq_state* st, int i, float* dst);
 /* Overwrite momentum B_i from src (host or device), e.g. to resume. */
 meq_status meq_write_momentum(meq_state* st, int i, const float* src);
 /* Copy the last step's Newton-Schulz output U_i (rows x cols fp32, before
- * equilibration) to dst (host or device). Hidden weights only. */
+ * equilibration) to dst (host or device). Hidden weights only. U is held on
+ * the device in fp16 (scaled by 2^14, so every entry above 4e-9 keeps 11
+ * significant bits); the values returned are those fp16 values, from which
+ * the row and column statistics are taken and which the update applies. */
 meq_status meq_read_ns_output(meq_state* st, int i, float* dst);
 /* Last step's statistics of entry i. Hidden weight: r (rows floats), c (cols
  * floats) of Eq. (7) for U, gamma_r, gamma_c of Eq. (8) and the direction of

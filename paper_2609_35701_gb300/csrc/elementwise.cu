@@ -30,7 +30,8 @@ __device__ __forceinline__ int find_mat(const MatInfo* mats, int nmat, int64_t k
                       : which == 1 ? mats[mid].tile_begin
                       : which == 2 ? mats[mid].hchunk_begin
                       : which == 3 ? mats[mid].rblk_begin
-                                   : mats[mid].slab_begin;
+                      : which == 4 ? mats[mid].slab_begin
+                                   : mats[mid].xblk_begin;
     if (b <= key) lo = mid; else hi = mid - 1;
   }
   return lo;
@@ -138,93 +139,115 @@ __device__ __forceinline__ uint16_t bf16_bits(float v) {
   return *reinterpret_cast<uint16_t*>(&h);
 }
 
-// Hidden weights, one 64 x 64 tile of W per block: B <- mu B + G (Eq. (10))
-// and X_0 = bf16(H) in the oriented NS layout (tall W transposed through
-// shared memory), H being the NS input (B, or G + mu B for Nesterov). X_0 is
-// left unnormalised: bf16 has the exponent range of fp32, and the first NS
-// products apply 1 / ||H||_F (Eq. (5)) in their epilogues. The squared norm
-// is reduced per tile in fixed order; the last tile of a matrix writes
-// 1 / ||H||_F (0 for a zero input) to ginv.
-__global__ void __launch_bounds__(kThreads) momentum_x0_kernel(const MatInfo* __restrict__ mats, int nmat,
-                                                              const GroupInfo* __restrict__ groups,
-                                                              float* __restrict__ mom,
-                                                              const float* const* __restrict__ grads,
-                                                              const StepScalars* __restrict__ sc,
-                                                              float* __restrict__ partials,
-                                                              unsigned int* __restrict__ counters,
-                                                              float* __restrict__ ginv) {
+// Hidden weights: B <- mu B + G (Eq. (10)) and X_0 = bf16(H) in the
+// oriented NS layout, H being the NS input (B, or G + mu B for Nesterov).
+// X_0 is left unnormalised: bf16 has the exponent range of fp32, and the
+// first NS products apply 1 / ||H||_F (Eq. (5)) in their epilogues.
+// Block t of the enumeration is a flat chunk of kChunk elements of W when
+// X_0 has W's layout (B and G are contiguous, so they move as float4s
+// whatever the row length), or a 64 x 64 tile of W transposed through shared
+// memory when X_0 = W^T (tall W). Each block writes the fixed-order sum of
+// squares of its part of H to partials[t]; x0norm_kernel reduces them.
+__global__ void __launch_bounds__(kThreads, 8) momentum_x0_kernel(const MatInfo* __restrict__ mats, int nmat,
+                                                                 const GroupInfo* __restrict__ groups,
+                                                                 float* __restrict__ mom,
+                                                                 const float* const* __restrict__ grads,
+                                                                 const StepScalars* __restrict__ sc,
+                                                                 float* __restrict__ partials) {
   pdl_allow_dependents();
   pdl_wait_predecessor();
   __shared__ float tile[kCastTile][kCastTile + 1];
   __shared__ float shf[32];
-  __shared__ int is_last;
   const int64_t t = blockIdx.x;
-  const int mi = find_mat(mats, nmat, t, 1);
+  const int mi = find_mat(mats, nmat, t, 5);
   const MatInfo& M = mats[mi];
   const GroupInfo& Gi = groups[M.group];
-  const int64_t tiles_n = (M.n + kCastTile - 1) / kCastTile;
-  const int64_t ntiles = ((M.m + kCastTile - 1) / kCastTile) * tiles_n;
-  const int64_t lt = t - M.tile_begin;
-  const int64_t r0 = (lt / tiles_n) * kCastTile;
-  const int64_t c0 = (lt % tiles_n) * kCastTile;
+  const int64_t lt = t - M.xblk_begin;
   const float mu = sc->mu;
   const int nesterov = sc->nesterov;
   float* B = mom + M.mom_off;
   const float* G = grads[mi];
   uint16_t* X = static_cast<uint16_t*>(Gi.x0) + M.gidx * Gi.s * Gi.lp;
-  const bool vec = (M.n & 3) == 0;
-  const int cx = (threadIdx.x & 15) * 4;  // 4 columns
-  const int ry = threadIdx.x >> 4;        // rows ry, ry + 16, ry + 32, ry + 48
-  float h[4][4];
   float ss = 0.f;
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const int64_t row = r0 + ry + 16 * k, col = c0 + cx;
-#pragma unroll
-    for (int u = 0; u < 4; ++u) h[k][u] = 0.f;
-    if (row >= M.m) continue;
-    if (vec && col + 3 < M.n) {
-      const float4 g = __ldcs(reinterpret_cast<const float4*>(G + row * M.n + col));
-      float4 b = *reinterpret_cast<const float4*>(B + row * M.n + col);
-      b.x = fmaf(mu, b.x, g.x), b.y = fmaf(mu, b.y, g.y), b.z = fmaf(mu, b.z, g.z), b.w = fmaf(mu, b.w, g.w);
-      *reinterpret_cast<float4*>(B + row * M.n + col) = b;
-      if (nesterov) {
-        h[k][0] = fmaf(mu, b.x, g.x), h[k][1] = fmaf(mu, b.y, g.y), h[k][2] = fmaf(mu, b.z, g.z);
-        h[k][3] = fmaf(mu, b.w, g.w);
-      } else {
-        h[k][0] = b.x, h[k][1] = b.y, h[k][2] = b.z, h[k][3] = b.w;
-      }
-    } else {
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (col + u < M.n) {
-          const float g = G[row * M.n + col + u];
-          const float b = fmaf(mu, B[row * M.n + col + u], g);
-          B[row * M.n + col + u] = b;
-          h[k][u] = nesterov ? fmaf(mu, b, g) : b;
-        }
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) ss += h[k][u] * h[k][u];
-  }
   if (!M.trans) {
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int64_t row = r0 + ry + 16 * k, col = c0 + cx;
-      if (row >= M.m) continue;
-      if (col + 3 < M.n) {
-        *reinterpret_cast<uint2*>(X + row * Gi.lp + col) = pack4_bf16(h[k][0], h[k][1], h[k][2], h[k][3]);
+    const int64_t e0 = lt * kChunk;
+    const int64_t e1 = min(e0 + kChunk, M.m * M.n);
+    for (int64_t e = e0 + 4 * threadIdx.x; e < e1; e += 4 * kThreads) {
+      float h[4];
+      if (e + 3 < e1) {
+        const float4 g = __ldcs(reinterpret_cast<const float4*>(G + e));
+        float4 b = *reinterpret_cast<const float4*>(B + e);
+        b.x = fmaf(mu, b.x, g.x), b.y = fmaf(mu, b.y, g.y), b.z = fmaf(mu, b.z, g.z), b.w = fmaf(mu, b.w, g.w);
+        *reinterpret_cast<float4*>(B + e) = b;
+        if (nesterov) {
+          h[0] = fmaf(mu, b.x, g.x), h[1] = fmaf(mu, b.y, g.y), h[2] = fmaf(mu, b.z, g.z), h[3] = fmaf(mu, b.w, g.w);
+        } else {
+          h[0] = b.x, h[1] = b.y, h[2] = b.z, h[3] = b.w;
+        }
       } else {
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
-          if (col + u < M.n) X[row * Gi.lp + col + u] = bf16_bits(h[k][u]);
+        for (int u = 0; u < 4; ++u) {
+          h[u] = 0.f;
+          if (e + u < e1) {
+            const float g = G[e + u];
+            const float b = fmaf(mu, B[e + u], g);
+            B[e + u] = b;
+            h[u] = nesterov ? fmaf(mu, b, g) : b;
+          }
+        }
+      }
+      ss += h[0] * h[0] + h[1] * h[1] + h[2] * h[2] + h[3] * h[3];
+      int64_t i = e / M.n, j = e - i * M.n;
+      if ((M.n & 3) == 0) {
+        // four columns of one row (m n is then a multiple of 4, so e + 3 < e1)
+        *reinterpret_cast<uint2*>(X + i * Gi.lp + j) = pack4_bf16(h[0], h[1], h[2], h[3]);
+      } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          if (e + u < e1) X[i * Gi.lp + j] = bf16_bits(h[u]);
+          if (++j == M.n) j = 0, ++i;
+        }
       }
     }
   } else {
+    const int64_t tiles_n = (M.n + kCastTile - 1) / kCastTile;
+    const int64_t r0 = (lt / tiles_n) * kCastTile;
+    const int64_t c0 = (lt % tiles_n) * kCastTile;
+    const bool vec = (M.n & 3) == 0;
+    const int cx = (threadIdx.x & 15) * 4;  // 4 columns
+    const int ry = threadIdx.x >> 4;        // rows ry, ry + 16, ry + 32, ry + 48
 #pragma unroll
-    for (int k = 0; k < 4; ++k)
+    for (int k = 0; k < 4; ++k) {
+      const int64_t row = r0 + ry + 16 * k, col = c0 + cx;
+      float h[4] = {0.f, 0.f, 0.f, 0.f};
+      if (row < M.m) {
+        if (vec && col + 3 < M.n) {
+          const float4 g = __ldcs(reinterpret_cast<const float4*>(G + row * M.n + col));
+          float4 b = *reinterpret_cast<const float4*>(B + row * M.n + col);
+          b.x = fmaf(mu, b.x, g.x), b.y = fmaf(mu, b.y, g.y), b.z = fmaf(mu, b.z, g.z), b.w = fmaf(mu, b.w, g.w);
+          *reinterpret_cast<float4*>(B + row * M.n + col) = b;
+          if (nesterov) {
+            h[0] = fmaf(mu, b.x, g.x), h[1] = fmaf(mu, b.y, g.y), h[2] = fmaf(mu, b.z, g.z), h[3] = fmaf(mu, b.w, g.w);
+          } else {
+            h[0] = b.x, h[1] = b.y, h[2] = b.z, h[3] = b.w;
+          }
+        } else {
 #pragma unroll
-      for (int u = 0; u < 4; ++u) tile[ry + 16 * k][cx + u] = h[k][u];
+          for (int u = 0; u < 4; ++u)
+            if (col + u < M.n) {
+              const float g = G[row * M.n + col + u];
+              const float b = fmaf(mu, B[row * M.n + col + u], g);
+              B[row * M.n + col + u] = b;
+              h[u] = nesterov ? fmaf(mu, b, g) : b;
+            }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        ss += h[u] * h[u];
+        tile[ry + 16 * k][cx + u] = h[u];
+      }
+    }
     __syncthreads();
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
@@ -242,22 +265,30 @@ __global__ void __launch_bounds__(kThreads) momentum_x0_kernel(const MatInfo* __
     }
   }
   const float part = block_sum_f32(ss, shf);
-  if (threadIdx.x == 0) {
-    partials[t] = part;
-    __threadfence();
-    const unsigned int prev = atomicAdd(&counters[mi], 1u);
-    is_last = (prev + 1 == static_cast<unsigned int>(ntiles));
-  }
-  __syncthreads();
-  if (!is_last) return;
-  __threadfence();
+  if (threadIdx.x == 0) partials[t] = part;
+}
+
+// 1 / ||H||_F of every hidden matrix (0 for a zero input, whose U is 0), one
+// block per matrix: fixed-order fp32 reduction of the partials its momentum
+// blocks wrote (fp32 throughout: this GPU's fp64 rate is a small fraction of
+// its fp32 rate).
+__global__ void __launch_bounds__(kThreads) x0norm_kernel(const MatInfo* __restrict__ mats,
+                                                         const GroupInfo* __restrict__ groups,
+                                                         const float* __restrict__ partials,
+                                                         float* __restrict__ ginv) {
+  pdl_allow_dependents();
+  pdl_wait_predecessor();
+  __shared__ float shf[32];
+  const MatInfo& M = mats[blockIdx.x];
+  if (M.kind != KIND_HIDDEN) return;
+  const int64_t nblk = M.trans ? ((M.m + kCastTile - 1) / kCastTile) * ((M.n + kCastTile - 1) / kCastTile)
+                               : (M.m * M.n + kChunk - 1) / kChunk;
   float acc = 0.f;
-  for (int64_t c = threadIdx.x; c < ntiles; c += kThreads) acc += __ldcg(partials + M.tile_begin + c);
+  for (int64_t c = threadIdx.x; c < nblk; c += kThreads) acc += partials[M.xblk_begin + c];
   const float total = block_sum_f32(acc, shf);
   if (threadIdx.x == 0) {
     const float nrm = sqrtf(total);
-    ginv[Gi.mbase + M.gidx] = nrm > 0.f ? 1.0f / nrm : 0.f;  // zero input: U = 0
-    counters[mi] = 0u;
+    ginv[groups[M.group].mbase + M.gidx] = nrm > 0.f ? 1.0f / nrm : 0.f;
   }
 }
 
@@ -587,9 +618,9 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
 // ----------------------------------------------------------------------- apply
 // W <- (1 - lr wd) W - rho lr U~ (Eq. (14)), U~ = scaled U (hidden) or scaled
 // B (remaining 2D: s_i t_j B_ij; vector: s_0 B_j).
-__global__ void __launch_bounds__(kThreads) apply_kernel(const MatInfo* __restrict__ mats, int nmat,
+__global__ void __launch_bounds__(kThreads, 8) apply_kernel(const MatInfo* __restrict__ mats, int nmat,
                                                          float* const* __restrict__ params,
-                                                         const float* __restrict__ uslab,
+                                                         const uint16_t* __restrict__ uslab,
                                                          const float* __restrict__ mom,
                                                          const float* __restrict__ svec,
                                                          const float* __restrict__ tvec,
@@ -604,21 +635,31 @@ __global__ void __launch_bounds__(kThreads) apply_kernel(const MatInfo* __restri
   const int64_t e0 = (chunk - M.chunk_begin) * kChunk;
   const int64_t e1 = min(e0 + kChunk, numel);
   const float decay = 1.0f - sc->lr * sc->wd;
-  const float step = sc->rho * sc->lr;
   const bool hidden = M.kind == KIND_HIDDEN;
+  // hidden: U is fp16(kUScale U) with row stride un; others: the momentum, fp32, contiguous
+  const float step = sc->rho * sc->lr * (hidden ? 1.0f / kUScale : 1.0f);
   // mode 0: per-row scale; 1: per-column scale; 2: row scale x column scale
   const int mode = hidden ? stats[mi].direction : (M.kind == KIND_TWO_SIDED ? 2 : 0);
   const float* sv = svec + M.vec_off;
   const float* tv = tvec + M.vec_off;
-  const float* U = hidden ? uslab + M.u_off : mom + M.mom_off;
-  const int64_t ustride = hidden ? M.un : M.n;
+  const uint16_t* U16 = uslab + M.u_off;
+  const float* U32 = mom + M.mom_off;
   float* W = params[mi];
   if ((M.n & 3) == 0) {
-    // Rows are whole float4s and the U stride equals n.
+    // four columns of one row per thread (m n is a multiple of 4, so e + 3 < e1)
     for (int64_t e = e0 + 4 * threadIdx.x; e < e1; e += 4 * kThreads) {
       const int64_t i = e / M.n, j = e - i * M.n;
       float4 w = *reinterpret_cast<const float4*>(W + e);
-      const float4 u = __ldcs(reinterpret_cast<const float4*>(U + e));
+      float u[4];
+      if (hidden) {
+        const uint2 h = __ldcs(reinterpret_cast<const uint2*>(U16 + i * M.un + j));
+        const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&h.x));
+        const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&h.y));
+        u[0] = a.x, u[1] = a.y, u[2] = b.x, u[3] = b.y;
+      } else {
+        const float4 b = __ldcs(reinterpret_cast<const float4*>(U32 + e));
+        u[0] = b.x, u[1] = b.y, u[2] = b.z, u[3] = b.w;
+      }
       float s0, s1, s2, s3;
       if (mode == 0) {
         s0 = s1 = s2 = s3 = sv[i];
@@ -630,18 +671,35 @@ __global__ void __launch_bounds__(kThreads) apply_kernel(const MatInfo* __restri
           s0 *= si, s1 *= si, s2 *= si, s3 *= si;
         }
       }
-      w.x = fmaf(decay, w.x, -step * (s0 * u.x));
-      w.y = fmaf(decay, w.y, -step * (s1 * u.y));
-      w.z = fmaf(decay, w.z, -step * (s2 * u.z));
-      w.w = fmaf(decay, w.w, -step * (s3 * u.w));
+      w.x = fmaf(decay, w.x, -step * (s0 * u[0]));
+      w.y = fmaf(decay, w.y, -step * (s1 * u[1]));
+      w.z = fmaf(decay, w.z, -step * (s2 * u[2]));
+      w.w = fmaf(decay, w.w, -step * (s3 * u[3]));
       *reinterpret_cast<float4*>(W + e) = w;
     }
   } else {
-    for (int64_t e = e0 + threadIdx.x; e < e1; e += kThreads) {
-      const int64_t i = e / M.n, j = e - i * M.n;
-      const float u = U[i * ustride + j];
-      const float s = mode == 0 ? sv[i] : (mode == 1 ? sv[j] : sv[i] * tv[j]);
-      W[e] = fmaf(decay, W[e], -step * (s * u));
+    // rows of any length: a warp reads and writes 32 consecutive elements
+    // of W (and of a row of U); each thread has four elements in flight
+    int64_t e = e0 + threadIdx.x;
+    int64_t i = e / M.n, j = e - i * M.n;
+    for (; e < e1; e += 4 * kThreads) {
+      float w[4], u[4], f[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int64_t ek = e + k * kThreads;
+        w[k] = u[k] = f[k] = 0.f;
+        if (ek < e1) {
+          w[k] = W[ek];
+          u[k] = hidden ? __half2float(__ushort_as_half(__ldcs(U16 + i * M.un + j))) : __ldcs(U32 + ek);
+          f[k] = mode == 0 ? sv[i] : (mode == 1 ? sv[j] : sv[i] * tv[j]);
+        }
+        for (j += kThreads; j >= M.n; j -= M.n) ++i;
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int64_t ek = e + k * kThreads;
+        if (ek < e1) W[ek] = fmaf(decay, w[k], -step * (f[k] * u[k]));
+      }
     }
   }
 }
@@ -669,8 +727,13 @@ cudaError_t launch_momentum_norm(const LaunchCtx& L, cudaStream_t st) {
 }
 
 cudaError_t launch_momentum_x0(const LaunchCtx& L, cudaStream_t st) {
-  return launch_pdl(momentum_x0_kernel, dim3((unsigned)L.total_tiles), dim3(kThreads), 0, st, 1, L.mats, L.nmat,
-                    L.groups, L.mom, L.grads, L.sc, L.partials, L.counters, L.ginv);
+  return launch_pdl(momentum_x0_kernel, dim3((unsigned)L.total_xblks), dim3(kThreads), 0, st, 1, L.mats, L.nmat,
+                    L.groups, L.mom, L.grads, L.sc, L.partials);
+}
+
+cudaError_t launch_x0norm(const LaunchCtx& L, cudaStream_t st) {
+  return launch_pdl(x0norm_kernel, dim3((unsigned)L.nmat), dim3(kThreads), 0, st, 1, L.mats, L.groups,
+                    static_cast<const float*>(L.partials), L.ginv);
 }
 
 cudaError_t launch_rows(const LaunchCtx& L, cudaStream_t st) {
@@ -698,7 +761,7 @@ cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st) {
 
 cudaError_t launch_apply(const LaunchCtx& L, cudaStream_t st) {
   return launch_pdl(apply_kernel, dim3((unsigned)L.total_chunks), dim3(kThreads), 0, st, 1, L.mats, L.nmat, L.params,
-                    static_cast<const float*>(L.uslab), static_cast<const float*>(L.mom),
+                    static_cast<const uint16_t*>(L.uslab), static_cast<const float*>(L.mom),
                     static_cast<const float*>(L.svec), static_cast<const float*>(L.tvec),
                     static_cast<const MatStats*>(L.stats), L.sc);
 }

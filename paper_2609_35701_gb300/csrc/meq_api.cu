@@ -19,6 +19,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <limits>
 #include <map>
 #include <tuple>
 #include <mutex>
@@ -42,7 +43,7 @@ struct Group {
   int64_t s = 0, l = 0, lp = 0, sp = 0, count = 0;
   int trans = 0;           // members are tall (W = X^T)
   int64_t m = 0, n = 0, un = 0;  // weight shape of every member, U row stride
-  int64_t u_base = 0;      // float offset of the group's U block [count][m][un]
+  int64_t u_base = 0;      // element offset of the group's fp16 U block [count][m][un]
   int64_t mbase = 0;       // first slot of the group in the per-matrix inverse-norm array
   int64_t rpart_base = 0;  // float offsets of the fused-statistics partials
   int64_t cpart_base = 0;
@@ -75,15 +76,15 @@ struct meq_state {
   int num_sms = 0;
   std::vector<MatInfo> mats;
   std::vector<Group> groups;
-  int64_t total_chunks = 0, total_hchunks = 0, total_tiles = 0, total_rblks = 0, total_slabs = 0;
-  int64_t mom_floats = 0, u_floats = 0, vec_floats = 0, parts_floats = 0;
+  int64_t total_chunks = 0, total_hchunks = 0, total_tiles = 0, total_rblks = 0, total_slabs = 0, total_xblks = 0;
+  int64_t mom_floats = 0, u_halves = 0, vec_floats = 0, parts_floats = 0;
   char* arena = nullptr;
   int64_t arena_bytes = 0;
   // device views
   MatInfo* d_mats = nullptr;
   GroupInfo* d_groups = nullptr;
   float* d_mom = nullptr;
-  float* d_u = nullptr;
+  uint16_t* d_u = nullptr;
   float* d_rvec = nullptr;
   float* d_cvec = nullptr;
   float* d_svec = nullptr;
@@ -115,6 +116,17 @@ struct meq_state {
 };
 
 namespace {
+
+// IEEE 754 binary16 -> binary32 (exact): sign, 5-bit exponent with bias 15,
+// 10-bit fraction; exponent 0 holds zero and the subnormals, 31 inf / NaN.
+float half_bits_to_float(uint16_t h) {
+  const float sign = (h & 0x8000u) ? -1.0f : 1.0f;
+  const int ex = (h >> 10) & 0x1f;
+  const int fr = h & 0x3ff;
+  if (ex == 0) return sign * std::ldexp(static_cast<float>(fr), -24);
+  if (ex == 31) return fr ? std::numeric_limits<float>::quiet_NaN() : sign * std::numeric_limits<float>::infinity();
+  return sign * std::ldexp(static_cast<float>(fr | 0x400), ex - 25);
+}
 
 meq_status fail(meq_state* st, meq_status s, const std::string& msg) {
   if (st) st->last_error = msg; else g_init_error = msg;
@@ -199,7 +211,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
       Group G;
       G.s = M.s, G.l = M.l;
       G.trans = M.trans;
-      G.m = m, G.n = c, G.un = round_up(c, 4);
+      G.m = m, G.n = c, G.un = round_up(c, 8);  // whole 16-byte chunks per fp16 row
       G.lp = round_up(M.l, 64), G.sp = round_up(M.s, 64);
       G.alpha0 = std::min(pow2_round(std::sqrt(static_cast<double>(M.s) * static_cast<double>(M.l))), 16384.f);
       G.alpha = std::min(pow2_round(std::sqrt(static_cast<double>(M.l))), 16384.f);
@@ -211,7 +223,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
     M.gidx = st->groups[g].count++;
     st->groups[g].mats.push_back(i);
   }
-  int64_t mom = 0, u = 0, vec = 0, parts = 0, chunks = 0, hchunks = 0, tiles = 0, rblks = 0, slabs = 0;
+  int64_t mom = 0, u = 0, vec = 0, parts = 0, chunks = 0, hchunks = 0, tiles = 0, rblks = 0, slabs = 0, xblks = 0;
   int64_t mslots = 0;
   for (auto& G : st->groups) {
     G.mbase = mslots;
@@ -235,6 +247,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
     chunks += (M.m * M.n + kChunk - 1) / kChunk;
     M.hchunk_begin = hchunks;
     M.tile_begin = tiles;
+    M.xblk_begin = xblks;
     M.rblk_begin = rblks;
     M.slab_begin = slabs;
     if (M.kind == KIND_HIDDEN) {
@@ -245,6 +258,9 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
       M.cpart_off = G.cpart_base + M.gidx * ((G.s + 31) / 32) * G.l;
       hchunks += (M.m * M.n + kChunk - 1) / kChunk;
       tiles += ((M.m + kCastTile - 1) / kCastTile) * ((M.n + kCastTile - 1) / kCastTile);
+      // momentum + X_0: flat chunks of W, or 64 x 64 tiles when X_0 is W transposed
+      xblks += M.trans ? ((M.m + kCastTile - 1) / kCastTile) * ((M.n + kCastTile - 1) / kCastTile)
+                       : (M.m * M.n + kChunk - 1) / kChunk;
     } else {
       M.un = M.n;
       rblks += (M.m + 7) / 8;  // 8 rows (warps) per block
@@ -256,17 +272,17 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
       }
     }
   }
-  st->mom_floats = mom, st->u_floats = u, st->vec_floats = vec, st->parts_floats = parts;
-  st->total_chunks = chunks, st->total_hchunks = hchunks, st->total_tiles = tiles;
+  st->mom_floats = mom, st->u_halves = u, st->vec_floats = vec, st->parts_floats = parts;
+  st->total_chunks = chunks, st->total_hchunks = hchunks, st->total_tiles = tiles, st->total_xblks = xblks;
   st->total_rblks = rblks, st->total_slabs = slabs;
   st->persistent_bytes = 0;
   for (int i = 0; i < n; ++i) st->persistent_bytes += 4 * st->mats[i].m * st->mats[i].n;
 
   *off_mom = L->add(mom * 4);
-  *off_u = L->add(u * 4);
+  *off_u = L->add(u * 2);
   *off_vec4 = L->add(vec * 4 * 4);  // r, c, s, t
   *off_cpart = L->add(parts * 4);
-  *off_partials = L->add(std::max(hchunks, tiles) * 4);  // per momentum chunk or fused tile
+  *off_partials = L->add(std::max({hchunks, tiles, xblks}) * 4);  // per momentum chunk or block
   *off_counters = L->add(int64_t(n) * 4);
   *off_x0s = L->add(int64_t(n) * 4 * 2);  // x0scale (cast pass) and the inverse norms (fused)
   *off_stats = L->add(int64_t(n) * sizeof(MatStats));
@@ -405,10 +421,10 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
               if (per_matrix) Q.minv = st->d_ginv + G.mbase, Q.minv_pow = 1;
               Q.out_fp16 = dX(k + 1);
             } else {
-              Q.out = st->d_u + G.u_base, Q.out_ld = G.un * 4, Q.out_mstride = G.m * G.un * 4;
+              Q.out = st->d_u + G.u_base, Q.out_ld = G.un * 2, Q.out_mstride = G.m * G.un * 2;
               Q.scale = 1.0f / ak;
               if (per_matrix) Q.minv = st->d_ginv + G.mbase, Q.minv_pow = 1;
-              Q.out_fp16 = 0;
+              Q.out_fp16 = 1;  // fp16(kUScale * U)
               Q.rpart = st->d_parts + G.rpart_base;
               Q.cpart = st->d_parts + G.cpart_base;
             }
@@ -557,7 +573,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   st->arena_bytes = L.total;
   char* A = st->arena;
   st->d_mom = reinterpret_cast<float*>(A + off_mom);
-  st->d_u = reinterpret_cast<float*>(A + off_u);
+  st->d_u = reinterpret_cast<uint16_t*>(A + off_u);
   st->d_rvec = reinterpret_cast<float*>(A + off_vec4);
   st->d_cvec = st->d_rvec + st->vec_floats;
   st->d_svec = st->d_cvec + st->vec_floats;
@@ -628,9 +644,11 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   C.total_chunks = st->total_chunks;
   C.total_hchunks = st->total_hchunks;
   C.total_tiles = st->total_tiles;
+  C.total_xblks = st->total_xblks;
+  C.n_hidden = st->n_hidden;
   C.total_rblks = st->total_rblks;
   C.total_slabs = st->total_slabs;
-  st->kernels_per_step = (st->n_hidden ? (o.ns_x0_fused ? 1 : 2) : 0) + (st->n_rows ? 1 : 0) + (st->n_two ? 1 : 0) + 2 +
+  st->kernels_per_step = (st->n_hidden ? 2 : 0) + (st->n_rows ? 1 : 0) + (st->n_two ? 1 : 0) + 2 +
                          static_cast<int>(st->gemm.size());
   st->step_host.assign(static_cast<size_t>(st->step_bytes), 0);
   st->last_stream = s;
@@ -654,6 +672,10 @@ static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev
   if (st->n_hidden) {
     e = fused ? launch_momentum_x0(C, s) : launch_momentum_norm(C, s);
     if (e != cudaSuccess) return cuda_fail(st, e, "momentum launch");
+    if (fused) {
+      e = launch_x0norm(C, s);
+      if (e != cudaSuccess) return cuda_fail(st, e, "x0norm launch");
+    }
   }
   if (st->n_rows) {
     e = launch_rows(C, s);
@@ -822,9 +844,14 @@ meq_status meq_read_ns_output(meq_state* st, int i, float* dst) {
   if (!dst) return fail(st, MEQ_ERR_INVALID_ARG, "dst is NULL");
   if (st->kinds[i] != KIND_HIDDEN) return fail(st, MEQ_ERR_INVALID_ARG, "entry has no Newton-Schulz output (not hidden)");
   const MatInfo& M = st->mats[i];
-  cudaError_t e = cudaMemcpy2D(dst, M.n * sizeof(float), st->d_u + M.u_off, M.un * sizeof(float), M.n * sizeof(float),
-                               M.m, cudaMemcpyDefault);
-  return e == cudaSuccess ? MEQ_OK : cuda_fail(st, e, "cudaMemcpy2D");
+  std::vector<uint16_t> h(static_cast<size_t>(M.m * M.n));
+  cudaError_t e = cudaMemcpy2D(h.data(), M.n * sizeof(uint16_t), st->d_u + M.u_off, M.un * sizeof(uint16_t),
+                               M.n * sizeof(uint16_t), M.m, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(st, e, "cudaMemcpy2D");
+  std::vector<float> f(h.size());
+  for (size_t k = 0; k < h.size(); ++k) f[k] = half_bits_to_float(h[k]) * (1.0f / kUScale);
+  e = cudaMemcpy(dst, f.data(), f.size() * sizeof(float), cudaMemcpyDefault);
+  return e == cudaSuccess ? MEQ_OK : cuda_fail(st, e, "cudaMemcpy");
 }
 
 meq_status meq_read_stats(meq_state* st, int i, float* r, float* c, double* gamma_r, double* gamma_c, int* direction) {

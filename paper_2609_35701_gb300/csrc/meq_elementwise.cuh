@@ -30,20 +30,22 @@ struct LaunchCtx {
   unsigned int* counters;
   float* x0scale;
   float* ginv;           // 1 / ||H||_F per hidden matrix, ordered group by group
-  float* uslab;
+  uint16_t* uslab;       // U of every hidden matrix, fp16, scaled by kUScale
   float* parts;          // NS-row and NS-column partial sums of squares
   float* rvec;
   float* cvec;
   float* svec;           // hidden: scale of the chosen side; others: 1 / row RMS
   float* tvec;           // remaining 2D: 1 / column RMS of the row-normalised momentum
   MatStats* stats;
-  int64_t total_chunks, total_hchunks, total_tiles, total_rblks, total_slabs;
+  int64_t total_chunks, total_hchunks, total_tiles, total_rblks, total_slabs, total_xblks;
+  int n_hidden;
 };
 
 constexpr int KIND_HIDDEN = 0, KIND_TWO_SIDED = 1, KIND_VECTOR = 2;
 
 cudaError_t launch_momentum_norm(const LaunchCtx& L, cudaStream_t st);
 cudaError_t launch_momentum_x0(const LaunchCtx& L, cudaStream_t st);  // fused momentum + bf16 X_0
+cudaError_t launch_x0norm(const LaunchCtx& L, cudaStream_t st);       // 1 / ||H||_F from its partials
 cudaError_t launch_rows(const LaunchCtx& L, cudaStream_t st);      // remaining 2D + vectors
 cudaError_t launch_colpart(const LaunchCtx& L, cudaStream_t st);   // remaining 2D
 cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st);

@@ -25,6 +25,12 @@ enum DevErr : int {
 
 constexpr int kMaxGroups = 8;        // shape groups per GEMM launch
 
+// U of the hidden weights is stored as fp16(kUScale * U). Every entry of U
+// is bounded by its largest singular value, which the quintic keeps below
+// about 1.25, so the scaled values stay far from fp16's overflow while
+// entries down to 4e-9 keep fp16's full 11-bit precision.
+constexpr float kUScale = 16384.0f;
+
 // Per-matrix metadata (device copy built at init).
 struct MatInfo {
   int64_t m, n;          // W layout: rows, cols
@@ -35,14 +41,15 @@ struct MatInfo {
   int32_t pad_;
   int64_t gidx;          // index inside its group
   int64_t mom_off;       // float offset of B in the momentum slab
-  int64_t u_off;         // float offset of U in the U slab (row stride un)
-  int64_t un;            // U row stride (cols rounded up to 4)
+  int64_t u_off;         // element offset of U in the fp16 U slab (row stride un)
+  int64_t un;            // U row stride: cols rounded up to 8 (hidden), cols (others)
   int64_t vec_off;       // float offset of r (m), c (n) and scale (max(m, n))
   int64_t chunk_begin;   // first apply chunk (all kinds)
   int64_t hchunk_begin;  // first momentum-and-norm chunk (hidden weights only)
   int64_t rblk_begin;    // first 8-row block of the row pass (remaining 2D and vectors)
   int64_t slab_begin;    // first row slab of the column pass (remaining 2D only)
   int64_t tile_begin;    // first cast tile (hidden weights only)
+  int64_t xblk_begin;    // first momentum-and-X_0 block (hidden weights only)
   int64_t rpart_off;     // float offset of NS-row partial sums of squares [2 * ceil(l/256)][s]
   int64_t cpart_off;     // float offset of column partial sums of squares: NS columns
                          // [ceil(s/32)][l] (hidden) or normalised columns [slabs][n] (remaining 2D)

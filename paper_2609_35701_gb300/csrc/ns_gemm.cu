@@ -8,9 +8,9 @@
 //               a I + b A is added in fp32 from the same 16-bit A the
 //               product uses, so P is exactly a polynomial of that matrix
 //   MODE_XUPD : X'  = P X * (alpha'/alpha)      (s x l, contraction over s)
-//   MODE_XLAST: U   = P X / alpha, written as fp32 in the weight's own layout,
-//               with the sums of squares of U's rows and columns (Eq. (7))
-//               reduced in the epilogue into per-tile partials
+//   MODE_XLAST: U   = P X / alpha, written as fp16(2^14 U) in the weight's own
+//               layout, with the sums of squares of the stored U's rows and
+//               columns (Eq. (7)) reduced into per-tile partials
 //
 // P X equals a X + (b A + c A^2) X of Eq. (5) exactly in real arithmetic.
 // A and P are symmetric: their launches run only the tiles that hold a 32 x 32
@@ -20,7 +20,8 @@
 // normal range of fp16; the epilogues undo the scale in fp32.
 //
 // Roles (320 threads, one CTA per SM):
-//   warp 0 : TMA producer (one thread), 4-stage shared-memory ring
+//   warp 0 : TMA producer (one thread), shared-memory ring of 4 stages
+//            (single CTA) or 6 (CTA pair)
 //   warp 1 : TMEM allocator and tcgen05.mma issuer (one thread)
 //   warps 2-9 : epilogue; warp w reads TMEM lanes 32*(w%4) .. +31 and takes
 //               every other 32-column chunk (two warps per lane quarter, so
@@ -45,7 +46,8 @@ constexpr int A_BYTES = BM * BK * 2;                 // 16 KB
 constexpr int NUM_EPI_WARPS = 8;                     // two per TMEM lane quarter
 constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
 constexpr uint32_t TMEM_COLS = 512;
-constexpr int SLOT_BYTES = 2048;                     // one 32 x 32 16-bit block (or 32 x 16 fp32)
+constexpr int SLOT_BYTES = 2048;                     // one 32 x 32 16-bit block
+constexpr float kUInvScale2 = 1.0f / (kUScale * kUScale);  // exact: kUScale is a power of two
 
 // kPair = 1: one CTA computes a 128 x 256 tile (tcgen05 cta_group::1).
 // kPair = 2: a cluster of two CTAs computes a 256 x 256 tile with
@@ -327,21 +329,7 @@ __device__ __forceinline__ void fill_half_cols(uint8_t* slot, int r, const float
     *reinterpret_cast<uint16_t*>(slot + off) = to_half_bits(v[j], fp16);
   }
 }
-// fp32 16-column half of a row, 64-byte rows, 64B swizzle.
-__device__ __forceinline__ void fill_f32_rows16(uint8_t* slot, int r, const float* v) {
-#pragma unroll
-  for (int k = 0; k < 4; ++k)
-    *reinterpret_cast<float4*>(slot + r * 64 + ((k ^ ((r >> 1) & 3)) << 4)) =
-        make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
-}
-// fp32 transposed: 16 rows (j) x 32 columns (r), 128-byte rows, 128B swizzle.
-__device__ __forceinline__ void fill_f32_cols16(uint8_t* slot, int r, const float* v) {
-#pragma unroll
-  for (int j = 0; j < 16; ++j)
-    *reinterpret_cast<float*>(slot + j * 128 + ((((r >> 2) ^ (j & 7))) << 4) + ((r & 3) << 2)) = v[j];
-}
-
-// 32 rows x 64 bytes (16-bit 32 x 32, or fp32 32 x 16) -> global: rows
+// 32 rows x 64 bytes (a 16-bit 32 x 32 block) -> global: rows
 // r < rows_valid, 16-byte chunks k < chunks_valid of each row.
 __device__ __forceinline__ void store_block64(const uint8_t* slot, int lane, uint8_t* dst, int64_t ld_bytes,
                                               int rows_valid, int chunks_valid) {
@@ -353,19 +341,6 @@ __device__ __forceinline__ void store_block64(const uint8_t* slot, int lane, uin
     if (r < rows_valid && k < chunks_valid) *reinterpret_cast<uint4*>(dst + r * ld_bytes + k * 16) = w;
   }
 }
-// 16 rows x 128 bytes (fp32 16 x 32, 128B swizzle) -> global: rows
-// r < rows_valid, 16-byte chunks k < chunks_valid of each row.
-__device__ __forceinline__ void store_block128(const uint8_t* slot, int lane, uint8_t* dst, int64_t ld_bytes,
-                                               int rows_valid, int chunks_valid) {
-  const int k = lane & 7;
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int r = (lane >> 3) + 4 * i;
-    const uint4 w = *reinterpret_cast<const uint4*>(slot + r * 128 + ((k ^ (r & 7)) << 4));
-    if (r < rows_valid && k < chunks_valid) *reinterpret_cast<uint4*>(dst + r * ld_bytes + k * 16) = w;
-  }
-}
-
 template <int kPair>
 __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_constant__ GemmParams p) {
   using C_ = Cfg<kPair>;
@@ -623,6 +598,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
           for (int j = 0; j < 32; ++j) v[j] *= sc;
         }
         if (mode == MODE_XLAST) {
+          // U is stored as fp16(kUScale U). The sums of squares are taken from
+          // those stored values (v holds them exactly) and scaled back by
+          // kUScale^-2 (a power of two) when written, so the statistics
+          // describe the U the update applies.
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = __half2float(__float2half_rn(v[j] * kUScale));
           // Column sums of squares over the warp's 32 rows: transpose-reduce
           // so that lane j ends with the sum for column col0 + j.
           float sq[32];
@@ -642,26 +623,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
             }
           }
           if (col0 + lane < G.N)
-            G.cpart[(static_cast<int64_t>(c.mat) * ((G.M + 31) / 32) + R) * G.N + col0 + lane] = sq[0];
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            if (!G.trans) {
-              // U rows = NS rows; 16 columns col0 + 16h .. of 4-float chunks
-              fill_f32_rows16(slot, lane, v + 16 * h);
-              __syncwarp();
-              // 4-float chunks starting below N stay inside the padded row (stride = N rounded up to 4)
-              if (col0 + 16 * h < G.N)
-                store_block64(slot, lane, outm + static_cast<int64_t>(row0) * G.out_ld + (col0 + 16 * h) * 4, G.out_ld,
-                              rows_valid, (G.N - (col0 + 16 * h) + 3) / 4);
-            } else {
-              // U rows = NS columns col0 + 16h + j, U columns = NS rows row0 + r
-              fill_f32_cols16(slot, lane, v + 16 * h);
-              __syncwarp();
-              if (col0 + 16 * h < G.N)
-                store_block128(slot, lane, outm + static_cast<int64_t>(col0 + 16 * h) * G.out_ld + row0 * 4, G.out_ld,
-                               min(16, G.N - (col0 + 16 * h)), (rows_valid + 3) / 4);
-            }
+            G.cpart[(static_cast<int64_t>(c.mat) * ((G.M + 31) / 32) + R) * G.N + col0 + lane] = sq[0] * kUInvScale2;
+          // 8-element chunks that start below the row length stay inside the
+          // padded row (stride = row length rounded up to 8)
+          if (!G.trans) {
+            // U rows = NS rows row0 + r, U columns = NS columns col0 + j
+            fill_half_rows(slot, lane, v, 1);
             __syncwarp();
+            store_block64(slot, lane, outm + static_cast<int64_t>(row0) * G.out_ld + col0 * 2, G.out_ld, rows_valid,
+                          min(4, (G.N - col0 + 7) / 8));
+          } else {
+            // U rows = NS columns col0 + j, U columns = NS rows row0 + r
+            fill_half_cols(slot, lane, v, 1);
+            __syncwarp();
+            store_block64(slot, lane, outm + static_cast<int64_t>(col0) * G.out_ld + row0 * 2, G.out_ld,
+                          min(32, G.N - col0), min(4, (G.M - row0 + 7) / 8));
           }
         } else {
           // 16-bit rows are padded to a multiple of 64 elements: whole 32-column blocks stay inside them
@@ -679,7 +655,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
         __syncwarp();  // slots free again; reconverge before the next warp-wide tcgen05.ld
       }
       if (mode == MODE_XLAST && row0 < G.M && row0 + lane < G.M)  // one partial per (tile column, half)
-        G.rpart[(static_cast<int64_t>(c.mat) * G.tiles_n * 2 + c.tn * 2 + half) * G.M + row0 + lane] = rsum;
+        G.rpart[(static_cast<int64_t>(c.mat) * G.tiles_n * 2 + c.tn * 2 + half) * G.M + row0 + lane] = rsum * kUInvScale2;
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
