@@ -13,6 +13,9 @@ Gram shortcut): each function is the equation it cites, written out.
 
 Equation numbers are the paper's:
   Eq. (5)  quintic Newton-Schulz iteration           (Section 2, "Muon")
+  Eq. (6)  Muon with decoupled weight decay and RMS
+           alignment (the Moonlight form), the baseline
+           MeqMuon is compared with                   (Section 2, "Muon")
   Eq. (7)  row / column RMS vectors                  (Section 3.1)
   Eq. (8)  coefficients of variation, delta rule     (Section 3.1)
   Eq. (9)  row / column normalisation operators      (Section 3.2)
@@ -217,6 +220,23 @@ def param_step(kind, W, G, B_prev, lr, mu, weight_decay, eps=DELTA, rho=RHO, **k
     else:
         raise ValueError(kind)
     return apply_update(W, Ut, lr, weight_decay, rho), B, Ut
+
+
+def moonlight_update(W, U, lr, weight_decay, rho=RHO):
+    """Eq. (6): W_{t+1} = (1 - eta_t lambda) W_t - eta_t rho sqrt(max(m, n)) U_t.
+    sqrt(max(m, n)) compensates the update RMS for the matrix shape."""
+    m, n = np.shape(U)
+    return (1.0 - lr * weight_decay) * _f64(W) - lr * rho * np.sqrt(max(m, n)) * _f64(U)
+
+
+def moonlight_step(W, G, B_prev, lr, mu, weight_decay, rho=RHO, steps=NS_STEPS, coeffs=NS_COEFFS,
+                   nesterov=False):
+    """Eq. (6) for one 2D weight in a hidden layer: Eq. (10) momentum, Orth
+    approximated by the K iterations of Eq. (5), then the shape-compensated
+    update, with no equilibration. Returns (W_next, B_t, U_t)."""
+    B = momentum_update(B_prev, G, mu)
+    U = newton_schulz(ns_input(B, G, mu, nesterov), steps, coeffs)
+    return moonlight_update(W, U, lr, weight_decay, rho), B, U
 
 
 def hidden_step_all(Ws, Gs, Bs_prev, lr, mu, weight_decay, **kw):

@@ -14,7 +14,10 @@ the oracle disagrees with a value fixed by the paper or by mathematics:
   * invariants: unit-RMS rows / columns after Eq. (9), idempotence, scale
     and sign invariance, transpose equivariance, zero rows and columns,
     and the orthogonality constraint of Section 3.1 on exact Orth;
-  * paper tables: Table 5 state memory from Table 8 architectures.
+  * paper tables: Table 5 state memory from Table 8 architectures;
+  * the Muon baseline of Eq. (6): the shape factor sqrt(max(m, n)) gives an
+    exactly orthogonal update unit RMS; closed forms on the Hadamard and
+    known-SVD inputs.
 
 tests/test_oracle_mutations.py plants plausible mistakes in a copy of the
 oracle and asserts that at least one of these checks fails for each.
@@ -398,6 +401,57 @@ def check_hidden_step_composition(O):
     assert np.abs(W1 - ((1 - 0.002) * W0 - 0.2 * 0.02 * H)).max() < 1e-14
 
 
+def check_moonlight_update(O):
+    """Eq. (6): sqrt(max(m, n)) makes the update RMS independent of the shape.
+    For U with orthonormal rows (m <= n) or columns (m > n), ||U||_F^2 =
+    min(m, n), so the applied update (W_{t+1} - (1 - eta lambda) W_t) /
+    (eta rho) has RMS exactly 1; decay is decoupled."""
+    rng = np.random.default_rng(31)
+    lr, wd, rho = 0.02, 0.1, 0.2
+    for m, n in [(12, 30), (30, 12), (16, 16), (1, 9), (9, 1)]:
+        U = _orthonormal(rng, max(m, n), min(m, n))
+        U = U.T if m < n else U
+        assert U.shape == (m, n)
+        W0 = rng.standard_normal((m, n))
+        V = (O.moonlight_update(W0, U, lr, wd, rho) - (1 - lr * wd) * W0) / (-lr * rho)
+        assert abs(np.sqrt((V * V).mean()) - 1.0) < 1e-12, (m, n)
+        assert np.abs(V - np.sqrt(max(m, n)) * U).max() < 1e-12
+    # no update and no decay: identity
+    W0 = rng.standard_normal((4, 5))
+    assert np.abs(O.moonlight_update(W0, np.zeros((4, 5)), lr, 0.0, rho) - W0).max() == 0.0
+
+
+def check_moonlight_step(O):
+    """Eq. (6) composed with Eqs. (10) and (5), from B_{-1} = 0.
+    Hadamard gradient: U = f(1/sqrt 8) H_8 / sqrt 8, so the update is
+    -eta rho f(1/sqrt 8) H_8 (MeqMuon's would be -eta rho H_8: the factor f is
+    what equilibration removes). Known SVD, rectangular: U = P f(s/||s||) Q^T
+    and the update is -eta rho sqrt(max(m, n)) U."""
+    lr, mu, wd, rho = 0.02, 0.95, 0.1, 0.2
+    H = _sylvester_hadamard(8)
+    W0 = np.arange(64, dtype=np.float64).reshape(8, 8) / 100.0
+    W1, B, U = O.moonlight_step(W0, H, np.zeros((8, 8)), lr, mu, wd, rho)
+    f = f_scalar(1.0 / math.sqrt(8.0))
+    assert np.abs(B - H).max() == 0.0
+    assert np.abs(W1 - ((1 - lr * wd) * W0 - lr * rho * f * H)).max() < 1e-13
+    rng = np.random.default_rng(77)
+    for m, n in [(10, 26), (26, 10)]:
+        r = min(m, n)
+        P = _orthonormal(rng, m, r)
+        Q = _orthonormal(rng, n, r)
+        sv = np.exp(rng.uniform(np.log(0.1), np.log(2.0), r))
+        G = P @ np.diag(sv) @ Q.T
+        Uk = P @ np.diag([f_scalar(v / np.linalg.norm(sv)) for v in sv]) @ Q.T
+        W1, _, _ = O.moonlight_step(np.zeros((m, n)), G, np.zeros((m, n)), lr, mu, wd, rho)
+        assert np.abs(W1 + lr * rho * np.sqrt(max(m, n)) * Uk).max() < 1e-12, (m, n)
+    # Nesterov: the NS input is G_t + mu B_t
+    Bp = rng.standard_normal((6, 9))
+    G = rng.standard_normal((6, 9))
+    _, _, U = O.moonlight_step(np.zeros((6, 9)), G, Bp, lr, mu, wd, rho, nesterov=True)
+    Bt = mu * Bp + G
+    assert np.abs(U - O.newton_schulz(G + mu * Bt)).max() < 1e-13
+
+
 # ------------------------------------------------------------ paper tables
 def llama_hidden_counts(a):
     q = a["q_heads"] * a["head_dim"]
@@ -433,4 +487,5 @@ ALL_CHECKS = [
     check_cv_hand_values, check_selection_rule, check_equilibration_invariants,
     check_orthogonality_constraint, check_two_sided_and_vector, check_momentum_closed_form,
     check_apply_closed_form, check_hidden_step_composition, check_param_step_branches,
+    check_moonlight_update, check_moonlight_step,
 ]

@@ -102,6 +102,12 @@ MUTATIONS = {
     "nesterov_wrong": ("ns_input", lambda B, G, mu, nesterov=False: np.asarray(B) + (mu * np.asarray(G) if nesterov else 0)),
     "two_sided_order_swapped": ("two_sided_normalize", lambda B, delta=1e-7: _col_then_row(B)),
     "vector_uses_l2": ("vector_normalize", lambda b, delta=1e-7: np.asarray(b) / np.linalg.norm(b)),
+    "moonlight_sqrt_min": ("moonlight_update", lambda W, U, lr, wd, rho=0.2: (1 - lr * wd) * np.asarray(W)
+                           - lr * rho * np.sqrt(min(np.shape(U))) * np.asarray(U)),
+    "moonlight_no_shape_factor": ("moonlight_update", lambda W, U, lr, wd, rho=0.2: (1 - lr * wd) * np.asarray(W)
+                                  - lr * rho * np.asarray(U)),
+    "moonlight_coupled_decay": ("moonlight_update", lambda W, U, lr, wd, rho=0.2: (1 - wd) * np.asarray(W)
+                                - lr * rho * np.sqrt(max(np.shape(U))) * np.asarray(U)),
 }
 
 
