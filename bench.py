@@ -139,7 +139,7 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def oracle_sample(wl, seed_step=0, max_per_class=1):
+def oracle_sample(wl, seed_step=0, max_per_class=1, rule="meqmuon"):
     """Times the fp64 oracle on one matrix of every (rows, cols) class of the
     workload and extrapolates to the whole model step (ms)."""
     import numpy as np
@@ -160,7 +160,10 @@ def oracle_sample(wl, seed_step=0, max_per_class=1):
         W0 = np.zeros((r, c))
         Bp = np.zeros((r, c))
         t0 = time.perf_counter()
-        O.param_step(k, W0, G, Bp, LR, MU, WD, eps=EPS)
+        if rule == "muon":
+            O.moonlight_step(W0, G, Bp, LR, MU, WD)
+        else:
+            O.param_step(k, W0, G, Bp, LR, MU, WD, eps=EPS)
         dt = (time.perf_counter() - t0) * 1e3
         total_ms += dt * len(idx)
         sampled.append(f"{r}x{c}" + ("" if k == 0 else ("/2-sided" if k == 1 else "/vector")))
@@ -187,11 +190,11 @@ def run_reference(args):
 
     wl = W.get_workload(args.workload)
     for w in range(args.warmup):
-        oracle_sample(wl, w)
+        oracle_sample(wl, w, rule=args.update_rule)
     vals = []
     sampled = None
     for k in range(args.steps):
-        ms, sampled = oracle_sample(wl, k)
+        ms, sampled = oracle_sample(wl, k, rule=args.update_rule)
         vals.append(ms)
     v = statistics.median(vals)
     cores = cpu_cores()
@@ -201,7 +204,8 @@ def run_reference(args):
         "impl": "reference", "metric": "MeqMuon optimizer step time (all hidden 2D weights)", "value": v,
         "unit": "ms/step", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": v, "higher_is_better": False, "scaling": "strong", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": args.workload, "matrices": len(wl.shapes), "elements": wl.numel},
+        "data": "synthetic", "config": {"workload": args.workload, "matrices": len(wl.shapes), "elements": wl.numel,
+                                        "update_rule": "Eq. (11) + Eq. (14)" if args.update_rule == "meqmuon" else "Eq. (6)"},
         "cpu_baseline": {"value": v, "unit": "ms/step", "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": v, "unit": "ms/step", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -218,6 +222,8 @@ def main():
     ap.add_argument("--ns-fp16-mask", type=lambda x: int(x, 0), default=0xFFFFFFFF)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--update-rule", default="meqmuon", choices=["meqmuon", "muon"],
+                    help="meqmuon: Eq. (11) + Eq. (14); muon: the Eq. (6) comparison baseline (hidden weights only)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.impl == "reference":
@@ -274,7 +280,8 @@ def main():
     params = [v.view(r, c) for v, (r, c) in zip(pviews, shapes)]
     grads = [[v.view(r, c) for v, (r, c) in zip(gv, shapes)] for _, gv in gbufs]
 
-    opt = meq.MeqMuon(shapes, kinds=kinds, ns_fp16_mask=args.ns_fp16_mask)
+    rule = meq.RULE_MUON if args.update_rule == "muon" else meq.RULE_MEQMUON
+    opt = meq.MeqMuon(shapes, kinds=kinds, ns_fp16_mask=args.ns_fp16_mask, update_rule=rule)
     stream = torch.cuda.current_stream()
     for k in range(args.warmup):
         opt.step(params, grads[k % 2], LR, MU, WD, EPS)
@@ -390,7 +397,7 @@ def main():
         vals, sampled = [], None
         t_start = time.perf_counter()
         while True:
-            v, sampled = oracle_sample(wl, len(vals))
+            v, sampled = oracle_sample(wl, len(vals), rule=args.update_rule)
             vals.append(v)
             if time.perf_counter() - t_start > 10.0 or len(vals) >= 5:
                 break
@@ -408,7 +415,8 @@ def main():
             "config": {"workload": args.workload, "matrices": len(wl.shapes), "elements": wl.numel,
                        "ns_steps": K, "ns_operands": "fp16" if args.ns_fp16_mask == 0xFFFFFFFF else hex(args.ns_fp16_mask),
                        "accumulate": "fp32", "l2": "inputs larger than L2 (params+grads+momentum %.2f GB)" % (12 * wl.numel / 1e9),
-                       "parallelism": f"matrices split over {world} GPU(s)" if world > 1 else "single GPU"},
+                       "parallelism": f"matrices split over {world} GPU(s)" if world > 1 else "single GPU",
+                       "update_rule": "Eq. (11) + Eq. (14)" if args.update_rule == "meqmuon" else "Eq. (6)"},
             "roofline": {
                 "bound": "tensor", "kernel": "ns_gemm_kernel",
                 "achieved": ns_tflops, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",

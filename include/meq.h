@@ -72,7 +72,18 @@ typedef struct {
                              bf16, and the first NS products apply 1/||B||_F; iteration 0
                              then runs its X and P operands in bf16. 0: a separate pass
                              writes the normalised X_0 in the format ns_fp16_mask gives it. */
+  int update_rule;        /* meq_update_rule; default MEQ_RULE_MEQMUON */
 } meq_options;
+
+/* Update applied to the hidden 2D weights after momentum and Newton-Schulz. */
+typedef enum {
+  MEQ_RULE_MEQMUON = 0, /* Eq. (11) equilibration, then Eq. (14) (Algorithm 1) */
+  MEQ_RULE_MUON = 1     /* Muon with decoupled weight decay and RMS alignment, Eq. (6)
+                           (the comparison baseline of Section 4): W <- (1 - lr wd) W
+                           - lr rho sqrt(max(m, n)) U, no equilibration. Every entry must
+                           be MEQ_KIND_HIDDEN (that baseline updates the others with
+                           AdamW, which this library does not provide). */
+} meq_update_rule;
 
 /* Parameter type, selecting the branch of Algorithm 1 applied to it. */
 typedef enum {
@@ -150,12 +161,20 @@ meq_status meq_write_momentum(meq_state* st, int i, const float* src);
 meq_status meq_read_ns_output(meq_state* st, int i, float* dst);
 /* Last step's statistics of entry i. Hidden weight: r (rows floats), c (cols
  * floats) of Eq. (7) for U, gamma_r, gamma_c of Eq. (8) and the direction of
- * Eq. (11) (0 = row, 1 = column). Remaining 2D parameter: r = row RMS of
- * B_t, c = column RMS of N_r(B_t), their CVs, direction 2. Vector: r[0] =
- * RMS of B_t, gammas 0, direction 3. Any output may be NULL; r and c are
- * host or device memory. */
+ * Eq. (11) (0 = row, 1 = column; 4 under MEQ_RULE_MUON, whose update is
+ * the uniform sqrt(max(m, n)) U of Eq. (6) while r, c and the CVs still
+ * describe U). Remaining 2D parameter: r = row RMS of B_t, c = column RMS
+ * of N_r(B_t), their CVs, direction 2. Vector: r[0] = RMS of B_t, gammas 0,
+ * direction 3. Any output may be NULL; r and c are host or device memory. */
 meq_status meq_read_stats(meq_state* st, int i, float* r, float* c,
                           double* gamma_r, double* gamma_c, int* direction);
+/* How often Eq. (11) chose row-wise (*rows) and column-wise (*cols)
+ * normalisation for hidden weight i since the state was created or the
+ * counts were last reset (both 0 for other entries and under MEQ_RULE_MUON).
+ * The counts are kept on the device by the statistics kernel. */
+meq_status meq_read_direction_counts(meq_state* st, int i, int64_t* rows, int64_t* cols);
+/* Zero every entry's direction counts (enqueued on the state's stream). */
+meq_status meq_reset_direction_counts(meq_state* st);
 /* Number of kernels one meq_step launches (for launch accounting), and how
  * many of them are Newton-Schulz GEMM launches. */
 int meq_kernels_per_step(const meq_state* st);

@@ -525,7 +525,8 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
                                                                const float* __restrict__ parts,
                                                                float* __restrict__ rvec, float* __restrict__ cvec,
                                                                float* __restrict__ svec, float* __restrict__ tvec,
-                                                               MatStats* __restrict__ stats) {
+                                                               MatStats* __restrict__ stats,
+                                                               unsigned long long* __restrict__ dircount) {
   pdl_allow_dependents();
   pdl_wait_predecessor();
   __shared__ float shf[32];
@@ -601,23 +602,33 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
   // fp32 with fixed-order block reductions.
   const float gam0 = block_cv(r, M.m, delta, shf);
   const float gam1 = block_cv(c, M.n, delta, shf);
-  const int dir = gam0 >= gam1 - sc->tie_atol ? 0 : 1;
-  const float* v = dir == 0 ? r : c;
-  const int64_t len = dir == 0 ? M.m : M.n;
-  for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
-    const float x = v[i];
-    s[i] = x > delta ? 1.0f / x : 0.0f;   // RMS at or below delta: treated as zero
+  int dir;
+  if (sc->rule == 1) {
+    // Eq. (6): every row scaled by sqrt(max(m, n)), no equilibration
+    dir = 4;
+    const float f = sqrtf(static_cast<float>(max(M.m, M.n)));
+    for (int64_t i = threadIdx.x; i < M.m; i += blockDim.x) s[i] = f;
+  } else {
+    dir = gam0 >= gam1 - sc->tie_atol ? 0 : 1;
+    const float* v = dir == 0 ? r : c;
+    const int64_t len = dir == 0 ? M.m : M.n;
+    for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
+      const float x = v[i];
+      s[i] = x > delta ? 1.0f / x : 0.0f;   // RMS at or below delta: treated as zero
+    }
   }
   if (threadIdx.x == 0) {
     stats[blockIdx.x].gamma_r = static_cast<double>(gam0);
     stats[blockIdx.x].gamma_c = static_cast<double>(gam1);
     stats[blockIdx.x].direction = dir;
+    if (dir < 2) dircount[2 * blockIdx.x + dir] += 1ull;  // one block per entry: no other writer
   }
 }
 
 // ----------------------------------------------------------------------- apply
 // W <- (1 - lr wd) W - rho lr U~ (Eq. (14)), U~ = scaled U (hidden) or scaled
-// B (remaining 2D: s_i t_j B_ij; vector: s_0 B_j).
+// B (remaining 2D: s_i t_j B_ij; vector: s_0 B_j). Under the Muon rule the
+// hidden scale is sqrt(max(m, n)) for every row (Eq. (6)).
 __global__ void __launch_bounds__(kThreads, 8) apply_kernel(const MatInfo* __restrict__ mats, int nmat,
                                                          float* const* __restrict__ params,
                                                          const uint16_t* __restrict__ uslab,
@@ -638,8 +649,10 @@ __global__ void __launch_bounds__(kThreads, 8) apply_kernel(const MatInfo* __res
   const bool hidden = M.kind == KIND_HIDDEN;
   // hidden: U is fp16(kUScale U) with row stride un; others: the momentum, fp32, contiguous
   const float step = sc->rho * sc->lr * (hidden ? 1.0f / kUScale : 1.0f);
-  // mode 0: per-row scale; 1: per-column scale; 2: row scale x column scale
-  const int mode = hidden ? stats[mi].direction : (M.kind == KIND_TWO_SIDED ? 2 : 0);
+  // mode 0: per-row scale (also the uniform scale of Eq. (6), held per row);
+  // 1: per-column scale; 2: row scale x column scale
+  const int dir = hidden ? stats[mi].direction : (M.kind == KIND_TWO_SIDED ? 2 : 0);
+  const int mode = dir == 4 ? 0 : dir;
   const float* sv = svec + M.vec_off;
   const float* tv = tvec + M.vec_off;
   const uint16_t* U16 = uslab + M.u_off;
@@ -756,7 +769,7 @@ cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st) {
 
 cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st) {
   return launch_pdl(finalize_kernel, dim3(L.nmat), dim3(kFinThreads), 0, st, 1, L.mats, L.sc,
-                    static_cast<const float*>(L.parts), L.rvec, L.cvec, L.svec, L.tvec, L.stats);
+                    static_cast<const float*>(L.parts), L.rvec, L.cvec, L.svec, L.tvec, L.stats, L.dircount);
 }
 
 cudaError_t launch_apply(const LaunchCtx& L, cudaStream_t st) {

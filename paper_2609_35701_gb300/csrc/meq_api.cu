@@ -95,6 +95,7 @@ struct meq_state {
   float* d_x0scale = nullptr;
   float* d_ginv = nullptr;
   MatStats* d_stats = nullptr;
+  unsigned long long* d_dircount = nullptr;  // [n][2]: row / column choices of Eq. (11)
   char* d_step = nullptr;  // StepScalars, params[n], grads[n]
   int* d_err = nullptr;
   int* d_flag = nullptr;
@@ -146,12 +147,20 @@ bool valid_options(const meq_options& o, std::string* why) {
   if (o.workspace_limit_bytes < 0) { *why = "workspace_limit_bytes must be >= 0"; return false; }
   if (o.ns_cta_pair != 0 && o.ns_cta_pair != 1) { *why = "ns_cta_pair must be 0 or 1"; return false; }
   if (o.ns_x0_fused != 0 && o.ns_x0_fused != 1) { *why = "ns_x0_fused must be 0 or 1"; return false; }
+  if (o.update_rule != MEQ_RULE_MEQMUON && o.update_rule != MEQ_RULE_MUON) {
+    *why = "update_rule must be MEQ_RULE_MEQMUON or MEQ_RULE_MUON";
+    return false;
+  }
   return true;
 }
 
-bool valid_kinds(const meq_shape* shapes, const int* kinds, int n, std::string* why) {
+bool valid_kinds(const meq_shape* shapes, const int* kinds, int n, int rule, std::string* why) {
   if (!kinds) return true;
   for (int i = 0; i < n; ++i) {
+    if (rule == MEQ_RULE_MUON && kinds[i] != KIND_HIDDEN) {
+      *why = "MEQ_RULE_MUON (Eq. (6)) applies to hidden 2D weights only; entry " + std::to_string(i) + " is not one";
+      return false;
+    }
     if (kinds[i] < 0 || kinds[i] > 2) { *why = "kind of entry " + std::to_string(i) + " is not a meq_kind"; return false; }
     if (kinds[i] == KIND_VECTOR && shapes[i].rows != 1) {
       *why = "vector entry " + std::to_string(i) + " must have shape (1, d)";
@@ -285,7 +294,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
   *off_partials = L->add(std::max({hchunks, tiles, xblks}) * 4);  // per momentum chunk or block
   *off_counters = L->add(int64_t(n) * 4);
   *off_x0s = L->add(int64_t(n) * 4 * 2);  // x0scale (cast pass) and the inverse norms (fused)
-  *off_stats = L->add(int64_t(n) * sizeof(MatStats));
+  *off_stats = L->add(int64_t(n) * sizeof(MatStats) + int64_t(n) * 2 * 8);  // stats, then direction counts
   st->step_bytes = sizeof(StepScalars) + 2 * int64_t(n) * sizeof(void*);
   *off_step = L->add(st->step_bytes);
   *off_err = L->add(64);
@@ -498,7 +507,7 @@ meq_status meq_state_bytes_kinds(const meq_shape* shapes, const int* kinds, int 
   meq_options o;
   if (opt) o = *opt; else meq_default_options(&o);
   std::string why;
-  if (!valid_shapes(shapes, n, &why) || !valid_kinds(shapes, kinds, n, &why) || !valid_options(o, &why))
+  if (!valid_shapes(shapes, n, &why) || !valid_options(o, &why) || !valid_kinds(shapes, kinds, n, o.update_rule, &why))
     return fail(nullptr, MEQ_ERR_INVALID_ARG, why);
   meq_state tmp;
   tmp.n = n;
@@ -526,7 +535,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   meq_options o;
   if (opt) o = *opt; else meq_default_options(&o);
   std::string why;
-  if (!valid_shapes(shapes, n, &why) || !valid_kinds(shapes, kinds, n, &why) || !valid_options(o, &why))
+  if (!valid_shapes(shapes, n, &why) || !valid_options(o, &why) || !valid_kinds(shapes, kinds, n, o.update_rule, &why))
     return fail(nullptr, MEQ_ERR_INVALID_ARG, why);
 
   int dev = 0;
@@ -584,6 +593,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   st->d_x0scale = reinterpret_cast<float*>(A + off_x0s);
   st->d_ginv = st->d_x0scale + n;
   st->d_stats = reinterpret_cast<MatStats*>(A + off_stats);
+  st->d_dircount = reinterpret_cast<unsigned long long*>(st->d_stats + n);
   st->d_step = A + off_step;
   st->d_err = reinterpret_cast<int*>(A + off_err);
   st->d_flag = st->d_err + 4;
@@ -641,6 +651,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   C.svec = st->d_svec;
   C.tvec = st->d_tvec;
   C.stats = st->d_stats;
+  C.dircount = st->d_dircount;
   C.total_chunks = st->total_chunks;
   C.total_hchunks = st->total_hchunks;
   C.total_tiles = st->total_tiles;
@@ -754,6 +765,7 @@ meq_status meq_step(float* const* params, const float* const* grads, meq_state* 
   std::memset(&sc, 0, sizeof(sc));
   sc.lr = lr, sc.mu = momentum, sc.wd = weight_decay, sc.eps = eps;
   sc.rho = st->opt.rho, sc.tie_atol = st->opt.tie_atol, sc.nesterov = st->opt.nesterov;
+  sc.rule = st->opt.update_rule;
   char* h = st->step_host.data();
   std::memcpy(h, &sc, sizeof(sc));
   std::memcpy(h + sizeof(sc), params, n * sizeof(void*));
@@ -868,6 +880,23 @@ meq_status meq_read_stats(meq_state* st, int i, float* r, float* c, double* gamm
   if (gamma_c) *gamma_c = hs.gamma_c;
   if (direction) *direction = hs.direction;
   return MEQ_OK;
+}
+
+meq_status meq_read_direction_counts(meq_state* st, int i, int64_t* rows, int64_t* cols) {
+  meq_status ms = check_index(st, i);
+  if (ms != MEQ_OK) return ms;
+  unsigned long long h[2];
+  cudaError_t e = cudaMemcpy(h, st->d_dircount + 2 * i, sizeof(h), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(st, e, "cudaMemcpy");
+  if (rows) *rows = static_cast<int64_t>(h[0]);
+  if (cols) *cols = static_cast<int64_t>(h[1]);
+  return MEQ_OK;
+}
+
+meq_status meq_reset_direction_counts(meq_state* st) {
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  cudaError_t e = cudaMemsetAsync(st->d_dircount, 0, sizeof(unsigned long long) * 2 * st->n, st->last_stream);
+  return e == cudaSuccess ? MEQ_OK : cuda_fail(st, e, "cudaMemsetAsync");
 }
 
 meq_status meq_set_profiling(meq_state* st, int enable) {

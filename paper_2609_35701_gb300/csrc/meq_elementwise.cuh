@@ -13,7 +13,7 @@ constexpr int kColSlab = 128;      // rows per block of the remaining-2D column 
 struct MatStats {
   double gamma_r;
   double gamma_c;
-  int32_t direction;  // 0 = row (N_r), 1 = column (N_c)
+  int32_t direction;  // 0 = row (N_r), 1 = column (N_c), 2 = two-sided, 3 = vector, 4 = Eq. (6) shape factor
   int32_t pad;
 };
 
@@ -37,6 +37,7 @@ struct LaunchCtx {
   float* svec;           // hidden: scale of the chosen side; others: 1 / row RMS
   float* tvec;           // remaining 2D: 1 / column RMS of the row-normalised momentum
   MatStats* stats;
+  unsigned long long* dircount;  // per entry: Eq. (11) row choices, column choices
   int64_t total_chunks, total_hchunks, total_tiles, total_rblks, total_slabs, total_xblks;
   int n_hidden;
 };

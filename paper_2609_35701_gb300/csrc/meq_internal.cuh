@@ -69,7 +69,7 @@ struct StepScalars {
   float lr, mu, wd, eps;
   float rho, tie_atol;
   int32_t nesterov;
-  int32_t pad;
+  int32_t rule;          // meq_update_rule
 };
 
 // --------------------------------------------------------------- GEMM side

@@ -41,6 +41,7 @@ class MeqOptions(ctypes.Structure):
         ("wait_timeout_ms", ctypes.c_float),
         ("ns_cta_pair", ctypes.c_int),
         ("ns_x0_fused", ctypes.c_int),
+        ("update_rule", ctypes.c_int),
     ]
 
 
@@ -50,8 +51,10 @@ EXPORTED = [
     "meq_read_ns_output", "meq_read_stats", "meq_kernels_per_step", "meq_debug_wait_selftest",
     "meq_set_profiling", "meq_read_profile", "meq_row_col_stats_noalloc",
     "meq_init_state_kinds", "meq_state_bytes_kinds", "meq_ns_gemm_launches_per_step",
+    "meq_read_direction_counts", "meq_reset_direction_counts",
 ]
 HIDDEN, REMAINING_2D, VECTOR = 0, 1, 2  # meq_kind
+RULE_MEQMUON, RULE_MUON = 0, 1          # meq_update_rule
 
 
 def _load():
@@ -102,6 +105,10 @@ def _load():
     lib.meq_state_bytes_kinds.restype = I
     lib.meq_ns_gemm_launches_per_step.argtypes = [P]
     lib.meq_ns_gemm_launches_per_step.restype = I
+    lib.meq_read_direction_counts.argtypes = [P, I, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)]
+    lib.meq_read_direction_counts.restype = I
+    lib.meq_reset_direction_counts.argtypes = [P]
+    lib.meq_reset_direction_counts.restype = I
     return lib
 
 
@@ -247,6 +254,15 @@ class MeqMuon:
         self._check(lib.meq_read_stats(self._st, i, rv.ctypes.data, cv.ctypes.data, ctypes.byref(gr),
                                        ctypes.byref(gc), ctypes.byref(d)))
         return {"r": rv, "c": cv, "gamma_r": gr.value, "gamma_c": gc.value, "direction": d.value}
+
+    def read_direction_counts(self, i):
+        """(row choices, column choices) of Eq. (11) for hidden weight i."""
+        r, c = ctypes.c_int64(), ctypes.c_int64()
+        self._check(lib.meq_read_direction_counts(self._st, i, ctypes.byref(r), ctypes.byref(c)))
+        return r.value, c.value
+
+    def reset_direction_counts(self):
+        self._check(lib.meq_reset_direction_counts(self._st))
 
     def set_profiling(self, enable):
         self._check(lib.meq_set_profiling(self._st, int(bool(enable))))

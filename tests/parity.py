@@ -53,6 +53,42 @@ def staged_update(U_gpu, direction, eps=O.DELTA):
     return O.row_normalize(U, eps) if direction == O.ROW else O.col_normalize(U, eps)
 
 
+def check_staged_stats(Ug, st_gpu, eps, out):
+    """Eqs. (7), (8) staged on the GPU's own U; returns the oracle's CVs."""
+    r_o, c_o = O.row_col_rms(Ug)
+    gr_o = O.coefficient_of_variation(r_o, eps)
+    gc_o = O.coefficient_of_variation(c_o, eps)
+    out["r"] = max_rel(st_gpu["r"], r_o, floor_frac=1e-6)
+    out["c"] = max_rel(st_gpu["c"], c_o, floor_frac=1e-6)
+    out["gamma_r"] = abs(st_gpu["gamma_r"] - gr_o) / max(gr_o, 1e-6)
+    out["gamma_c"] = abs(st_gpu["gamma_c"] - gc_o) / max(gc_o, 1e-6)
+    for k in ("r", "c", "gamma_r", "gamma_c"):
+        assert out[k] <= STATS_TOL, (k, out)
+    return gr_o, gc_o
+
+
+def check_muon_step(W0, G, B_prev, W1_gpu, B_gpu, U_gpu, st_gpu, lr, mu, wd, eps=O.DELTA, nesterov=False,
+                    update_tol=UPDATE_TOL):
+    """All checks of one matrix after one GPU step under the Muon rule,
+    Eq. (6): momentum end to end, statistics and params staged on the GPU's
+    own U, and the applied update U against the oracle's."""
+    W0 = np.asarray(W0, np.float64)
+    m, n = W0.shape
+    W1_ora, B_ora, U_ora = O.moonlight_step(W0, np.asarray(G, np.float64), np.asarray(B_prev, np.float64), lr, mu,
+                                            wd, nesterov=nesterov)
+    out = {"momentum": max_rel(B_gpu, B_ora, floor_frac=1.0)}
+    assert out["momentum"] <= MOMENTUM_TOL, out
+    Ug = np.asarray(U_gpu, np.float64)
+    check_staged_stats(Ug, st_gpu, eps, out)
+    assert st_gpu["direction"] == 4, st_gpu["direction"]
+    out["params_staged"] = max_rel(W1_gpu, O.moonlight_update(W0, Ug, lr, wd), floor_frac=1.0)
+    assert out["params_staged"] <= PARAM_TOL, out
+    applied = ((1.0 - lr * wd) * W0 - np.asarray(W1_gpu, np.float64)) / (lr * O.RHO * np.sqrt(max(m, n)))
+    out["update"] = rel_frob(applied, U_ora)
+    assert out["update"] <= update_tol, out
+    return out, W1_ora, B_ora
+
+
 def check_step(W0, G, B_prev, W1_gpu, B_gpu, U_gpu, st_gpu, lr, mu, wd, eps=O.DELTA, nesterov=False,
                update_tol=UPDATE_TOL, report=None):
     """All checks of one matrix after one GPU step. Returns a dict of errors."""
@@ -63,17 +99,8 @@ def check_step(W0, G, B_prev, W1_gpu, B_gpu, U_gpu, st_gpu, lr, mu, wd, eps=O.DE
     # momentum, Eq. (10)
     out["momentum"] = max_rel(B_gpu, B_ora, floor_frac=1.0)
     assert out["momentum"] <= MOMENTUM_TOL, out
-    # statistics staged on the GPU's own U, Eqs. (7), (8)
     Ug = np.asarray(U_gpu, np.float64)
-    r_o, c_o = O.row_col_rms(Ug)
-    gr_o = O.coefficient_of_variation(r_o, eps)
-    gc_o = O.coefficient_of_variation(c_o, eps)
-    out["r"] = max_rel(st_gpu["r"], r_o, floor_frac=1e-6)
-    out["c"] = max_rel(st_gpu["c"], c_o, floor_frac=1e-6)
-    out["gamma_r"] = abs(st_gpu["gamma_r"] - gr_o) / max(gr_o, 1e-6)
-    out["gamma_c"] = abs(st_gpu["gamma_c"] - gc_o) / max(gc_o, 1e-6)
-    for k in ("r", "c", "gamma_r", "gamma_c"):
-        assert out[k] <= STATS_TOL, (k, out)
+    gr_o, gc_o = check_staged_stats(Ug, st_gpu, eps, out)
     d_staged = O.select_direction(gr_o, gc_o)
     if d_staged != st_gpu["direction"]:
         assert abs(gr_o - gc_o) <= 2 * STATS_TOL * max(gr_o, gc_o) + 1e-6, ("staged direction", out)

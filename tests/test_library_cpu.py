@@ -47,7 +47,7 @@ def test_default_options_are_the_papers():
     assert abs(o.ns_a - g["ns"]["a"]) < 1e-6 and abs(o.ns_b - g["ns"]["b"]) < 1e-6 and abs(o.ns_c - g["ns"]["c"]) < 1e-6
     assert o.ns_steps == g["ns"]["steps"] and abs(o.rho - g["rho"]) < 1e-7
     assert o.nesterov == 0 and o.use_graph == 1
-    assert o.ns_cta_pair == 1 and o.ns_x0_fused == 1
+    assert o.ns_cta_pair == 1 and o.ns_x0_fused == 1 and o.update_rule == meq.RULE_MEQMUON
 
 
 def test_state_holds_momentum_only():
@@ -98,6 +98,11 @@ def test_host_validation_errors():
         assert e.value.status == 1
     with pytest.raises(meq.MeqError):
         meq.state_bytes([(4, 4)], ns_steps=0)
-    for field in ("ns_cta_pair", "ns_x0_fused"):
+    for field in ("ns_cta_pair", "ns_x0_fused", "update_rule"):
         with pytest.raises(meq.MeqError):
             meq.state_bytes([(4, 4)], **{field: 2})
+    # Eq. (6) is the hidden-weight baseline only
+    meq.state_bytes([(4, 4)], update_rule=meq.RULE_MUON)
+    with pytest.raises(meq.MeqError) as e:
+        meq.state_bytes([(4, 4), (1, 4)], kinds=[meq.HIDDEN, meq.VECTOR], update_rule=meq.RULE_MUON)
+    assert e.value.status == 1
