@@ -12,7 +12,8 @@ reordering or shape trick (no transposition of tall matrices, no symmetric
 Gram shortcut): each function is the equation it cites, written out.
 
 Equation numbers are the paper's:
-  Eq. (5)  quintic Newton-Schulz iteration           (Section 2, "Muon")
+  Eq. (5)  quintic Newton-Schulz iteration           (Section 2, "Muon");
+           its row / column CV trajectory               (Section 3.1)
   Eq. (6)  Muon with decoupled weight decay and RMS
            alignment (the Moonlight form), the baseline
            MeqMuon is compared with                   (Section 2, "Muon")
@@ -98,6 +99,26 @@ def newton_schulz(H, steps=NS_STEPS, coeffs=NS_COEFFS):
         AA = np.matmul(A, A)
         X = a * X + np.matmul(b * A + c * AA, X)
     return X
+
+
+def ns_cv_trajectory(H, steps=20, coeffs=NS_COEFFS, delta=DELTA):
+    """Eq. (8) CVs of the row and column RMS (Eq. (7)) of every iterate of
+    Eq. (5), k = 0..steps (Section 3.1 replays the NS iteration this way on
+    saved pre-NS matrices). Returns (gamma_r, gamma_c), each of length
+    steps + 1; a zero H gives zeros."""
+    a, b, c = coeffs
+    H = _f64(H)
+    nrm = np.sqrt(np.sum(H * H))
+    gr, gc = [], []
+    X = H / nrm if nrm > 0.0 else np.zeros_like(H)
+    for k in range(steps + 1):
+        r, cc = row_col_rms(X)
+        gr.append(coefficient_of_variation(r, delta))
+        gc.append(coefficient_of_variation(cc, delta))
+        if k < steps:
+            A = np.matmul(X, X.T)
+            X = a * X + np.matmul(b * A + c * np.matmul(A, A), X)
+    return np.array(gr), np.array(gc)
 
 
 def row_col_rms(X):

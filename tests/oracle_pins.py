@@ -452,6 +452,38 @@ def check_moonlight_step(O):
     assert np.abs(U - O.newton_schulz(G + mu * Bt)).max() < 1e-13
 
 
+def check_ns_cv_trajectory(O):
+    """Section 3.1 replay of Eq. (5). diag(3, 4, 12) with a zero row: every
+    iterate is [diag(f_k(3/13), f_k(4/13), f_k(12/13)); 0], so both CVs at k
+    are the population CV of the three scalar iterates (the zero row is
+    excluded). Rank one u v^T: every iterate is a multiple of u v^T, so the
+    trajectory is flat at (CV|u|, CV|v|). The last point is the CVs of the
+    K-step NS output, and the trajectory is scale-free."""
+    H = np.zeros((4, 3))
+    H[0, 0], H[1, 1], H[2, 2] = 3.0, 4.0, 12.0
+    gr, gc = O.ns_cv_trajectory(H, steps=20)
+    assert len(gr) == len(gc) == 21
+    x = np.array([3.0, 4.0, 12.0]) / 13.0
+    for k in range(21):
+        cv = np.std(x) / np.mean(x)
+        assert abs(gr[k] - cv) < 1e-12 and abs(gc[k] - cv) < 1e-12, (k, gr[k], gc[k], cv)
+        x = np.array([p_scalar(v) for v in x])
+    rng = np.random.default_rng(41)
+    u = rng.uniform(0.5, 2.0, 9) * rng.choice([-1.0, 1.0], 9)
+    v = rng.uniform(0.1, 3.0, 14) * rng.choice([-1.0, 1.0], 14)
+    gr, gc = O.ns_cv_trajectory(np.outer(u, v), steps=12)
+    cvu = np.std(np.abs(u)) / np.mean(np.abs(u))
+    cvv = np.std(np.abs(v)) / np.mean(np.abs(v))
+    assert np.abs(gr - cvu).max() < 1e-12 and np.abs(gc - cvv).max() < 1e-12
+    G = rng.standard_normal((10, 17)) * rng.uniform(0.1, 5.0, 10)[:, None]
+    gr, gc = O.ns_cv_trajectory(G, steps=5)
+    r5, c5 = O.row_col_rms(O.newton_schulz(G, steps=5))
+    assert abs(gr[5] - O.coefficient_of_variation(r5)) < 1e-12
+    assert abs(gc[5] - O.coefficient_of_variation(c5)) < 1e-12
+    gr2, gc2 = O.ns_cv_trajectory(1024.0 * G, steps=5)
+    assert np.abs(gr2 - gr).max() < 1e-12 and np.abs(gc2 - gc).max() < 1e-12
+
+
 # ------------------------------------------------------------ paper tables
 def llama_hidden_counts(a):
     q = a["q_heads"] * a["head_dim"]
@@ -487,5 +519,5 @@ ALL_CHECKS = [
     check_cv_hand_values, check_selection_rule, check_equilibration_invariants,
     check_orthogonality_constraint, check_two_sided_and_vector, check_momentum_closed_form,
     check_apply_closed_form, check_hidden_step_composition, check_param_step_branches,
-    check_moonlight_update, check_moonlight_step,
+    check_moonlight_update, check_moonlight_step, check_ns_cv_trajectory,
 ]

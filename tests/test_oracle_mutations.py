@@ -106,9 +106,17 @@ MUTATIONS = {
                            - lr * rho * np.sqrt(min(np.shape(U))) * np.asarray(U)),
     "moonlight_no_shape_factor": ("moonlight_update", lambda W, U, lr, wd, rho=0.2: (1 - lr * wd) * np.asarray(W)
                                   - lr * rho * np.asarray(U)),
+    "trajectory_skips_x0": ("ns_cv_trajectory", lambda H, steps=20, coeffs=None, delta=1e-7: _traj_shifted(H, steps)),
     "moonlight_coupled_decay": ("moonlight_update", lambda W, U, lr, wd, rho=0.2: (1 - wd) * np.asarray(W)
                                 - lr * rho * np.sqrt(max(np.shape(U))) * np.asarray(U)),
 }
+
+
+def _traj_shifted(H, steps):
+    """Trajectory that starts at X_1 instead of X_0 (an off-by-one)."""
+    O = fresh_oracle()
+    gr, gc = O.ns_cv_trajectory(H, steps + 1)
+    return gr[1:], gc[1:]
 
 
 def _col_then_row(B):
