@@ -55,7 +55,7 @@ typedef struct {
 /* Options fixed at init. meq_default_options() fills the paper's values. */
 typedef struct {
   float rho;              /* RMS alignment coefficient, Eq. (14); 0.2 (Section 4) */
-  int ns_steps;           /* K of Eq. (5); 5 (Sections 2 and 4); 1..16 */
+  int ns_steps;           /* K of Eq. (5); 5 (Sections 2 and 4); 1..32 */
   float ns_a, ns_b, ns_c; /* (3.4445, -4.7750, 2.0315), Section 2 */
   int nesterov;           /* 0: NS input B_t (Eq. (10), Algorithm 1);
                              1: NS input G_t + mu B_t (Nesterov look-ahead, Section 4) */
@@ -175,6 +175,21 @@ meq_status meq_read_stats(meq_state* st, int i, float* r, float* c,
 meq_status meq_read_direction_counts(meq_state* st, int i, int64_t* rows, int64_t* cols);
 /* Zero every entry's direction counts (enqueued on the state's stream). */
 meq_status meq_reset_direction_counts(meq_state* st);
+
+/* ---- diagnostics -------------------------------------------------------- */
+
+/* Row / column CV trajectory of the Newton-Schulz iterates (Section 3.1
+ * replays Eq. (5) on saved pre-NS matrices this way): gamma_r[k] and
+ * gamma_c[k] are the Eq. (8) CVs (over entries > eps) of the row and column
+ * RMS (Eq. (7)) of X_k, k = 0..steps, computed by this library's CUDA path
+ * with the NS options of opt (NULL: defaults; its ns_steps and update_rule
+ * are ignored). h: device fp32, rows x cols row-major, 16-byte aligned, read
+ * only. gamma_r, gamma_c: host arrays of steps + 1 doubles. steps: 0..32.
+ * Synchronous; allocates and frees its own device scratch. Errors:
+ * MEQ_ERR_INVALID_ARG (NULL, misaligned, bad sizes), MEQ_ERR_OOM, or the
+ * error of the step it runs. */
+meq_status meq_ns_cv_trajectory(const float* h, int64_t rows, int64_t cols, int steps, float eps,
+                                const meq_options* opt, double* gamma_r, double* gamma_c, void* cuda_stream);
 /* Number of kernels one meq_step launches (for launch accounting), and how
  * many of them are Newton-Schulz GEMM launches. */
 int meq_kernels_per_step(const meq_state* st);

@@ -139,7 +139,7 @@ meq_status cuda_fail(meq_state* st, cudaError_t e, const char* what) {
 }
 
 bool valid_options(const meq_options& o, std::string* why) {
-  if (o.ns_steps < 1 || o.ns_steps > 16) { *why = "ns_steps must be in 1..16"; return false; }
+  if (o.ns_steps < 1 || o.ns_steps > 32) { *why = "ns_steps must be in 1..32"; return false; }
   if (!(o.rho > 0.f) || !std::isfinite(o.rho)) { *why = "rho must be positive and finite"; return false; }
   if (!std::isfinite(o.ns_a) || !std::isfinite(o.ns_b) || !std::isfinite(o.ns_c)) { *why = "NS coefficients must be finite"; return false; }
   if (!(o.tie_atol >= 0.f)) { *why = "tie_atol must be >= 0"; return false; }
@@ -880,6 +880,66 @@ meq_status meq_read_stats(meq_state* st, int i, float* r, float* c, double* gamm
   if (gamma_c) *gamma_c = hs.gamma_c;
   if (direction) *direction = hs.direction;
   return MEQ_OK;
+}
+
+meq_status meq_ns_cv_trajectory(const float* h, int64_t rows, int64_t cols, int steps, float eps,
+                                const meq_options* opt, double* gamma_r, double* gamma_c, void* cuda_stream) {
+  if (!h || !gamma_r || !gamma_c) return fail(nullptr, MEQ_ERR_INVALID_ARG, "h, gamma_r and gamma_c must not be NULL");
+  if (reinterpret_cast<uintptr_t>(h) & 15u) return fail(nullptr, MEQ_ERR_INVALID_ARG, "h is not 16-byte aligned");
+  if (steps < 0 || steps > 32) return fail(nullptr, MEQ_ERR_INVALID_ARG, "steps must be in 0..32");
+  if (!(eps >= 0.f) || !std::isfinite(eps)) return fail(nullptr, MEQ_ERR_INVALID_ARG, "eps must be finite and >= 0");
+  meq_shape shape{rows, cols};
+  std::string why;
+  if (!valid_shapes(&shape, 1, &why)) return fail(nullptr, MEQ_ERR_INVALID_ARG, why);
+  meq_options o;
+  if (opt) o = *opt; else meq_default_options(&o);
+  o.update_rule = MEQ_RULE_MEQMUON;
+  o.use_graph = 0;
+  o.ns_steps = 1;
+  if (!valid_options(o, &why)) return fail(nullptr, MEQ_ERR_INVALID_ARG, why);
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  // scratch: W (rows x cols, left unchanged by lr = 0), r, c, the two CVs, the direction
+  const int64_t wb = round_up(rows * cols * 4, 256), rb = round_up(rows * 4, 256), cb = round_up(cols * 4, 256);
+  char* tmp = nullptr;
+  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&tmp), static_cast<size_t>(wb + rb + cb + 256));
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(nullptr, MEQ_ERR_OOM, "scratch allocation failed");
+  }
+  float* w = reinterpret_cast<float*>(tmp);
+  float* r = reinterpret_cast<float*>(tmp + wb);
+  float* c = reinterpret_cast<float*>(tmp + wb + rb);
+  double* g = reinterpret_cast<double*>(tmp + wb + rb + cb);
+  int* d = reinterpret_cast<int*>(g + 2);
+  meq_status ms = MEQ_OK;
+  e = cudaMemsetAsync(w, 0, static_cast<size_t>(rows * cols * 4), s);
+  if (e != cudaSuccess) ms = cuda_fail(nullptr, e, "cudaMemsetAsync");
+  // k = 0: X_0 = H / ||H||_F has the CVs of H (Eq. (8) is scale-free)
+  if (ms == MEQ_OK) ms = meq_row_col_stats_noalloc(h, rows, cols, eps, o.tie_atol, r, c, g, d, s);
+  double hg[2] = {0.0, 0.0};
+  if (ms == MEQ_OK) {
+    e = cudaMemcpyAsync(hg, g, sizeof(hg), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) ms = cuda_fail(nullptr, e, "cudaMemcpyAsync");
+  }
+  if (ms == MEQ_OK) gamma_r[0] = hg[0], gamma_c[0] = hg[1];
+  // k >= 1: the statistics of the k-step NS output of a one-matrix state fed
+  // H with no momentum history and mu = 0 (so its NS input is H), lr = 0
+  for (int k = 1; ms == MEQ_OK && k <= steps; ++k) {
+    o.ns_steps = k;
+    meq_state* st = nullptr;
+    ms = meq_init_state(&shape, 1, &o, cuda_stream, &st);
+    if (ms != MEQ_OK) break;
+    float* wp = w;
+    const float* hp = h;
+    ms = meq_step(&wp, &hp, st, &shape, 1, 0.f, 0.f, 0.f, eps, cuda_stream);
+    if (ms == MEQ_OK) ms = meq_sync(st);
+    if (ms == MEQ_OK) ms = meq_read_stats(st, 0, nullptr, nullptr, gamma_r + k, gamma_c + k, nullptr);
+    if (ms != MEQ_OK) g_init_error = st->last_error;
+    meq_free(st);
+  }
+  cudaFree(tmp);
+  return ms;
 }
 
 meq_status meq_read_direction_counts(meq_state* st, int i, int64_t* rows, int64_t* cols) {

@@ -51,7 +51,7 @@ EXPORTED = [
     "meq_read_ns_output", "meq_read_stats", "meq_kernels_per_step", "meq_debug_wait_selftest",
     "meq_set_profiling", "meq_read_profile", "meq_row_col_stats_noalloc",
     "meq_init_state_kinds", "meq_state_bytes_kinds", "meq_ns_gemm_launches_per_step",
-    "meq_read_direction_counts", "meq_reset_direction_counts",
+    "meq_read_direction_counts", "meq_reset_direction_counts", "meq_ns_cv_trajectory",
 ]
 HIDDEN, REMAINING_2D, VECTOR = 0, 1, 2  # meq_kind
 RULE_MEQMUON, RULE_MUON = 0, 1          # meq_update_rule
@@ -109,6 +109,9 @@ def _load():
     lib.meq_read_direction_counts.restype = I
     lib.meq_reset_direction_counts.argtypes = [P]
     lib.meq_reset_direction_counts.restype = I
+    lib.meq_ns_cv_trajectory.argtypes = [P, ctypes.c_int64, ctypes.c_int64, I, F, ctypes.POINTER(MeqOptions),
+                                         ctypes.POINTER(D), ctypes.POINTER(D), P]
+    lib.meq_ns_cv_trajectory.restype = I
     return lib
 
 
@@ -155,6 +158,19 @@ def state_bytes(shapes, kinds=None, **opts):
     if st != MEQ_OK:
         raise MeqError(st, lib.meq_last_error(None).decode())
     return p.value, w.value
+
+
+def ns_cv_trajectory(H, steps=20, eps=1e-7, stream=None, **opts):
+    """(gamma_r, gamma_c) of the NS iterates X_0..X_steps of a CUDA fp32
+    matrix H (meq_ns_cv_trajectory)."""
+    gr = (ctypes.c_double * (steps + 1))()
+    gc = (ctypes.c_double * (steps + 1))()
+    o = default_options(**opts)
+    st = lib.meq_ns_cv_trajectory(H.data_ptr(), H.shape[0], H.shape[1], int(steps), float(eps), ctypes.byref(o),
+                                  gr, gc, _stream_handle(stream))
+    if st != MEQ_OK:
+        raise MeqError(st, lib.meq_last_error(None).decode())
+    return np.array(list(gr)), np.array(list(gc))
 
 
 def row_col_stats_noalloc(U, r, c, gammas, direction, eps=1e-7, tie_atol=1e-6, stream=None):

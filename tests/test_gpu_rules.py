@@ -116,3 +116,30 @@ def test_direction_counts_follow_the_orthogonality_constraint(meq):
     assert opt.read_direction_counts(0) == (0, 5)   # wide: column-wise
     assert opt.read_direction_counts(1) == (5, 0)   # tall: row-wise
     opt.close()
+
+
+def test_ns_cv_trajectory_matches_oracle(meq):
+    """Section 3.1 replay of Eq. (5) through the CUDA path: the row and column
+    CVs of X_0..X_20 agree with the fp64 oracle's trajectory (the GPU runs
+    its 16-bit NS, so the CVs carry its ~1e-3 relative output error)."""
+    import torch
+
+    wl = W.custom_workload([(256, 640), (640, 256), (384, 384)], pattern="both", seed=17)
+    for i, (_, m, n) in enumerate(wl.shapes):
+        G = W.gradient(wl, i, 0)
+        gr, gc = meq.ns_cv_trajectory(G.cuda().contiguous(), steps=20)
+        orr, oc = O.ns_cv_trajectory(G.double().numpy(), steps=20)
+        assert gr.shape == (21,) and gc.shape == (21,)
+        assert abs(gr[0] - orr[0]) <= 1e-4 * orr[0] and abs(gc[0] - oc[0]) <= 1e-4 * max(oc[0], 1e-6)
+        assert np.all(np.abs(gr - orr) <= 5e-3 + 2e-2 * orr), (m, n, np.abs(gr - orr).max())
+        assert np.all(np.abs(gc - oc) <= 5e-3 + 2e-2 * oc), (m, n, np.abs(gc - oc).max())
+        # Section 3.1: orthogonalisation equalises the rows of a wide matrix
+        # and the columns of a tall one, leaving the other side's imbalance;
+        # a square matrix has both sides constrained
+        if m < n:
+            assert gr[20] < 0.1 * gr[0] and gr[20] < 0.2 * gc[20], (m, n, gr[[0, 20]], gc[[0, 20]])
+        elif m > n:
+            assert gc[20] < 0.1 * gc[0] and gc[20] < 0.2 * gr[20], (m, n, gr[[0, 20]], gc[[0, 20]])
+        else:
+            assert gr[20] < 0.1 * gr[0] and gc[20] < 0.1 * gc[0], (m, n, gr[[0, 20]], gc[[0, 20]])
+    torch.cuda.synchronize()
