@@ -212,6 +212,55 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_trajectory(args):
+    """Times meq_ns_cv_trajectory (one matrix of every hidden shape of the
+    workload, gradients of step 0) and the fp64 oracle's replay of the same
+    matrices on the host cores. One JSON line."""
+    import numpy as np
+    import torch
+
+    import __graft_entry__
+
+    __graft_entry__.build()
+    from oracle import meqmuon as O
+    from paper_2609_35701_gb300 import meq
+    from paper_2609_35701_gb300 import workloads as W
+
+    wl = W.get_workload(args.workload)
+    kinds = wl.kind_list()
+    firsts = {}
+    for i, (_, r, c) in enumerate(wl.shapes):
+        if kinds[i] == W.HIDDEN:
+            firsts.setdefault((r, c), i)
+    Hs = {rc: W.gradient(wl, i, 0) for rc, i in firsts.items()}
+    dev = {rc: h.cuda().contiguous() for rc, h in Hs.items()}
+    K = args.ns_trajectory
+    for _ in range(2):
+        for h in dev.values():
+            meq.ns_cv_trajectory(h, steps=K)
+    torch.cuda.synchronize()
+    reps = max(1, min(args.steps, 5))
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        for h in dev.values():
+            meq.ns_cv_trajectory(h, steps=K)
+    gpu_ms = (time.perf_counter() - t0) * 1e3 / reps
+    t0 = time.perf_counter()
+    for h in Hs.values():
+        O.ns_cv_trajectory(h.double().numpy(), steps=K)
+    cpu_ms = (time.perf_counter() - t0) * 1e3
+    shapes = ", ".join(f"{r}x{c}" for r, c in Hs)
+    line = {
+        "metric": f"NS CV trajectory replay, k = 0..{K} (Section 3.1)", "value": gpu_ms, "unit": "ms (all shapes)",
+        "n_gpus": 1, "steps": reps, "warmup": 2, "higher_is_better": False, "dtype": "fp16", "data": "synthetic",
+        "config": {"workload": args.workload, "shapes": shapes,
+                   "method": "one state per k (ns_steps = k) through the CUDA step, k = 0 by the statistics kernel"},
+        "cpu_baseline": {"value": cpu_ms, "unit": "ms (all shapes)", "cores": cpu_cores(), "kind": "oracle",
+                         "sample": f"fp64 oracle replay of the same {len(Hs)} matrices"},
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -224,10 +273,15 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--update-rule", default="meqmuon", choices=["meqmuon", "muon"],
                     help="meqmuon: Eq. (11) + Eq. (14); muon: the Eq. (6) comparison baseline (hidden weights only)")
+    ap.add_argument("--ns-trajectory", type=int, default=0, metavar="K",
+                    help="instead of the step, time the Section 3.1 CV replay of X_0..X_K (one matrix per shape)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.impl == "reference":
         run_reference(args)
+        return
+    if args.ns_trajectory:
+        run_trajectory(args)
         return
 
     import torch
