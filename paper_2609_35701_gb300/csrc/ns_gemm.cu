@@ -322,11 +322,32 @@ __device__ __forceinline__ void fill_half_rows(uint8_t* slot, int r, const float
   }
 }
 // The transposed block: element (row j, col r) = v[j] of lane r.
-__device__ __forceinline__ void fill_half_cols(uint8_t* slot, int r, const float* v, int fp16) {
+// Transposes, in place, the 32 x 32 16-bit block a warp holds in its slot
+// (64-byte rows of four 16-byte chunks, chunk k of row r at k ^ ((r >> 1) & 3)):
+// ldmatrix .trans reads each 8 x 8 sub-block (g, q) as its transpose and
+// stmatrix writes it back as sub-block (q, g). All reads finish before the
+// first write (the warp holds the whole block in registers in between).
+__device__ __forceinline__ void transpose_slot(uint8_t* slot, int lane) {
+  const uint32_t base = smem_u32(slot);
+  const int r8 = lane & 7, q = lane >> 3;
+  uint32_t f[4][4];
 #pragma unroll
-  for (int j = 0; j < 32; ++j) {
-    const int off = j * 64 + ((((r >> 3) ^ ((j >> 1) & 3))) << 4) + ((r & 7) << 1);
-    *reinterpret_cast<uint16_t*>(slot + off) = to_half_bits(v[j], fp16);
+  for (int g = 0; g < 4; ++g) {
+    const int row = 8 * g + r8;  // lane group q addresses sub-block (g, q)
+    const uint32_t addr = base + row * 64 + ((q ^ ((row >> 1) & 3)) << 4);
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(f[g][0]), "=r"(f[g][1]), "=r"(f[g][2]), "=r"(f[g][3])
+                 : "r"(addr)
+                 : "memory");
+  }
+  __syncwarp();
+#pragma unroll
+  for (int g = 0; g < 4; ++g) {
+    const int row = 8 * q + r8;  // the transpose of sub-block (g, q) is sub-block (q, g)
+    const uint32_t addr = base + row * 64 + ((g ^ ((row >> 1) & 3)) << 4);
+    asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(f[g][0]),
+                 "r"(f[g][1]), "r"(f[g][2]), "r"(f[g][3])
+                 : "memory");
   }
 }
 // 32 rows x 64 bytes (a 16-bit 32 x 32 block) -> global: rows
@@ -634,7 +655,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
                           min(4, (G.N - col0 + 7) / 8));
           } else {
             // U rows = NS columns col0 + j, U columns = NS rows row0 + r
-            fill_half_cols(slot, lane, v, 1);
+            fill_half_rows(slot, lane, v, 1);
+            __syncwarp();
+            transpose_slot(slot, lane);
             __syncwarp();
             store_block64(slot, lane, outm + static_cast<int64_t>(col0) * G.out_ld + row0 * 2, G.out_ld,
                           min(32, G.N - col0), min(4, (G.M - row0 + 7) / 8));
@@ -646,7 +669,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
           store_block64(slot, lane, outm + static_cast<int64_t>(row0) * G.out_ld + col0 * 2, G.out_ld, rows_valid, 4);
           if (G.sym && C > R) {
             __syncwarp();
-            fill_half_cols(slot, lane, v, G.out_fp16);
+            transpose_slot(slot, lane);
             __syncwarp();
             store_block64(slot, lane, outm + static_cast<int64_t>(col0) * G.out_ld + row0 * 2, G.out_ld,
                           min(32, G.M - col0), 4);
