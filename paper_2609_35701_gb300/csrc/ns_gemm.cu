@@ -15,14 +15,16 @@
 // P X equals a X + (b A + c A^2) X of Eq. (5) exactly in real arithmetic.
 // A and P are symmetric: their launches run only the tiles that hold a 32 x 32
 // block on or above the diagonal and store each strictly-upper block twice
-// (as is, and transposed), so every element is written from one accumulator.
+// (as is, and transposed in shared memory with ldmatrix.trans / stmatrix), so
+// every element is written from one accumulator.
 // X is stored scaled by a power of two alpha so its entries stay in the
 // normal range of fp16; the epilogues undo the scale in fp32.
 //
 // Roles (320 threads, one CTA per SM):
 //   warp 0 : TMA producer (one thread), shared-memory ring of 4 stages
 //            (single CTA) or 6 (CTA pair)
-//   warp 1 : TMEM allocator and tcgen05.mma issuer (one thread)
+//   warp 1 : TMEM allocator and tcgen05.mma issuer (one thread; with CTA
+//            pairs, the leader's thread issues cta_group::2 MMAs for both)
 //   warps 2-9 : epilogue; warp w reads TMEM lanes 32*(w%4) .. +31 and takes
 //               every other 32-column chunk (two warps per lane quarter, so
 //               each SM sub-partition can hide one warp's latencies behind
