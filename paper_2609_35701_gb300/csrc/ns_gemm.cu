@@ -287,14 +287,6 @@ __device__ __forceinline__ uint32_t pack_half2(float a, float b, int fp16) {
   __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<uint32_t*>(&h);
 }
-__device__ __forceinline__ uint16_t to_half_bits(float a, int fp16) {
-  if (fp16) {
-    __half h = __float2half_rn(a);
-    return *reinterpret_cast<uint16_t*>(&h);
-  }
-  __nv_bfloat16 h = __float2bfloat16_rn(a);
-  return *reinterpret_cast<uint16_t*>(&h);
-}
 __device__ __forceinline__ float2 unpack_half2(uint32_t w, int fp16) {
   if (fp16) {
     __half2 h = *reinterpret_cast<__half2*>(&w);
