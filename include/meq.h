@@ -41,7 +41,7 @@ typedef enum {
   MEQ_ERR_INVALID_ARG = 1,   /* null pointer, bad size, misaligned pointer, shape list differs from init */
   MEQ_ERR_OOM = 2,           /* device allocation failed or the workspace limit was exceeded */
   MEQ_ERR_CUDA = 3,          /* a CUDA runtime call failed (see meq_last_error) */
-  MEQ_ERR_NONFINITE = 4,     /* reserved: non-finite gradient detected */
+  MEQ_ERR_NONFINITE = 4,     /* a step's momentum had a non-finite norm (reported by meq_sync) */
   MEQ_ERR_TIMEOUT = 5,       /* a device-side bounded wait expired; the kernel returned early */
   MEQ_ERR_UNSUPPORTED = 6    /* no sm_103a device, or a size beyond the library's limits */
 } meq_status;
@@ -136,7 +136,13 @@ meq_status meq_step(float* const* params, const float* const* grads, meq_state* 
                     float weight_decay, float eps, void* cuda_stream);
 
 /* Wait for the state's enqueued work and report device-side errors
- * (MEQ_ERR_TIMEOUT for an expired bounded wait, MEQ_ERR_CUDA otherwise). */
+ * (MEQ_ERR_TIMEOUT for an expired bounded wait, MEQ_ERR_CUDA otherwise), then
+ * MEQ_ERR_NONFINITE if, in a step since the last meq_sync, the momentum of
+ * some entry had a NaN or infinite sum of squares (a non-finite gradient, or
+ * a momentum already non-finite); meq_last_error names the first such entry.
+ * Each report clears the condition. Such an entry's momentum and parameters
+ * take the non-finite values (no step is skipped); every other entry's step
+ * is unaffected, since entries are updated independently. */
 meq_status meq_sync(meq_state* st);
 
 /* Release all device memory of the state (synchronises first). NULL is a no-op. */

@@ -62,7 +62,8 @@ __global__ void __launch_bounds__(kThreads) momentum_norm_kernel(const MatInfo* 
                                                                  const StepScalars* __restrict__ sc,
                                                                  float* __restrict__ partials,
                                                                  unsigned int* __restrict__ counters,
-                                                                 float* __restrict__ x0scale) {
+                                                                 float* __restrict__ x0scale,
+                                                                 int* __restrict__ nonfinite) {
   pdl_allow_dependents();
   pdl_wait_predecessor();
   __shared__ float shf[32];
@@ -121,6 +122,7 @@ __global__ void __launch_bounds__(kThreads) momentum_norm_kernel(const MatInfo* 
   const float total = block_sum_f32(acc, shf);
   if (threadIdx.x == 0) {
     const float nrm = sqrtf(total);
+    if (!isfinite(total)) atomicCAS(nonfinite, 0, mi + 1);  // first non-finite entry, 1-based
     // Zero input: U = 0 (Eq. (5) is defined for a nonzero input only).
     x0scale[mi] = nrm > 0.f ? groups[M.group].alpha0 / nrm : 0.f;
     counters[mi] = 0u;
@@ -275,7 +277,7 @@ __global__ void __launch_bounds__(kThreads, 8) momentum_x0_kernel(const MatInfo*
 __global__ void __launch_bounds__(kThreads) x0norm_kernel(const MatInfo* __restrict__ mats,
                                                          const GroupInfo* __restrict__ groups,
                                                          const float* __restrict__ partials,
-                                                         float* __restrict__ ginv) {
+                                                         float* __restrict__ ginv, int* __restrict__ nonfinite) {
   pdl_allow_dependents();
   pdl_wait_predecessor();
   __shared__ float shf[32];
@@ -288,6 +290,7 @@ __global__ void __launch_bounds__(kThreads) x0norm_kernel(const MatInfo* __restr
   const float total = block_sum_f32(acc, shf);
   if (threadIdx.x == 0) {
     const float nrm = sqrtf(total);
+    if (!isfinite(total)) atomicCAS(nonfinite, 0, static_cast<int>(blockIdx.x) + 1);  // first non-finite entry, 1-based
     ginv[groups[M.group].mbase + M.gidx] = nrm > 0.f ? 1.0f / nrm : 0.f;
   }
 }
@@ -526,7 +529,8 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
                                                                float* __restrict__ rvec, float* __restrict__ cvec,
                                                                float* __restrict__ svec, float* __restrict__ tvec,
                                                                MatStats* __restrict__ stats,
-                                                               unsigned long long* __restrict__ dircount) {
+                                                               unsigned long long* __restrict__ dircount,
+                                                               int* __restrict__ nonfinite) {
   pdl_allow_dependents();
   pdl_wait_predecessor();
   __shared__ float shf[32];
@@ -539,6 +543,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
   const float inv_m = 1.0f / static_cast<float>(M.m);
   if (M.kind == KIND_VECTOR) {
     if (threadIdx.x == 0) {
+      if (!isfinite(r[0])) atomicCAS(nonfinite, 0, static_cast<int>(blockIdx.x) + 1);
       const float rms = sqrtf(r[0] * inv_n);  // r[0] holds the sum of squares
       r[0] = rms;
       s[0] = rms > delta ? 1.0f / rms : 0.f;
@@ -551,6 +556,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
   if (M.kind == KIND_TWO_SIDED) {
     float* t = tvec + M.vec_off;
     for (int64_t i = threadIdx.x; i < M.m; i += blockDim.x) {
+      if (!isfinite(r[i])) atomicCAS(nonfinite, 0, static_cast<int>(blockIdx.x) + 1);
       const float rms = sqrtf(r[i] * inv_n);  // r holds the row sums of squares
       r[i] = rms;
       s[i] = rms > delta ? 1.0f / rms : 0.f;
@@ -736,7 +742,7 @@ __global__ void wait_selftest_kernel(const volatile int* flag, int* err, unsigne
 
 cudaError_t launch_momentum_norm(const LaunchCtx& L, cudaStream_t st) {
   return launch_pdl(momentum_norm_kernel, dim3((unsigned)L.total_hchunks), dim3(kThreads), 0, st, 1, L.mats, L.nmat,
-                    L.groups, L.mom, L.grads, L.sc, L.partials, L.counters, L.x0scale);
+                    L.groups, L.mom, L.grads, L.sc, L.partials, L.counters, L.x0scale, L.nonfinite);
 }
 
 cudaError_t launch_momentum_x0(const LaunchCtx& L, cudaStream_t st) {
@@ -746,7 +752,7 @@ cudaError_t launch_momentum_x0(const LaunchCtx& L, cudaStream_t st) {
 
 cudaError_t launch_x0norm(const LaunchCtx& L, cudaStream_t st) {
   return launch_pdl(x0norm_kernel, dim3((unsigned)L.nmat), dim3(kThreads), 0, st, 1, L.mats, L.groups,
-                    static_cast<const float*>(L.partials), L.ginv);
+                    static_cast<const float*>(L.partials), L.ginv, L.nonfinite);
 }
 
 cudaError_t launch_rows(const LaunchCtx& L, cudaStream_t st) {
@@ -769,7 +775,8 @@ cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st) {
 
 cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st) {
   return launch_pdl(finalize_kernel, dim3(L.nmat), dim3(kFinThreads), 0, st, 1, L.mats, L.sc,
-                    static_cast<const float*>(L.parts), L.rvec, L.cvec, L.svec, L.tvec, L.stats, L.dircount);
+                    static_cast<const float*>(L.parts), L.rvec, L.cvec, L.svec, L.tvec, L.stats, L.dircount,
+                    L.nonfinite);
 }
 
 cudaError_t launch_apply(const LaunchCtx& L, cudaStream_t st) {

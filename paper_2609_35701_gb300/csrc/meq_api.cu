@@ -99,6 +99,7 @@ struct meq_state {
   char* d_step = nullptr;  // StepScalars, params[n], grads[n]
   int* d_err = nullptr;
   int* d_flag = nullptr;
+  int* d_nonfinite = nullptr;  // 1 + first entry with a non-finite momentum norm, 0 if none
   int64_t step_bytes = 0;
   std::vector<char> step_host;
   // launch plan
@@ -597,6 +598,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   st->d_step = A + off_step;
   st->d_err = reinterpret_cast<int*>(A + off_err);
   st->d_flag = st->d_err + 4;
+  st->d_nonfinite = st->d_err + 8;
   st->d_mats = reinterpret_cast<MatInfo*>(A + off_mats);
   st->d_groups = reinterpret_cast<GroupInfo*>(A + off_groups);
   for (size_t g = 0; g < st->groups.size(); ++g) {
@@ -652,6 +654,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   C.tvec = st->d_tvec;
   C.stats = st->d_stats;
   C.dircount = st->d_dircount;
+  C.nonfinite = st->d_nonfinite;
   C.total_chunks = st->total_chunks;
   C.total_hchunks = st->total_hchunks;
   C.total_tiles = st->total_tiles;
@@ -809,6 +812,15 @@ meq_status meq_sync(meq_state* st) {
     char buf[96];
     std::snprintf(buf, sizeof(buf), "device-side bounded wait expired (code 0x%x)", err);
     return fail(st, MEQ_ERR_TIMEOUT, buf);
+  }
+  int bad = 0;
+  e = cudaMemcpy(&bad, st->d_nonfinite, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(st, e, "reading the non-finite flag");
+  if (bad != 0) {
+    int zero = 0;
+    cudaMemcpy(st->d_nonfinite, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    return fail(st, MEQ_ERR_NONFINITE, "non-finite momentum (gradient, or a previous non-finite step) in entry " +
+                                           std::to_string(bad - 1));
   }
   return MEQ_OK;
 }

@@ -38,6 +38,7 @@ struct LaunchCtx {
   float* tvec;           // remaining 2D: 1 / column RMS of the row-normalised momentum
   MatStats* stats;
   unsigned long long* dircount;  // per entry: Eq. (11) row choices, column choices
+  int* nonfinite;                // 1 + index of the first entry whose momentum had a non-finite norm, or 0
   int64_t total_chunks, total_hchunks, total_tiles, total_rblks, total_slabs, total_xblks;
   int n_hidden;
 };
