@@ -43,7 +43,8 @@ typedef enum {
   MEQ_ERR_CUDA = 3,          /* a CUDA runtime call failed (see meq_last_error) */
   MEQ_ERR_NONFINITE = 4,     /* a step's momentum had a non-finite norm (reported by meq_sync) */
   MEQ_ERR_TIMEOUT = 5,       /* a device-side bounded wait expired; the kernel returned early */
-  MEQ_ERR_UNSUPPORTED = 6    /* no sm_103a device, or a size beyond the library's limits */
+  MEQ_ERR_UNSUPPORTED = 6,   /* no sm_103a device, or a size beyond the library's limits */
+  MEQ_ERR_CORRUPTED = 7      /* meq_check_canaries found a workspace guard band overwritten */
 } meq_status;
 
 /* One matrix: rows = out features (m), cols = in features (n). */
@@ -73,6 +74,8 @@ typedef struct {
                              then runs its X and P operands in bf16. 0: a separate pass
                              writes the normalised X_0 in the format ns_fp16_mask gives it. */
   int update_rule;        /* meq_update_rule; default MEQ_RULE_MEQMUON */
+  int debug_canaries;     /* 1: guard bands of a fixed byte pattern surround every workspace
+                             buffer (meq_check_canaries); default 0 */
 } meq_options;
 
 /* Update applied to the hidden 2D weights after momentum and Newton-Schulz. */
@@ -183,6 +186,17 @@ meq_status meq_read_direction_counts(meq_state* st, int i, int64_t* rows, int64_
 meq_status meq_reset_direction_counts(meq_state* st);
 
 /* ---- diagnostics -------------------------------------------------------- */
+
+/* With debug_canaries set at init: synchronise the state's stream and check
+ * that every guard band still holds its pattern. MEQ_OK, or
+ * MEQ_ERR_CORRUPTED with *bad_offset (may be NULL) = the arena offset of the
+ * first changed byte (-1 otherwise); MEQ_ERR_INVALID_ARG without guards. */
+meq_status meq_check_canaries(meq_state* st, int64_t* bad_offset);
+/* Number of guard bands (0 without debug_canaries). */
+int meq_canary_count(const meq_state* st);
+/* Test hook: overwrite one byte of guard band `index` from the host
+ * (cudaMemset), so that tests can check meq_check_canaries. */
+meq_status meq_debug_corrupt_canary(meq_state* st, int index);
 
 /* Row / column CV trajectory of the Newton-Schulz iterates (Section 3.1
  * replays Eq. (5) on saved pre-NS matrices this way): gamma_r[k] and

@@ -55,11 +55,27 @@ struct Group {
 };
 
 // Sub-allocation plan of the arena (offsets in bytes).
+// With guards on (option debug_canaries), a band of kGuardBytes precedes the
+// first buffer and follows every buffer; it is filled with kGuardByte at init
+// and meq_check_canaries looks for bytes a kernel wrote into it.
+constexpr int64_t kGuardBytes = 4096;
+constexpr int kGuardByte = 0xA5;
+
 struct Layout {
   int64_t total = 0;
+  bool guards = false;
+  std::vector<std::pair<int64_t, int64_t>> guard_ranges;  // (offset, bytes)
+  explicit Layout(bool with_guards = false) : guards(with_guards) {
+    if (guards) guard(0);
+  }
+  void guard(int64_t off) {
+    guard_ranges.emplace_back(off, kGuardBytes);
+    total = off + kGuardBytes;
+  }
   int64_t add(int64_t bytes) {
     const int64_t off = total;
     total += round_up(std::max<int64_t>(bytes, 1), kAlignBytes);
+    if (guards) guard(total);
     return off;
   }
 };
@@ -115,6 +131,7 @@ struct meq_state {
   std::vector<std::vector<cudaEvent_t>> prof_events;  // 6 events per profiled step
   std::string last_error;
   int64_t persistent_bytes = 0;
+  std::vector<std::pair<int64_t, int64_t>> guard_ranges;  // arena guard bands (debug_canaries)
 };
 
 namespace {
@@ -148,6 +165,7 @@ bool valid_options(const meq_options& o, std::string* why) {
   if (o.workspace_limit_bytes < 0) { *why = "workspace_limit_bytes must be >= 0"; return false; }
   if (o.ns_cta_pair != 0 && o.ns_cta_pair != 1) { *why = "ns_cta_pair must be 0 or 1"; return false; }
   if (o.ns_x0_fused != 0 && o.ns_x0_fused != 1) { *why = "ns_x0_fused must be 0 or 1"; return false; }
+  if (o.debug_canaries != 0 && o.debug_canaries != 1) { *why = "debug_canaries must be 0 or 1"; return false; }
   if (o.update_rule != MEQ_RULE_MEQMUON && o.update_rule != MEQ_RULE_MUON) {
     *why = "update_rule must be MEQ_RULE_MEQMUON or MEQ_RULE_MUON";
     return false;
@@ -482,6 +500,7 @@ void meq_default_options(meq_options* o) {
   o->wait_timeout_ms = 4000.f;
   o->ns_cta_pair = 1;
   o->ns_x0_fused = 1;
+  o->debug_canaries = 0;
 }
 
 const char* meq_status_string(meq_status s) {
@@ -493,6 +512,7 @@ const char* meq_status_string(meq_status s) {
     case MEQ_ERR_NONFINITE: return "MEQ_ERR_NONFINITE";
     case MEQ_ERR_TIMEOUT: return "MEQ_ERR_TIMEOUT";
     case MEQ_ERR_UNSUPPORTED: return "MEQ_ERR_UNSUPPORTED";
+    case MEQ_ERR_CORRUPTED: return "MEQ_ERR_CORRUPTED";
   }
   return "MEQ_ERR_UNKNOWN";
 }
@@ -516,7 +536,7 @@ meq_status meq_state_bytes_kinds(const meq_shape* shapes, const int* kinds, int 
   tmp.kinds.assign(n, KIND_HIDDEN);
   if (kinds) tmp.kinds.assign(kinds, kinds + n);
   tmp.opt = o;
-  Layout L;
+  Layout L(o.debug_canaries != 0);
   int64_t a[13];
   std::vector<int64_t> goffs;
   plan(&tmp, &L, &a[0], &a[1], &a[2], &a[3], &a[4], &a[5], &a[6], &a[7], &a[8], &a[9], &a[10], &a[11], &goffs);
@@ -564,7 +584,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   st->device = dev;
   st->num_sms = prop.multiProcessorCount;
 
-  Layout L;
+  Layout L(o.debug_canaries != 0);
   int64_t off_mom, off_u, off_vec4, off_cpart, off_partials, off_counters, off_x0s, off_stats, off_step, off_err, off_mats,
       off_groups;
   std::vector<int64_t> goffs;
@@ -619,6 +639,9 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
     gi[g].mbase = G.mbase;
   }
   bool ok = cudaMemsetAsync(st->arena, 0, static_cast<size_t>(L.total), s) == cudaSuccess;
+  st->guard_ranges = L.guard_ranges;
+  for (const auto& g : st->guard_ranges)
+    ok = ok && cudaMemsetAsync(st->arena + g.first, kGuardByte, static_cast<size_t>(g.second), s) == cudaSuccess;
   ok = ok && cudaMemcpyAsync(st->d_mats, st->mats.data(), sizeof(MatInfo) * n, cudaMemcpyHostToDevice, s) == cudaSuccess;
   ok = ok && cudaMemcpyAsync(st->d_groups, gi.data(), sizeof(GroupInfo) * gi.size(), cudaMemcpyHostToDevice, s) == cudaSuccess;
   ok = ok && cudaStreamSynchronize(s) == cudaSuccess;
@@ -953,6 +976,36 @@ meq_status meq_ns_cv_trajectory(const float* h, int64_t rows, int64_t cols, int 
   cudaFree(tmp);
   return ms;
 }
+
+meq_status meq_check_canaries(meq_state* st, int64_t* bad_offset) {
+  if (bad_offset) *bad_offset = -1;
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  if (st->guard_ranges.empty()) return fail(st, MEQ_ERR_INVALID_ARG, "the state was created without debug_canaries");
+  cudaError_t e = cudaStreamSynchronize(st->last_stream);
+  if (e != cudaSuccess) return cuda_fail(st, e, "cudaStreamSynchronize");
+  std::vector<unsigned char> h(static_cast<size_t>(kGuardBytes));
+  for (const auto& g : st->guard_ranges) {
+    e = cudaMemcpy(h.data(), st->arena + g.first, static_cast<size_t>(g.second), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(st, e, "cudaMemcpy");
+    for (int64_t k = 0; k < g.second; ++k)
+      if (h[static_cast<size_t>(k)] != kGuardByte) {
+        if (bad_offset) *bad_offset = g.first + k;
+        return fail(st, MEQ_ERR_CORRUPTED, "workspace guard band overwritten at arena offset " + std::to_string(g.first + k));
+      }
+  }
+  return MEQ_OK;
+}
+
+meq_status meq_debug_corrupt_canary(meq_state* st, int index) {
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  if (index < 0 || index >= static_cast<int>(st->guard_ranges.size()))
+    return fail(st, MEQ_ERR_INVALID_ARG, "no guard band with that index");
+  const auto& g = st->guard_ranges[static_cast<size_t>(index)];
+  cudaError_t e = cudaMemset(st->arena + g.first + g.second / 2, 0, 1);  // host-side write of one byte
+  return e == cudaSuccess ? MEQ_OK : cuda_fail(st, e, "cudaMemset");
+}
+
+int meq_canary_count(const meq_state* st) { return st ? static_cast<int>(st->guard_ranges.size()) : 0; }
 
 meq_status meq_read_direction_counts(meq_state* st, int i, int64_t* rows, int64_t* cols) {
   meq_status ms = check_index(st, i);

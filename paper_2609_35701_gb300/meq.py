@@ -17,7 +17,7 @@ LIB_PATH = os.path.join(_HERE, "libmeq.so")
 MEQ_OK = 0
 STATUS_NAMES = {
     0: "MEQ_OK", 1: "MEQ_ERR_INVALID_ARG", 2: "MEQ_ERR_OOM", 3: "MEQ_ERR_CUDA",
-    4: "MEQ_ERR_NONFINITE", 5: "MEQ_ERR_TIMEOUT", 6: "MEQ_ERR_UNSUPPORTED",
+    4: "MEQ_ERR_NONFINITE", 5: "MEQ_ERR_TIMEOUT", 6: "MEQ_ERR_UNSUPPORTED", 7: "MEQ_ERR_CORRUPTED",
 }
 ROW, COL = 0, 1
 
@@ -42,6 +42,7 @@ class MeqOptions(ctypes.Structure):
         ("ns_cta_pair", ctypes.c_int),
         ("ns_x0_fused", ctypes.c_int),
         ("update_rule", ctypes.c_int),
+        ("debug_canaries", ctypes.c_int),
     ]
 
 
@@ -52,6 +53,7 @@ EXPORTED = [
     "meq_set_profiling", "meq_read_profile", "meq_row_col_stats_noalloc",
     "meq_init_state_kinds", "meq_state_bytes_kinds", "meq_ns_gemm_launches_per_step",
     "meq_read_direction_counts", "meq_reset_direction_counts", "meq_ns_cv_trajectory",
+    "meq_check_canaries", "meq_canary_count", "meq_debug_corrupt_canary",
 ]
 HIDDEN, REMAINING_2D, VECTOR = 0, 1, 2  # meq_kind
 RULE_MEQMUON, RULE_MUON = 0, 1          # meq_update_rule
@@ -112,6 +114,12 @@ def _load():
     lib.meq_ns_cv_trajectory.argtypes = [P, ctypes.c_int64, ctypes.c_int64, I, F, ctypes.POINTER(MeqOptions),
                                          ctypes.POINTER(D), ctypes.POINTER(D), P]
     lib.meq_ns_cv_trajectory.restype = I
+    lib.meq_check_canaries.argtypes = [P, ctypes.POINTER(ctypes.c_int64)]
+    lib.meq_check_canaries.restype = I
+    lib.meq_canary_count.argtypes = [P]
+    lib.meq_canary_count.restype = I
+    lib.meq_debug_corrupt_canary.argtypes = [P, I]
+    lib.meq_debug_corrupt_canary.restype = I
     return lib
 
 
@@ -276,6 +284,15 @@ class MeqMuon:
         r, c = ctypes.c_int64(), ctypes.c_int64()
         self._check(lib.meq_read_direction_counts(self._st, i, ctypes.byref(r), ctypes.byref(c)))
         return r.value, c.value
+
+    def check_canaries(self):
+        """Raises MeqError (MEQ_ERR_CORRUPTED) if a workspace guard band changed."""
+        off = ctypes.c_int64()
+        self._check(lib.meq_check_canaries(self._st, ctypes.byref(off)))
+
+    @property
+    def canary_count(self):
+        return lib.meq_canary_count(self._st)
 
     def reset_direction_counts(self):
         self._check(lib.meq_reset_direction_counts(self._st))

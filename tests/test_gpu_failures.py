@@ -60,3 +60,60 @@ def test_nonfinite_gradient_reported_and_contained(meq, bad, value):
             assert not np.isfinite(poisoned[i]).all()
         else:
             assert np.array_equal(clean[i], poisoned[i]), i
+
+
+@pytest.mark.parametrize("pair", [1, 0], ids=["cta_pair", "single_cta"])
+def test_no_write_outside_buffers(meq, pair):
+    """Ragged shapes of every parameter type, three steps: the guard bands
+    around every workspace buffer keep their pattern, the caller's parameter
+    buffers are not written outside their extent (guard bands of a sentinel
+    value before and after each), and the gradients are not written at all."""
+    import torch
+
+    shapes = [(200, 333), (333, 200), (1, 7), (7, 1), (129, 385), (1, 300), (300, 90)]
+    kinds = [meq.HIDDEN] * 5 + [meq.VECTOR, meq.REMAINING_2D]
+    wl = W.custom_workload(shapes, pattern="both", seed=23)
+    opt = meq.MeqMuon(shapes, kinds=kinds, debug_canaries=1, ns_cta_pair=pair)
+    assert opt.canary_count > 2 * len(shapes)
+    GB = 1024  # floats of guard on each side (keeps every view 16-byte aligned)
+    sentinel = 12345.0
+
+    def banded(ts):
+        bufs, views = [], []
+        for t in ts:
+            b = torch.full((2 * GB + t.numel(),), sentinel, device="cuda")
+            b[GB:GB + t.numel()] = t.reshape(-1).cuda()
+            bufs.append(b)
+            views.append(b[GB:GB + t.numel()].view(t.shape))
+        return bufs, views
+
+    pbufs, params = banded(W.initial_weights(wl))
+    for t in range(3):
+        gbufs, grads = banded(W.gradients(wl, t))
+        before = [g.clone() for g in grads]
+        opt.step(params, grads, LR, MU, WD, EPS)
+        opt.sync()
+        for b, g, g0, (r, c) in zip(gbufs, grads, before, shapes):
+            assert torch.equal(g, g0)
+            assert (b[:GB] == sentinel).all() and (b[GB + r * c:] == sentinel).all()
+        for b, (r, c) in zip(pbufs, shapes):
+            assert (b[:GB] == sentinel).all() and (b[GB + r * c:] == sentinel).all()
+    opt.check_canaries()
+    opt.close()
+
+
+def test_canary_check_detects_a_change(meq):
+    """The checker itself: a byte written into one guard band (from the host)
+    is reported as MEQ_ERR_CORRUPTED."""
+    shapes = [(128, 192), (192, 128)]
+    wl = W.custom_workload(shapes, pattern="both", seed=3)
+    opt = meq.MeqMuon(shapes, debug_canaries=1)
+    params = [w.cuda() for w in W.initial_weights(wl)]
+    opt.step(params, [g.cuda() for g in W.gradients(wl, 0)], LR, MU, WD, EPS)
+    opt.sync()
+    opt.check_canaries()
+    meq.lib.meq_debug_corrupt_canary(opt._st, opt.canary_count // 2)
+    with pytest.raises(meq.MeqError) as e:
+        opt.check_canaries()
+    assert e.value.status == 7
+    opt.close()
