@@ -27,6 +27,8 @@
 #include <vector>
 
 #include "../../include/meq.h"
+
+#include <nvtx3/nvToolsExt.h>
 #include "meq_elementwise.cuh"
 
 using namespace meq;
@@ -700,9 +702,32 @@ static void drop_profile(meq_state* st) {
   st->prof_events.clear();
 }
 
+// One open NVTX range at a time (closed on the next stage and on scope exit).
+struct NvtxStages {
+  bool open = false;
+  void next(const char* name) {
+    if (open) nvtxRangePop();
+    open = name != nullptr;
+    if (open) nvtxRangePushA(name);
+  }
+  ~NvtxStages() { next(nullptr); }
+};
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+};
+
 static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev = nullptr) {
   const LaunchCtx& C = st->ctx;
-  auto mark = [&](int i) { if (ev) cudaEventRecord(ev[i], s); };
+  // NVTX ranges name the stages on the host timeline (each eager enqueue, or
+  // the capture of the graph); CUDA events time them on the stream.
+  // (nested in the "meq_step" range: ncu selects e.g. --nvtx-include "meq_step/ns_gemm/")
+  static const char* const kStage[5] = {"momentum", "cast_x0", "ns_gemm", "statistics", "apply"};
+  NvtxStages stage;
+  auto mark = [&](int i) {
+    if (ev) cudaEventRecord(ev[i], s);
+    stage.next(i < 5 ? kStage[i] : nullptr);
+  };
   cudaError_t e = cudaSuccess;
   mark(0);
   const bool fused = st->opt.ns_x0_fused != 0;
@@ -774,6 +799,7 @@ static meq_status capture_graph(meq_state* st) {
 
 meq_status meq_step(float* const* params, const float* const* grads, meq_state* st, const meq_shape* shapes, int n,
                     float lr, float momentum, float weight_decay, float eps, void* cuda_stream) {
+  NvtxRange range("meq_step");
   if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
   if (!params || !grads || !shapes) return fail(st, MEQ_ERR_INVALID_ARG, "params, grads and shapes must be non-NULL");
   if (n != st->n) return fail(st, MEQ_ERR_INVALID_ARG, "n differs from the init-time shape list");
