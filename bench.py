@@ -34,6 +34,7 @@ sys.path.insert(0, ROOT)
 LR, MU, WD, EPS = 0.02, 0.95, 0.1, 1e-7
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 BW_BYTES_PER_ELEM = 24  # read G, B; write B; write X_0 (2 B); read U (2 B); read + write W
+REFERENCE_BUDGET_S = 150.0   # wall-clock cap on the timed oracle samples of --impl reference
 COPY_CHUNK = 8 << 20          # elements (32 MB) per host <-> device copy of the end-to-end loop
 
 
@@ -206,9 +207,12 @@ def run_reference(args):
         oracle_sample(wl, w, rule=args.update_rule)
     vals = []
     sampled = None
+    t0 = time.perf_counter()
     for k in range(args.steps):
         ms, sampled = oracle_sample(wl, k, rule=args.update_rule)
         vals.append(ms)
+        if time.perf_counter() - t0 > REFERENCE_BUDGET_S:
+            break  # the samples are timed on the host cores: keep the whole run to a few minutes
     v = statistics.median(vals)
     cores = cpu_cores()
     sample = (f"one matrix per shape class ({', '.join(sampled)}) per step, fp64 oracle, "
@@ -217,7 +221,7 @@ def run_reference(args):
         "impl": "reference", "metric": "MeqMuon optimizer step time (all hidden 2D weights)", "value": v,
         "unit": "ms/step", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": v, "higher_is_better": False, "scaling": "strong", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": args.workload, "matrices": len(wl.shapes), "elements": wl.numel,
+        "timed_steps": len(vals), "data": "synthetic", "config": {"workload": args.workload, "matrices": len(wl.shapes), "elements": wl.numel,
                                         "update_rule": "Eq. (11) + Eq. (14)" if args.update_rule == "meqmuon" else "Eq. (6)"},
         "cpu_baseline": {"value": v, "unit": "ms/step", "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": v, "unit": "ms/step", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},

@@ -22,7 +22,7 @@ def test_reference_arm_json_line():
     for k in ("impl", "metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better",
               "scaling", "vs_baseline", "dtype", "data", "config", "cpu_baseline", "e2e"):
         assert k in d, k
-    assert d["impl"] == "reference" and d["higher_is_better"] is False and d["steps"] == 2
+    assert d["impl"] == "reference" and d["higher_is_better"] is False and d["steps"] == 2 and d["timed_steps"] == 2
     assert d["value"] > 0 and d["unit"] == "ms/step" and d["config"]["workload"] == "single256"
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
