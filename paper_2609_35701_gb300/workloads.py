@@ -7,7 +7,7 @@ tensors it makes, so the two sides always see identical fp32 inputs.
 Shapes follow the paper's PyTorch layout (rows = output features, columns =
 input features, Section 3.1). The hidden 2D weights of one Llama-style layer
 are q/k/v/o (hidden x hidden for multi-head attention), gate/up (ffn x hidden)
-and down (hidden x ffn) (Section 1 and Table 8). The Llama-130M and
+and down (hidden x ffn) (Section 1 and Table 11). The Llama-130M and
 Llama-350M sets below are exactly the paper's N_h of Section 4 ("Memory
 overhead"), which the tests check against Table 5.
 
@@ -63,7 +63,7 @@ HIDDEN, REMAINING_2D, VECTOR = 0, 1, 2   # parameter types of Algorithm 1
 
 def full_model_params(layers, hidden, ffn, vocab, q_heads, kv_heads, head_dim=64, tied=False, qkv_bias=False):
     """(name, rows, cols, kind) of every trainable parameter of a
-    pre-norm SwiGLU decoder (Table 8 architectures): the hidden 2D weights,
+    pre-norm SwiGLU decoder (Table 11 architectures): the hidden 2D weights,
     the token embedding and LM head (one matrix when tied), two RMSNorm
     weights per layer and a final one, and q/k/v biases when present
     (Qwen2). 1D parameters are given as (1, d)."""
@@ -128,7 +128,7 @@ def _full(name, layers, hidden, ffn, vocab, heads, steps=10):
                     kinds=[k for _, _, _, k in params])
 
 
-# Every trainable parameter of Llama-60M / Llama-130M (Table 8), as one
+# Every trainable parameter of Llama-60M / Llama-130M (Table 11), as one
 # optimizer state (Algorithm 1 over all three parameter types).
 WORKLOADS["llama60m_full"] = _full("llama60m_full", 8, 512, 1376, 32000, 8)
 WORKLOADS["llama130m_full"] = _full("llama130m_full", 12, 768, 2048, 32000, 12)

@@ -14,7 +14,7 @@ the oracle disagrees with a value fixed by the paper or by mathematics:
   * invariants: unit-RMS rows / columns after Eq. (9), idempotence, scale
     and sign invariance, transpose equivariance, zero rows and columns,
     and the orthogonality constraint of Section 3.1 on exact Orth;
-  * paper tables: Table 5 state memory from Table 8 architectures;
+  * paper tables: Table 5 state memory from Table 11 architectures;
   * the Muon baseline of Eq. (6): the shape factor sqrt(max(m, n)) gives an
     exactly orthogonal update unit RMS; closed forms on the Hadamard and
     known-SVD inputs.
@@ -495,7 +495,7 @@ def llama_hidden_counts(a):
 
 
 def check_state_memory_table(O=None):
-    """Table 5 from Table 8: Muon = N_h + 2 N_a, NorMuon = + R_h, MeqMuon =
+    """Table 5 from Table 11: Muon = N_h + 2 N_a, NorMuon = + R_h, MeqMuon =
     N_h + N_a values of 4 bytes (Section 4, 'Memory overhead')."""
     g = golden()
     for name, a in g["architecture"].items():

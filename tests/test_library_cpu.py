@@ -66,7 +66,7 @@ def test_state_holds_momentum_only():
 
 def test_full_model_state_reproduces_table5():
     """Algorithm 1 over every trainable parameter keeps one fp32 momentum value
-    per parameter: the library's persistent bytes for the full Table 8 models
+    per parameter: the library's persistent bytes for the full Table 11 models
     equal the MeqMuon column of Table 5 (Section 4, 'Memory overhead')."""
     from paper_2609_35701_gb300 import meq, workloads as W
 

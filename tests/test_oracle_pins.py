@@ -18,7 +18,7 @@ def test_state_memory_table5():
 
 def test_llama_hidden_sets_match_paper_counts():
     """The llama130m / llama350m workloads are the paper's hidden sets: their
-    element counts equal N_h of Llama-130M / Llama-350M (Table 8)."""
+    element counts equal N_h of Llama-130M / Llama-350M (Table 11)."""
     from paper_2609_35701_gb300 import workloads as W
     g = P.golden()["architecture"]
     for wl, arch in (("llama130m", "Llama-130M"), ("llama350m", "Llama-350M")):
