@@ -75,6 +75,26 @@ def test_ragged_shapes_two_steps(meq, shapes, pair):
     assert all(r["update"] <= PT.UPDATE_TOL for r in rep)
 
 
+@pytest.mark.parametrize("pair", [1, 0], ids=["cta_pair", "single_cta"])
+def test_separate_x0_cast(meq, pair):
+    """X_0 normalised and cast by its own pass (ns_x0_fused = 0: momentum +
+    norm kernel, then the cast kernel) instead of inside the first NS
+    products; ragged shapes, two steps, staged against the oracle."""
+    wl = W.custom_workload([(200, 333), (333, 200), (129, 385), (7, 1)], pattern="both", seed=29)
+    rep = []
+    run_staged(meq, wl, 2, report=rep, ns_x0_fused=0, ns_cta_pair=pair)
+    assert all(r["update"] <= PT.UPDATE_TOL for r in rep)
+
+
+def test_mixed_iteration_formats(meq):
+    """Per-iteration operand formats: bf16 for iterations 0 and 1, fp16 for
+    2..4 (ns_fp16_mask = 0b11100), so the products switch format mid-way."""
+    wl = W.custom_workload([(256, 640), (640, 256), (384, 384)], pattern="both", seed=31)
+    rep = []
+    run_staged(meq, wl, 2, report=rep, update_tol=2e-2, ns_fp16_mask=0b11100)
+    assert all(r["update"] <= 2e-2 for r in rep)
+
+
 def test_llama130m_sampled_ten_steps(meq):
     """Llama-130M hidden set (84 matrices, the launch the benchmark times),
     10 steps; sampled matrices checked against the oracle at every step."""
