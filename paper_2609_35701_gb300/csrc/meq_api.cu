@@ -118,6 +118,7 @@ struct meq_state {
   int* d_err = nullptr;
   int* d_flag = nullptr;
   int* d_nonfinite = nullptr;  // 1 + first entry with a non-finite momentum norm, 0 if none
+  int* d_sched = nullptr;      // NS GEMM tile queue (two ints, zero between launches)
   int64_t step_bytes = 0;
   std::vector<char> step_host;
   // launch plan
@@ -318,7 +319,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
   *off_stats = L->add(int64_t(n) * sizeof(MatStats) + int64_t(n) * 2 * 8);  // stats, then direction counts
   st->step_bytes = sizeof(StepScalars) + 2 * int64_t(n) * sizeof(void*);
   *off_step = L->add(st->step_bytes);
-  *off_err = L->add(64);
+  *off_err = L->add(64);  // ints 0: error word, 4: self-test flag, 8: non-finite flag, 12-13: tile queue
   *off_mats = L->add(int64_t(n) * sizeof(MatInfo));
   *off_groups = L->add(int64_t(st->groups.size()) * sizeof(GroupInfo));
   group_offs->clear();
@@ -407,6 +408,7 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
         P.idesc = make_idesc(in16, P.b_mn_major, tile_m);
         P.ca = st->opt.ns_a, P.cb = st->opt.ns_b, P.cc = st->opt.ns_c;
         P.err = st->d_err;
+        P.sched = st->d_sched;
         P.timeout_ns = static_cast<unsigned long long>(static_cast<double>(st->opt.wait_timeout_ms) * 1e6);
         int tiles = 0;
         P.ngroups = std::min(kMaxGroups, ng - g0);
@@ -621,6 +623,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   st->d_err = reinterpret_cast<int*>(A + off_err);
   st->d_flag = st->d_err + 4;
   st->d_nonfinite = st->d_err + 8;
+  st->d_sched = st->d_err + 12;
   st->d_mats = reinterpret_cast<MatInfo*>(A + off_mats);
   st->d_groups = reinterpret_cast<GroupInfo*>(A + off_groups);
   for (size_t g = 0; g < st->groups.size(); ++g) {
@@ -856,8 +859,10 @@ meq_status meq_sync(meq_state* st) {
   e = cudaMemcpy(&err, st->d_err, sizeof(int), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_fail(st, e, "reading the device error word");
   if (err != 0) {
-    int zero = 0;
-    cudaMemcpy(st->d_err, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    int zero[2] = {0, 0};
+    cudaMemcpy(st->d_err, zero, sizeof(int), cudaMemcpyHostToDevice);
+    // a launch that returned early may have left its tile queue partly used
+    cudaMemcpy(st->d_sched, zero, 2 * sizeof(int), cudaMemcpyHostToDevice);
     char buf[96];
     std::snprintf(buf, sizeof(buf), "device-side bounded wait expired (code 0x%x)", err);
     return fail(st, MEQ_ERR_TIMEOUT, buf);

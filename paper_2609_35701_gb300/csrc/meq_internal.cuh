@@ -20,6 +20,8 @@ enum DevErr : int {
   DEV_TIMEOUT_MMA_TMEM = 0x103,  // MMA warp waited too long for a free accumulator
   DEV_TIMEOUT_EPI = 0x104,       // epilogue waited too long for an accumulator
   DEV_TIMEOUT_DRAIN = 0x105,     // waiting for in-flight copies / MMAs at exit
+  DEV_TIMEOUT_SCHED_PUT = 0x106, // tile scheduler waited too long for a free slot of the tile ring
+  DEV_TIMEOUT_SCHED_TAKE = 0x107,// a role waited too long for its next tile index
   DEV_TIMEOUT_TEST = 0x1FF,      // the wait-timeout self test
 };
 
@@ -110,6 +112,8 @@ struct GemmParams {
   int32_t reverse;         // 1: tiles are taken in reverse order (alternates between launches)
   float ca, cb, cc;        // NS coefficients
   int* err;                // device error word
+  int* sched;              // tile queue: [0] tiles handed out beyond the first wave, [1] units done;
+                           // zero between launches (the last unit to finish resets both)
   unsigned long long timeout_ns;
 };
 

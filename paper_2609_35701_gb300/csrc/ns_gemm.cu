@@ -29,6 +29,11 @@
 //               every other 32-column chunk (two warps per lane quarter, so
 //               each SM sub-partition can hide one warp's latencies behind
 //               the other's work)
+// Tiles are handed out dynamically: each unit (CTA or CTA pair) starts on
+// its own index and then draws from an atomic counter, and the leader's
+// producer passes every index to the other roles through a ring in shared
+// memory, so a launch ends within about one tile on every unit whatever the
+// mix of tile sizes and SM speeds.
 // Two 128x256 fp32 accumulators (512 TMEM columns) let the epilogue of one
 // tile overlap the MMAs of the next. The epilogue stages 32 x 32 blocks in
 // swizzled shared memory and writes them with coalesced 16-byte stores (the
@@ -49,6 +54,7 @@ constexpr int NUM_EPI_WARPS = 8;                     // two per TMEM lane quarte
 constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int SLOT_BYTES = 2048;                     // one 32 x 32 16-bit block
+constexpr int SCHED_D = 16;                          // entries of the tile-index ring
 constexpr float kUInvScale2 = 1.0f / (kUScale * kUScale);  // exact: kUScale is a power of two
 
 // kPair = 1: one CTA computes a 128 x 256 tile (tcgen05 cta_group::1).
@@ -63,10 +69,12 @@ struct Cfg {
   static constexpr int B_BYTES = BN_LOCAL * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int STAGES = kPair == 1 ? 4 : 6;
-  static constexpr int NUM_BARS = 2 * STAGES + 4 + 1;  // full, empty, tmem full x2, tmem empty x2, drain
+  // full, empty, tmem full x2, tmem empty x2, drain, tile ring full / empty
+  static constexpr int NUM_BARS = 2 * STAGES + 4 + 1 + 2 * SCHED_D;
   static constexpr int SMEM_EPI_OFF = STAGES * STAGE_BYTES;
   static constexpr int SMEM_BAR_OFF = SMEM_EPI_OFF + NUM_EPI_WARPS * SLOT_BYTES;
-  static constexpr int SMEM_BYTES = SMEM_BAR_OFF + NUM_BARS * 8 + 16 + 1024;
+  // barriers, the TMEM address word (16 bytes reserved), the tile ring
+  static constexpr int SMEM_BYTES = SMEM_BAR_OFF + NUM_BARS * 8 + 16 + 4 * SCHED_D + 1024;
   static_assert(SMEM_BYTES <= 232448, "shared memory budget of one sm_103a CTA");
 };
 
@@ -172,6 +180,28 @@ __device__ __forceinline__ void cluster_sync_all() {
 // the cluster, which the MMA issuer does not need.
 __device__ __forceinline__ void mbar_arrive_relaxed_cluster(uint32_t bar_cluster) {
   asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+// Writes a 32-bit value into the peer CTA's shared memory and completes it
+// as a 4-byte transaction on the peer's barrier, which this call also arms
+// (one arrival). A waiter on that barrier then sees the value, as after a TMA
+// load; no fence of the writer's other memory operations is involved.
+__device__ __forceinline__ void st_async_peer_u32(uint32_t addr_cluster, uint32_t bar_cluster, uint32_t v) {
+  asm volatile("mbarrier.arrive.expect_tx.relaxed.cluster.shared::cluster.b64 _, [%0], 4;" ::"r"(bar_cluster)
+               : "memory");
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.u32 [%0], %1, [%2];" ::"r"(addr_cluster), "r"(v),
+               "r"(bar_cluster)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_local(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void st_shared_u32(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t ld_shared_u32(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+  return v;
 }
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* tm) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
@@ -374,6 +404,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
 #define EMPTY_BAR(s) (bar0 + 8u * (STAGES + (s)))
 #define TFULL_BAR(a) (bar0 + 8u * (2 * STAGES + (a)))
 #define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
+#define SFULL_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + (i)))
+#define SEMPTY_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + SCHED_D + (i)))
+  const uint32_t ring = tmem_slot + 16;  // SCHED_D tile indices
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -395,6 +428,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       mbar_init(TEMPTY_BAR(a), kPair * NUM_EPI_WARPS);
     }
     mbar_init(drain_bar, 1);
+    for (int i = 0; i < SCHED_D; ++i) {
+      mbar_init(SFULL_BAR(i), 1);
+      // consumers of each index: the MMA issuer and the epilogue warps of the
+      // leader, and (pair) the peer's producer and epilogue warps
+      mbar_init(SEMPTY_BAR(i), kPair * (1 + NUM_EPI_WARPS));
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     for (int g = 0; g < p.ngroups; ++g) {
       prefetch_tmap(&p.g[g].tmA);
@@ -420,6 +459,37 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
   pdl_allow_dependents();
   pdl_wait_predecessor();  // operands come from the previous kernel of the step
 
+  // ------------------------------------------------------------------ tile queue
+  // Each unit (CTA pair) starts on tile `unit`; further tiles are handed out
+  // by the launch's atomic counter, so units that finish early take more and
+  // the launch ends within about one tile on every unit. The leader's
+  // producer fetches each index and publishes it in the tile ring of both
+  // CTAs (the peer's copy by st.async, which completes on the peer's barrier
+  // like a TMA load, so the producer never waits on a memory fence); every
+  // other role reads the ring in the same order. A reader hands its slot
+  // back with a relaxed arrive (a release would first wait for the
+  // epilogue's outstanding global stores). Its read has completed long
+  // before the slot can be written again: the producer writes index n + 16
+  // only after loading tile n + 15, by which time every role has used index
+  // n (the epilogue warps to release tile n's accumulator, the peer's
+  // producer to load its half of tile n) -- the operand ring holds at most
+  // 6 k-blocks and the accumulators 2 tiles.
+  auto sched_put = [&](int n, int t) -> bool {
+    const int i = n & (SCHED_D - 1);
+    if (!wait_bounded(SEMPTY_BAR(i), ((n / SCHED_D) & 1) ^ 1u, err, DEV_TIMEOUT_SCHED_PUT, tmo)) return false;
+    if (kPair == 2) st_async_peer_u32(map_to_rank(ring + 4u * i, 1), map_to_rank(SFULL_BAR(i), 1), static_cast<uint32_t>(t));
+    st_shared_u32(ring + 4u * i, static_cast<uint32_t>(t));
+    mbar_arrive_local(SFULL_BAR(i));  // release (CTA scope) of the store above
+    return true;
+  };
+  auto sched_take = [&](int n, int& t) -> bool {
+    const int i = n & (SCHED_D - 1);
+    if (!wait_bounded(SFULL_BAR(i), (n / SCHED_D) & 1, err, DEV_TIMEOUT_SCHED_TAKE, tmo)) return false;
+    t = static_cast<int>(ld_shared_u32(ring + 4u * i));
+    mbar_arrive_relaxed_cluster((kPair == 2 && !leader) ? map_to_rank(SEMPTY_BAR(i), 0) : SEMPTY_BAR(i));
+    return true;
+  };
+
   if (warp == 0) {
     if (lane == 0) {
       // ---------------------------------------------------------------- TMA producer
@@ -427,7 +497,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       uint32_t phase = 0;
       uint32_t issued_mask = 0, issued_parity = 0;  // bit s: stage s was filled / parity of its last fill
       bool ok = true;
-      for (int t = unit; ok && t < p.total_tiles; t += nunits) {
+      int t = unit;
+      int fetched = 0;  // leader: the counter value for the next tile
+      for (int n = 0; ok; ++n) {
+        if (n > 0 && leader) t = nunits + fetched;
+        if (leader ? !sched_put(n, t) : !sched_take(n, t)) break;
+        if (t >= p.total_tiles) break;
+        // The next index is fetched while this tile's operands are requested;
+        // its value is first read at the top of the next iteration.
+        if (leader) fetched = atomicAdd(p.sched, 1);
         const TileCoord c = decode_tile<kPair>(p, t);
         const GemmGroup& G = p.g[c.g];
         const int nk = (G.K + BK - 1) / BK;
@@ -489,7 +567,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       uint32_t acc_phase = 0;
       bool ok = true;
       const uint32_t b_lbo = p.b_mn_major ? (64u * BK * 2u) : 16u;
-      for (int t = unit; ok && t < p.total_tiles; t += nunits) {
+      for (int n = 0; ok; ++n) {
+        int t = 0;
+        if (!sched_take(n, t) || t >= p.total_tiles) break;
         const TileCoord c = decode_tile<kPair>(p, t);
         const int nk = (p.g[c.g].K + BK - 1) / BK;
         if (!wait_bounded(TEMPTY_BAR(acc), acc_phase ^ 1u, err, DEV_TIMEOUT_MMA_TMEM, tmo)) break;
@@ -548,7 +628,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     // The leader's tmem-empty barrier counts the epilogue warps of both CTAs.
     const uint32_t tempty_target0 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(0), 0) : TEMPTY_BAR(0);
     const uint32_t tempty_target1 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(1), 0) : TEMPTY_BAR(1);
-    for (int t = unit; t < p.total_tiles; t += nunits) {
+    for (int n = 0;; ++n) {
+      int t = 0, got = 1;
+      if (lane == 0) got = sched_take(n, t) ? 1 : 0;
+      got = __shfl_sync(0xffffffffu, got, 0);
+      t = __shfl_sync(0xffffffffu, t, 0);
+      if (!got || t >= p.total_tiles) break;
       const TileCoord c = decode_tile<kPair>(p, t);
       const GemmGroup& G = p.g[c.g];
       if (!wait_bounded_warp(TFULL_BAR(acc), acc_phase, err, DEV_TIMEOUT_EPI, tmo)) break;
@@ -686,6 +771,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
 #undef EMPTY_BAR
 #undef TFULL_BAR
 #undef TEMPTY_BAR
+#undef SFULL_BAR
+#undef SEMPTY_BAR
 
   if (kPair == 2 && *reinterpret_cast<volatile int*>(err) != 0) {
     // After an early exit, give copies still in flight towards either CTA
@@ -698,6 +785,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
   __syncthreads();
   if (kPair == 2) cluster_sync_all();  // no CTA leaves while its peer may still signal it
   tc_fence_after();
+  if (threadIdx.x == 0 && leader) {
+    // The last unit to finish resets the tile queue. Every unit's fetches
+    // precede its count here, and the next launch reads the queue only after
+    // this grid has completed.
+    __threadfence();
+    if (atomicAdd(p.sched + 1, 1) == nunits - 1) {
+      p.sched[0] = 0;
+      p.sched[1] = 0;
+    }
+  }
   if (warp == 1) {
     if (kPair == 2)
       asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS) : "memory");
