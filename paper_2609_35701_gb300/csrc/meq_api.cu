@@ -362,6 +362,7 @@ bool encode_map(CUtensorMap* m, void* base, int elem_bytes, int64_t inner, int64
   return r == CUDA_SUCCESS;
 }
 constexpr CUtensorMapSwizzle SW128 = CU_TENSOR_MAP_SWIZZLE_128B;
+constexpr CUtensorMapSwizzle SW64 = CU_TENSOR_MAP_SWIZZLE_64B;
 
 // Tiles (tile_m rows x 256 columns) holding a 32 x 32 block on or above the diagonal.
 int sym_tiles(int tiles_m, int tiles_n, int tile_m) {
@@ -422,13 +423,13 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
           Q.trans = G.trans;
           bool ok = true;
           const int64_t x_ld = G.lp * 2, x_ms = G.s * G.lp * 2;   // 16-bit X buffers, bytes
-          const int64_t s_ld = G.sp * 2, s_ms = G.s * G.sp * 2;   // 16-bit A / P buffers, bytes
+          const int64_t s_ld = G.sp * 2, s_ms = G.s * G.sp * 2;   // 16-bit A buffer, bytes
           if (mode == MODE_GRAM) {
             Q.M = (int32_t)G.s, Q.N = (int32_t)G.s, Q.K = (int32_t)G.l;
             Q.sym = 1;
             ok &= encode_map(&Q.tmA, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 128, SW128);
             ok &= encode_map(&Q.tmB, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, b_rows, SW128);
-            Q.out = G.a16, Q.out_ld = s_ld, Q.out_mstride = s_ms;
+            ok &= encode_map(&Q.tmO, G.a16, 2, G.s, G.s, G.count, G.sp, 32, 32, SW64);
             Q.scale = 1.0f / (ak * ak);
             if (per_matrix) Q.minv = st->d_ginv + G.mbase, Q.minv_pow = 2;
             Q.out_fp16 = dA(k);
@@ -437,7 +438,7 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             Q.sym = 1;
             ok &= encode_map(&Q.tmA, G.a16, 2, G.s, G.s, G.count, G.sp, 64, 128, SW128);
             ok &= encode_map(&Q.tmB, G.a16, 2, G.s, G.s, G.count, G.sp, 64, b_rows, SW128);
-            Q.out = G.p16, Q.out_ld = s_ld, Q.out_mstride = s_ms;
+            ok &= encode_map(&Q.tmO, G.p16, 2, G.s, G.s, G.count, G.sp, 32, 32, SW64);
             Q.aux = G.a16, Q.aux_ld = s_ld, Q.aux_mstride = s_ms;
             Q.scale = 1.0f;
             Q.out_fp16 = dX(k);

@@ -80,6 +80,8 @@ enum GemmMode : int { MODE_GRAM = 0, MODE_POLY = 1, MODE_XUPD = 2, MODE_XLAST = 
 struct GemmGroup {
   CUtensorMap tmA;        // A operand (K-major), box {64, 128, 1}
   CUtensorMap tmB;        // B operand: K-major box {64, 256, 1} or MN-major box {64, 64, 1}
+  CUtensorMap tmO;        // GRAM / POLY: the 16-bit symmetric output (A or P) for TMA stores,
+                          // box {32, 32, 1}, 64-byte swizzle (the epilogue's staging layout)
   int32_t M, N, K;        // output rows, output cols, contraction
   int32_t count;          // matrices in the group
   int32_t tiles_m, tiles_n;
@@ -92,9 +94,9 @@ struct GemmGroup {
   int32_t minv_pow;       // epilogue scale *= minv^minv_pow (0, 1 or 2)
   int32_t out_fp16;       // 16-bit format of the output (1 = fp16, 0 = bf16)
   int32_t aux_fp16;       // POLY: 16-bit format of the A it reads in the epilogue
-  void* out;              // GRAM: 16-bit A; POLY: 16-bit P; XUPD: 16-bit X next; XLAST: fp32 U (weight layout)
-  int64_t out_ld;         // output row stride in bytes
-  int64_t out_mstride;    // output matrix stride in bytes
+  void* out;              // XUPD: 16-bit X next; XLAST: fp16(kUScale U) in the weight's layout
+  int64_t out_ld;         // XUPD / XLAST: output row stride in bytes
+  int64_t out_mstride;    // XUPD / XLAST: output matrix stride in bytes
   const void* aux;        // POLY: 16-bit A
   int64_t aux_ld;         // bytes
   int64_t aux_mstride;    // bytes

@@ -36,8 +36,9 @@
 // mix of tile sizes and SM speeds.
 // Two 128x256 fp32 accumulators (512 TMEM columns) let the epilogue of one
 // tile overlap the MMAs of the next. The epilogue stages 32 x 32 blocks in
-// swizzled shared memory and writes them with coalesced 16-byte stores (the
-// SM's TMA unit stays free for the operand loads).
+// swizzled shared memory; the symmetric A and P (each block stored twice)
+// leave by TMA stores, X and U by coalesced 16-byte stores from the threads
+// (the update launches keep the SM's TMA unit for their operand loads).
 //
 // Every mbarrier wait is bounded (time and iteration count). On expiry the
 // waiting role records an error code, the others see it and stop, in-flight
@@ -53,7 +54,7 @@ constexpr int A_BYTES = BM * BK * 2;                 // 16 KB
 constexpr int NUM_EPI_WARPS = 8;                     // two per TMEM lane quarter
 constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
 constexpr uint32_t TMEM_COLS = 512;
-constexpr int SLOT_BYTES = 2048;                     // one 32 x 32 16-bit block
+constexpr int SLOT_BYTES = 2048;                     // one 32 x 32 16-bit block (two per epilogue warp)
 constexpr int SCHED_D = 16;                          // entries of the tile-index ring
 constexpr float kUInvScale2 = 1.0f / (kUScale * kUScale);  // exact: kUScale is a power of two
 
@@ -72,7 +73,7 @@ struct Cfg {
   // full, empty, tmem full x2, tmem empty x2, drain, tile ring full / empty
   static constexpr int NUM_BARS = 2 * STAGES + 4 + 1 + 2 * SCHED_D;
   static constexpr int SMEM_EPI_OFF = STAGES * STAGE_BYTES;
-  static constexpr int SMEM_BAR_OFF = SMEM_EPI_OFF + NUM_EPI_WARPS * SLOT_BYTES;
+  static constexpr int SMEM_BAR_OFF = SMEM_EPI_OFF + NUM_EPI_WARPS * 2 * SLOT_BYTES;
   // barriers, the TMEM address word (16 bytes reserved), the tile ring
   static constexpr int SMEM_BYTES = SMEM_BAR_OFF + NUM_BARS * 8 + 16 + 4 * SCHED_D + 1024;
   static_assert(SMEM_BYTES <= 232448, "shared memory budget of one sm_103a CTA");
@@ -351,8 +352,8 @@ __device__ __forceinline__ void fill_half_rows(uint8_t* slot, int r, const float
 // ldmatrix .trans reads each 8 x 8 sub-block (g, q) as its transpose and
 // stmatrix writes it back as sub-block (q, g). All reads finish before the
 // first write (the warp holds the whole block in registers in between).
-__device__ __forceinline__ void transpose_slot(uint8_t* slot, int lane) {
-  const uint32_t base = smem_u32(slot);
+__device__ __forceinline__ void transpose_slot(const uint8_t* src, uint8_t* dst, int lane) {
+  const uint32_t base = smem_u32(src), dbase = smem_u32(dst);
   const int r8 = lane & 7, q = lane >> 3;
   uint32_t f[4][4];
 #pragma unroll
@@ -364,18 +365,17 @@ __device__ __forceinline__ void transpose_slot(uint8_t* slot, int lane) {
                  : "r"(addr)
                  : "memory");
   }
-  __syncwarp();
 #pragma unroll
   for (int g = 0; g < 4; ++g) {
     const int row = 8 * q + r8;  // the transpose of sub-block (g, q) is sub-block (q, g)
-    const uint32_t addr = base + row * 64 + ((g ^ ((row >> 1) & 3)) << 4);
+    const uint32_t addr = dbase + row * 64 + ((g ^ ((row >> 1) & 3)) << 4);
     asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(f[g][0]),
                  "r"(f[g][1]), "r"(f[g][2]), "r"(f[g][3])
                  : "memory");
   }
 }
-// 32 rows x 64 bytes (a 16-bit 32 x 32 block) -> global: rows
-// r < rows_valid, 16-byte chunks k < chunks_valid of each row.
+// 32 rows x 64 bytes (a staged 16-bit 32 x 32 block) -> global with 16-byte
+// stores: rows r < rows_valid, 16-byte chunks k < chunks_valid of each row.
 __device__ __forceinline__ void store_block64(const uint8_t* slot, int lane, uint8_t* dst, int64_t ld_bytes,
                                               int rows_valid, int chunks_valid) {
   const int k = lane & 3;
@@ -386,6 +386,22 @@ __device__ __forceinline__ void store_block64(const uint8_t* slot, int lane, uin
     if (r < rows_valid && k < chunks_valid) *reinterpret_cast<uint4*>(dst + r * ld_bytes + k * 16) = w;
   }
 }
+// A staged 32 x 32 16-bit block -> global by TMA (tensor map box {32, 32, 1},
+// 64-byte swizzle = the staging layout). Rows and columns outside the
+// tensor's extent are not written. The writing threads make their
+// shared-memory stores visible to the TMA unit first (fence.proxy.async).
+__device__ __forceinline__ void tma_store_block(const CUtensorMap* tm, const uint8_t* src, int x, int y, int z) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(tm)),
+               "r"(smem_u32(src)), "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// The shared-memory reads of every committed store have completed.
+__device__ __forceinline__ void bulk_wait_reads() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// Every committed store has completed.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 template <int kPair>
 __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_constant__ GemmParams p) {
   using C_ = Cfg<kPair>;
@@ -438,6 +454,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     for (int g = 0; g < p.ngroups; ++g) {
       prefetch_tmap(&p.g[g].tmA);
       prefetch_tmap(&p.g[g].tmB);
+      if (p.g[g].sym) prefetch_tmap(&p.g[g].tmO);
     }
   }
   if (warp == 1) {
@@ -613,14 +630,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
   } else {
     // ------------------------------------------------------------------ epilogue
     // Warp ew (0..7) owns TMEM lanes 32*q .. +31 (q = warp % 4), i.e. rows
-    // 32q .. 32q+31 of the tile, chunks ch with ch % 2 == half, and one 2 KB
-    // shared-memory slot, used in turn for the polynomial's A block (which is
-    // prefetched into registers one chunk ahead), the block as computed and
-    // its transpose (symmetric outputs).
+    // 32q .. 32q+31 of the tile, chunks ch with ch % 2 == half, and two 2 KB
+    // shared-memory slots: `slot` takes the polynomial's A block (prefetched
+    // into registers one chunk ahead) and then the block as computed, `slot_t`
+    // its transpose (mirrored blocks, transposed U). The symmetric outputs
+    // (A, P: twice the stores, with the mirrors) leave by TMA stores, and a
+    // slot is rewritten only after the stores of the previous chunk have read
+    // it; X and U leave by 16-byte stores from the threads, which keeps the
+    // TMA unit free for the operand loads of the longer update launches.
     const int q = warp & 3;
     const int ew = warp - 2;
     const int half = ew >> 2;
-    uint8_t* slot = gbase + C_::SMEM_EPI_OFF + ew * SLOT_BYTES;
+    uint8_t* slot = gbase + C_::SMEM_EPI_OFF + ew * (2 * SLOT_BYTES);
+    uint8_t* slot_t = slot + SLOT_BYTES;
     const int mode = p.mode;
     int acc = 0;
     uint32_t acc_phase = 0;
@@ -666,6 +688,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
         const int C = c.tn * 8 + ch;
         float v[32];
         tmem_ld_32cols(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN + ch * 32), v);
+        if (G.sym) {
+          if (lane == 0) bulk_wait_reads();  // both slots free
+        }
+        __syncwarp();
         if (mode == MODE_POLY) {
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
@@ -726,35 +752,40 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
             G.cpart[(static_cast<int64_t>(c.mat) * ((G.M + 31) / 32) + R) * G.N + col0 + lane] = sq[0] * kUInvScale2;
           // 8-element chunks that start below the row length stay inside the
           // padded row (stride = row length rounded up to 8)
+          fill_half_rows(slot, lane, v, 1);
+          __syncwarp();
           if (!G.trans) {
             // U rows = NS rows row0 + r, U columns = NS columns col0 + j
-            fill_half_rows(slot, lane, v, 1);
-            __syncwarp();
             store_block64(slot, lane, outm + static_cast<int64_t>(row0) * G.out_ld + col0 * 2, G.out_ld, rows_valid,
                           min(4, (G.N - col0 + 7) / 8));
           } else {
             // U rows = NS columns col0 + j, U columns = NS rows row0 + r
-            fill_half_rows(slot, lane, v, 1);
+            transpose_slot(slot, slot_t, lane);
             __syncwarp();
-            transpose_slot(slot, lane);
-            __syncwarp();
-            store_block64(slot, lane, outm + static_cast<int64_t>(col0) * G.out_ld + row0 * 2, G.out_ld,
+            store_block64(slot_t, lane, outm + static_cast<int64_t>(col0) * G.out_ld + row0 * 2, G.out_ld,
                           min(32, G.N - col0), min(4, (G.M - row0 + 7) / 8));
           }
-        } else {
-          // 16-bit rows are padded to a multiple of 64 elements: whole 32-column blocks stay inside them
+        } else if (!G.sym) {
+          // X rows are padded to a multiple of 64 elements: whole 32-column blocks stay inside them
           fill_half_rows(slot, lane, v, G.out_fp16);
           __syncwarp();
           store_block64(slot, lane, outm + static_cast<int64_t>(row0) * G.out_ld + col0 * 2, G.out_ld, rows_valid, 4);
-          if (G.sym && C > R) {
+        } else {
+          fill_half_rows(slot, lane, v, G.out_fp16);
+          const bool mirror = G.sym && C > R;  // strictly above the diagonal: also store the transpose
+          if (mirror) {
             __syncwarp();
-            transpose_slot(slot, lane);
-            __syncwarp();
-            store_block64(slot, lane, outm + static_cast<int64_t>(col0) * G.out_ld + row0 * 2, G.out_ld,
-                          min(32, G.M - col0), 4);
+            transpose_slot(slot, slot_t, lane);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_block(&G.tmO, slot, col0, row0, c.mat);
+            if (mirror) tma_store_block(&G.tmO, slot_t, row0, col0, c.mat);
+            bulk_commit();
           }
         }
-        __syncwarp();  // slots free again; reconverge before the next warp-wide tcgen05.ld
+        __syncwarp();  // reconverge before the next warp-wide tcgen05.ld
       }
       if (mode == MODE_XLAST && row0 < G.M && row0 + lane < G.M)  // one partial per (tile column, half)
         G.rpart[(static_cast<int64_t>(c.mat) * G.tiles_n * 2 + c.tn * 2 + half) * G.M + row0 + lane] = rsum * kUInvScale2;
@@ -766,6 +797,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
     }
+    // The outputs are in global memory before the CTA leaves.
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
   }
 #undef FULL_BAR
 #undef EMPTY_BAR
