@@ -76,6 +76,13 @@ typedef struct {
   int update_rule;        /* meq_update_rule; default MEQ_RULE_MEQMUON */
   int debug_canaries;     /* 1: guard bands of a fixed byte pattern surround every workspace
                              buffer (meq_check_canaries); default 0 */
+  int ns_single_launch;   /* 1: all 3K products of Eq. (5) run in one cooperative launch of
+                             CTA pairs, each tile waiting (bounded) until the previous product
+                             of its matrix is complete; used when ns_cta_pair = 1 and the
+                             shape groups x 3K fit 48 segments (with at most 8 groups),
+                             else the step keeps one launch per product
+                             (meq_ns_gemm_launches_per_step tells which). 0 (default): one
+                             launch per product. */
 } meq_options;
 
 /* Update applied to the hidden 2D weights after momentum and Newton-Schulz. */

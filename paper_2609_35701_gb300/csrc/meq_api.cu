@@ -124,6 +124,10 @@ struct meq_state {
   // launch plan
   std::vector<GemmParams> gemm;  // in launch order
   std::vector<int> gemm_grid;
+  PersistParams persist;       // the one-launch NS (ns_single_launch), when it fits
+  int persist_grid = 0;
+  bool use_persist = false;
+  int* d_done = nullptr;       // its completion counters, [3K][n_hidden]
   LaunchCtx ctx{};
   bool graph_ready = false;
   cudaGraph_t graph = nullptr;
@@ -169,6 +173,7 @@ bool valid_options(const meq_options& o, std::string* why) {
   if (o.ns_cta_pair != 0 && o.ns_cta_pair != 1) { *why = "ns_cta_pair must be 0 or 1"; return false; }
   if (o.ns_x0_fused != 0 && o.ns_x0_fused != 1) { *why = "ns_x0_fused must be 0 or 1"; return false; }
   if (o.debug_canaries != 0 && o.debug_canaries != 1) { *why = "debug_canaries must be 0 or 1"; return false; }
+  if (o.ns_single_launch != 0 && o.ns_single_launch != 1) { *why = "ns_single_launch must be 0 or 1"; return false; }
   if (o.update_rule != MEQ_RULE_MEQMUON && o.update_rule != MEQ_RULE_MUON) {
     *why = "update_rule must be MEQ_RULE_MEQMUON or MEQ_RULE_MUON";
     return false;
@@ -314,7 +319,8 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
   *off_vec4 = L->add(vec * 4 * 4);  // r, c, s, t
   *off_cpart = L->add(parts * 4);
   *off_partials = L->add(std::max({hchunks, tiles, xblks}) * 4);  // per momentum chunk or block
-  *off_counters = L->add(int64_t(n) * 4);
+  // per-matrix counters, then the one-launch NS completion counters [3K][n_hidden]
+  *off_counters = L->add(int64_t(n) * 4 + int64_t(3) * st->opt.ns_steps * st->n_hidden * 4);
   *off_x0s = L->add(int64_t(n) * 4 * 2);  // x0scale (cast pass) and the inverse norms (fused)
   *off_stats = L->add(int64_t(n) * sizeof(MatStats) + int64_t(n) * 2 * 8);  // stats, then direction counts
   st->step_bytes = sizeof(StepScalars) + 2 * int64_t(n) * sizeof(void*);
@@ -404,9 +410,8 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
       for (int g0 = 0; g0 < ng; g0 += kMaxGroups) {
         GemmParams P;
         std::memset(&P, 0, sizeof(P));
-        P.mode = real_mode;
-        P.b_mn_major = (mode == MODE_XUPD) ? 1 : 0;
-        P.idesc = make_idesc(in16, P.b_mn_major, tile_m);
+        const int b_mn_major = (mode == MODE_XUPD) ? 1 : 0;
+        const uint32_t idesc = make_idesc(in16, b_mn_major, tile_m);
         P.ca = st->opt.ns_a, P.cb = st->opt.ns_b, P.cc = st->opt.ns_c;
         P.err = st->d_err;
         P.sched = st->d_sched;
@@ -416,6 +421,8 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
         for (int gi = 0; gi < P.ngroups; ++gi) {
           Group& G = st->groups[g0 + gi];
           GemmGroup& Q = P.g[gi];
+          Q.mode = real_mode, Q.idesc = idesc, Q.b_mn_major = b_mn_major;
+          Q.mat_base = static_cast<int32_t>(G.mbase);
           // storage scale of X_k; a fused X_0 is unscaled and its 1/||H||_F is applied per matrix
           const float ak = (k == 0) ? (fused ? 1.0f : G.alpha0) : G.alpha;
           const bool per_matrix = fused && k == 0;
@@ -430,6 +437,7 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             ok &= encode_map(&Q.tmA, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 128, SW128);
             ok &= encode_map(&Q.tmB, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, b_rows, SW128);
             ok &= encode_map(&Q.tmO, G.a16, 2, G.s, G.s, G.count, G.sp, 32, 32, SW64);
+            Q.tma_out = 1;
             Q.scale = 1.0f / (ak * ak);
             if (per_matrix) Q.minv = st->d_ginv + G.mbase, Q.minv_pow = 2;
             Q.out_fp16 = dA(k);
@@ -439,6 +447,7 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             ok &= encode_map(&Q.tmA, G.a16, 2, G.s, G.s, G.count, G.sp, 64, 128, SW128);
             ok &= encode_map(&Q.tmB, G.a16, 2, G.s, G.s, G.count, G.sp, 64, b_rows, SW128);
             ok &= encode_map(&Q.tmO, G.p16, 2, G.s, G.s, G.count, G.sp, 32, 32, SW64);
+            Q.tma_out = 1;
             Q.aux = G.a16, Q.aux_ld = s_ld, Q.aux_mstride = s_ms;
             Q.scale = 1.0f;
             Q.out_fp16 = dX(k);
@@ -450,6 +459,8 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             ok &= encode_map(&Q.tmB, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 64, SW128);
             if (real_mode == MODE_XUPD) {
               Q.out = G.x[nxt], Q.out_ld = x_ld, Q.out_mstride = x_ms;
+              // thread stores here; the one-launch NS switches to this map (below)
+              ok &= encode_map(&Q.tmO, G.x[nxt], 2, G.l, G.s, G.count, G.lp, 32, 32, SW64);
               Q.scale = G.alpha / ak;
               if (per_matrix) Q.minv = st->d_ginv + G.mbase, Q.minv_pow = 1;
               Q.out_fp16 = dX(k + 1);
@@ -482,6 +493,48 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
       }
     }
   }
+  // ns_single_launch: the per-product launches' groups become the segments of
+  // one tile queue in product order; a tile of product j waits until every
+  // epilogue warp of every tile of its matrix in product j - 1 has counted.
+  st->use_persist = false;
+  const int nprod = 3 * K;
+  if (st->opt.ns_single_launch && pair == 2 && ng <= kMaxGroups && static_cast<int>(st->gemm.size()) == nprod &&
+      nprod * ng <= kMaxSegs) {
+    const int max_pairs = ns_gemm_persistent_max_pairs();
+    if (max_pairs > 0) {
+      PersistParams& Q = st->persist;
+      std::memset(&Q, 0, sizeof(Q));
+      int tiles = 0, nseg = 0;
+      for (int j = 0; j < nprod; ++j) {
+        const GemmParams& P = st->gemm[j];
+        for (int gi = 0; gi < P.ngroups; ++gi) {
+          GemmGroup S = P.g[gi];
+          S.tile_begin = tiles;
+          S.prod = j;
+          S.dep_target = j == 0 ? 0 : st->gemm[j - 1].g[gi].tiles_per_mat * pair * kNsEpilogueWarps;
+          // every output another tile waits for leaves by TMA stores, whose
+          // completion a warp can wait for without waiting for later stores
+          if (S.mode == MODE_XUPD) S.tma_out = 1;
+          tiles += S.tiles_per_mat * S.count;
+          Q.g[nseg++] = S;
+        }
+      }
+      const GemmParams& P0 = st->gemm[0];
+      Q.ngroups = nseg;
+      Q.total_tiles = tiles;
+      Q.reverse = 0;
+      Q.persistent = 1;
+      Q.ca = P0.ca, Q.cb = P0.cb, Q.cc = P0.cc;
+      Q.err = st->d_err;
+      Q.sched = st->d_sched;
+      Q.done = st->d_done;
+      Q.nslots = static_cast<int32_t>(st->n_hidden);
+      Q.nprod = nprod;
+      Q.timeout_ns = P0.timeout_ns;
+      st->persist_grid = pair * std::max(1, std::min({tiles, st->num_sms / pair, max_pairs}));
+      st->use_persist = true;
+    }
+  }
   return true;
 }
 
@@ -506,6 +559,7 @@ void meq_default_options(meq_options* o) {
   o->ns_cta_pair = 1;
   o->ns_x0_fused = 1;
   o->debug_canaries = 0;
+  o->ns_single_launch = 0;
 }
 
 const char* meq_status_string(meq_status s) {
@@ -616,6 +670,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   st->d_parts = reinterpret_cast<float*>(A + off_cpart);
   st->d_partials = reinterpret_cast<float*>(A + off_partials);
   st->d_counters = reinterpret_cast<unsigned int*>(A + off_counters);
+  st->d_done = reinterpret_cast<int*>(st->d_counters + n);
   st->d_x0scale = reinterpret_cast<float*>(A + off_x0s);
   st->d_ginv = st->d_x0scale + n;
   st->d_stats = reinterpret_cast<MatStats*>(A + off_stats);
@@ -692,7 +747,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   C.total_rblks = st->total_rblks;
   C.total_slabs = st->total_slabs;
   st->kernels_per_step = (st->n_hidden ? 2 : 0) + (st->n_rows ? 1 : 0) + (st->n_two ? 1 : 0) + 2 +
-                         static_cast<int>(st->gemm.size());
+                         (st->use_persist ? 1 : static_cast<int>(st->gemm.size()));
   st->step_host.assign(static_cast<size_t>(st->step_bytes), 0);
   st->last_stream = s;
   *out = st;
@@ -753,9 +808,14 @@ static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev
     if (e != cudaSuccess) return cuda_fail(st, e, "cast_x0 launch");
   }
   mark(2);
-  for (size_t i = 0; i < st->gemm.size(); ++i) {
-    e = launch_ns_gemm(st->gemm[i], st->gemm_grid[i], st->opt.ns_cta_pair ? 2 : 1, s);
-    if (e != cudaSuccess) return cuda_fail(st, e, "ns_gemm launch");
+  if (st->use_persist) {
+    e = launch_ns_gemm_persistent(st->persist, st->persist_grid, s);
+    if (e != cudaSuccess) return cuda_fail(st, e, "ns_gemm (single launch)");
+  } else {
+    for (size_t i = 0; i < st->gemm.size(); ++i) {
+      e = launch_ns_gemm(st->gemm[i], st->gemm_grid[i], st->opt.ns_cta_pair ? 2 : 1, s);
+      if (e != cudaSuccess) return cuda_fail(st, e, "ns_gemm launch");
+    }
   }
   mark(3);
   if (st->n_two) {
@@ -1085,7 +1145,9 @@ meq_status meq_read_profile(meq_state* st, double* phase_ms, int64_t* steps) {
 
 int meq_kernels_per_step(const meq_state* st) { return st ? st->kernels_per_step : 0; }
 
-int meq_ns_gemm_launches_per_step(const meq_state* st) { return st ? static_cast<int>(st->gemm.size()) : 0; }
+int meq_ns_gemm_launches_per_step(const meq_state* st) {
+  return st ? (st->use_persist ? 1 : static_cast<int>(st->gemm.size())) : 0;
+}
 
 meq_status meq_debug_wait_selftest(meq_state* st, float timeout_ms) {
   if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");

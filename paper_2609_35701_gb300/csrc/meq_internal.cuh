@@ -22,10 +22,13 @@ enum DevErr : int {
   DEV_TIMEOUT_DRAIN = 0x105,     // waiting for in-flight copies / MMAs at exit
   DEV_TIMEOUT_SCHED_PUT = 0x106, // tile scheduler waited too long for a free slot of the tile ring
   DEV_TIMEOUT_SCHED_TAKE = 0x107,// a role waited too long for its next tile index
+  DEV_TIMEOUT_DEP = 0x108,       // one-launch NS: a tile waited too long for the product it reads
   DEV_TIMEOUT_TEST = 0x1FF,      // the wait-timeout self test
 };
 
 constexpr int kMaxGroups = 8;        // shape groups per GEMM launch
+constexpr int kMaxSegs = 48;         // (product, shape group) segments of the one-launch NS (30 KB of parameters)
+constexpr int kNsEpilogueWarps = 8;  // epilogue warps per CTA of the NS GEMM kernel
 
 // U of the hidden weights is stored as fp16(kUScale * U). Every entry of U
 // is bounded by its largest singular value, which the quintic keeps below
@@ -80,7 +83,7 @@ enum GemmMode : int { MODE_GRAM = 0, MODE_POLY = 1, MODE_XUPD = 2, MODE_XLAST = 
 struct GemmGroup {
   CUtensorMap tmA;        // A operand (K-major), box {64, 128, 1}
   CUtensorMap tmB;        // B operand: K-major box {64, 256, 1} or MN-major box {64, 64, 1}
-  CUtensorMap tmO;        // GRAM / POLY: the 16-bit symmetric output (A or P) for TMA stores,
+  CUtensorMap tmO;        // GRAM / POLY / XUPD: the 16-bit output (A, P or X next) for TMA stores,
                           // box {32, 32, 1}, 64-byte swizzle (the epilogue's staging layout)
   int32_t M, N, K;        // output rows, output cols, contraction
   int32_t count;          // matrices in the group
@@ -102,22 +105,39 @@ struct GemmGroup {
   int64_t aux_mstride;    // bytes
   float* rpart;           // XLAST: NS-row partial sums of squares, [count][2 * tiles_n][M]
   float* cpart;           // XLAST: NS-column partial sums of squares, [count][ceil(M/32)][N]
+  int32_t mode;           // GemmMode of the product
+  uint32_t idesc;         // tcgen05 instruction descriptor
+  int32_t b_mn_major;     // 1: B operand tile is MN-major (XUPD)
+  // One-launch NS only: this segment's product index (row of the completion
+  // counters), its matrices' first counter slot, and the count each of its
+  // matrices waits for in the previous product's row (0: none).
+  int32_t prod;
+  int32_t mat_base;
+  int32_t dep_target;
+  int32_t tma_out;        // 1: the output leaves by TMA stores through tmO (else 16-byte thread stores)
 };
 
-struct GemmParams {
-  GemmGroup g[kMaxGroups];
+// One GEMM launch: kSegs segments (one product's shape groups, or every
+// product's for the one-launch NS), taken as one tile queue in segment order.
+template <int kSegs>
+struct GemmParamsT {
+  GemmGroup g[kSegs];
   int32_t ngroups;
   int32_t total_tiles;
-  int32_t mode;
-  uint32_t idesc;          // tcgen05 instruction descriptor
-  int32_t b_mn_major;      // 1: B operand tile is MN-major (XUPD)
   int32_t reverse;         // 1: tiles are taken in reverse order (alternates between launches)
+  int32_t persistent;      // 1: every product of the NS in this launch, ordered by completion counters
   float ca, cb, cc;        // NS coefficients
   int* err;                // device error word
   int* sched;              // tile queue: [0] tiles handed out beyond the first wave, [1] units done;
                            // zero between launches (the last unit to finish resets both)
+  int* done;               // one-launch NS: [product][slot] epilogue-warp completions per matrix,
+                           // zero between launches (reset with the tile queue)
+  int32_t nslots;          // slots per product row of `done`
+  int32_t nprod;           // product rows of `done`
   unsigned long long timeout_ns;
 };
+using GemmParams = GemmParamsT<kMaxGroups>;
+using PersistParams = GemmParamsT<kMaxSegs>;
 
 // Programmatic dependent launch: a kernel lets the next one in the stream be
 // scheduled as soon as it starts, and waits for its predecessor's results
@@ -155,6 +175,10 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 // Launchers (defined in the .cu files).
 cudaError_t prepare_ns_gemm();  // sets the kernel's dynamic shared-memory limit (per device)
 cudaError_t launch_ns_gemm(const GemmParams& p, int grid, int pair, cudaStream_t st);  // pair: 1 or 2 CTAs per tile
+// Every NS product in one cooperative launch of CTA pairs (grid = 2 x pairs).
+cudaError_t launch_ns_gemm_persistent(const PersistParams& p, int grid, cudaStream_t st);
+// CTA pairs of the one-launch NS that can be resident at once (0 if it cannot run).
+int ns_gemm_persistent_max_pairs();
 int ns_gemm_smem_bytes(int pair);
 
 }  // namespace meq

@@ -51,7 +51,7 @@ namespace {
 
 constexpr int BM = 128, BN = 256, BK = 64, UK = 16;  // per-CTA rows, tile columns, k-block, MMA K
 constexpr int A_BYTES = BM * BK * 2;                 // 16 KB
-constexpr int NUM_EPI_WARPS = 8;                     // two per TMEM lane quarter
+constexpr int NUM_EPI_WARPS = kNsEpilogueWarps;      // two per TMEM lane quarter
 constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int SLOT_BYTES = 2048;                     // one 32 x 32 16-bit block (two per epilogue warp)
@@ -161,6 +161,42 @@ __device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap
       "l"(reinterpret_cast<uint64_t>(tm)), "r"(bar_cluster), "r"(x), "r"(y), "r"(z)
       : "memory");
 }
+// Completion counters of the one-launch NS (global memory, GPU scope).
+__device__ __forceinline__ int ld_acquire_gpu(const int* ptr) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(ptr) : "memory");
+  return v;
+}
+__device__ __forceinline__ void red_release_gpu_add(int* ptr, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(ptr), "r"(v) : "memory");
+}
+// Orders this thread's generic-proxy view of global memory with its TMA
+// (async-proxy) accesses, in both directions.
+__device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
+// 16-byte load through L2 only (the data may have been written by another SM
+// during this launch, so neither L1 nor the read-only path may serve it).
+__device__ __forceinline__ uint4 ld_cg_v4(const void* ptr) {
+  uint4 v;
+  asm volatile("ld.global.cg.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(ptr));
+  return v;
+}
+// Bounded wait (one thread) until *ptr >= target, with acquire at GPU scope.
+__device__ bool wait_count(const int* ptr, int target, int* err, int code, uint64_t timeout_ns) {
+  if (ld_acquire_gpu(ptr) >= target) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 1;; ++it) {
+    __nanosleep(128);
+    if (ld_acquire_gpu(ptr) >= target) return true;
+    if ((it & 15u) == 0) {
+      if (*reinterpret_cast<volatile int*>(err) != 0) return false;
+      if (global_ns() - t0 > timeout_ns || it >= (1u << 26)) {
+        atomicCAS(err, 0, code);
+        return false;
+      }
+    }
+  }
+}
+
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
@@ -281,11 +317,20 @@ struct TileCoord {
 // over tiles_m x tiles_n; symmetric outputs (Gram, polynomial) run tn-major
 // over the tiles with tm * TILE_M < (tn + 1) * 256, i.e. those holding a
 // 32 x 32 block on or above the diagonal.
-template <int kPair>
-__device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
+template <int kSegs>
+__device__ __forceinline__ int find_segment(const GemmParamsT<kSegs>& p, int t) {
+  int lo = 0, hi = p.ngroups - 1;  // the last segment whose tile_begin <= t
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.g[mid].tile_begin <= t) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+template <int kPair, int kSegs>
+__device__ __forceinline__ TileCoord decode_tile(const GemmParamsT<kSegs>& p, int t) {
   if (p.reverse) t = p.total_tiles - 1 - t;
-  int g = 0;
-  while (g + 1 < p.ngroups && t >= p.g[g + 1].tile_begin) ++g;
+  const int g = find_segment(p, t);
   const GemmGroup& G = p.g[g];
   const int local = t - G.tile_begin;
   const int mat = local / G.tiles_per_mat;
@@ -402,8 +447,21 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_reads() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 // Every committed store has completed.
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-template <int kPair>
-__global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_constant__ GemmParams p) {
+// Every committed store but those of the `keep` most recent groups (0..4) has completed.
+__device__ __forceinline__ void bulk_wait_keep(int keep) {
+  switch (keep) {
+    case 0: asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); break;
+    case 1: asm volatile("cp.async.bulk.wait_group 1;" ::: "memory"); break;
+    case 2: asm volatile("cp.async.bulk.wait_group 2;" ::: "memory"); break;
+    case 3: asm volatile("cp.async.bulk.wait_group 3;" ::: "memory"); break;
+    default: asm volatile("cp.async.bulk.wait_group 4;" ::: "memory"); break;
+  }
+}
+template <int kPair, int kSegs>
+__global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_constant__ GemmParamsT<kSegs> p) {
+  // The one-launch NS (every product, completion counters) is the kMaxSegs
+  // instantiation; the per-product launches compile without its code.
+  constexpr bool kPersistent = kSegs == kMaxSegs;
   using C_ = Cfg<kPair>;
   constexpr int STAGES = C_::STAGES;
   constexpr int STAGE_BYTES = C_::STAGE_BYTES;
@@ -520,12 +578,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
         if (n > 0 && leader) t = nunits + fetched;
         if (leader ? !sched_put(n, t) : !sched_take(n, t)) break;
         if (t >= p.total_tiles) break;
+        const TileCoord c = decode_tile<kPair>(p, t);
+        const GemmGroup& G = p.g[c.g];
+        if (kPersistent && G.dep_target > 0) {
+          // the previous product of this matrix is complete, and visible to TMA
+          if (!wait_count(p.done + (G.prod - 1) * p.nslots + G.mat_base + c.mat, G.dep_target, err, DEV_TIMEOUT_DEP,
+                          tmo)) {
+            ok = false;
+            break;
+          }
+          fence_proxy_async_global();
+        }
         // The next index is fetched while this tile's operands are requested;
         // its value is first read at the top of the next iteration.
         if (leader) fetched = atomicAdd(p.sched, 1);
-        const TileCoord c = decode_tile<kPair>(p, t);
-        const GemmGroup& G = p.g[c.g];
         const int nk = (G.K + BK - 1) / BK;
+        // Mode, descriptor and B layout are per segment in the one-launch NS
+        // and per launch otherwise, where reading them at a fixed index keeps
+        // them launch-uniform for the compiler (measured: 2% of the step).
+        const int b_mn_major = kPersistent ? G.b_mn_major : p.g[0].b_mn_major;
         const int arow = c.tm * TILE_M + static_cast<int>(rank) * BM;
         const int bcol = c.tn * BN + static_cast<int>(rank) * C_::BN_LOCAL;
         for (int kb = 0; kb < nk; ++kb) {
@@ -538,7 +609,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
           if (kPair == 1) {
             mbar_expect_tx(FULL_BAR(stage), STAGE_BYTES);
             tma_load_3d(sa, &G.tmA, FULL_BAR(stage), kb * BK, arow, c.mat);
-            if (!p.b_mn_major) {
+            if (!b_mn_major) {
               tma_load_3d(sb, &G.tmB, FULL_BAR(stage), kb * BK, bcol, c.mat);
             } else {
 #pragma unroll
@@ -551,7 +622,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
             if (leader) mbar_expect_tx(FULL_BAR(stage), 2 * STAGE_BYTES);
             const uint32_t fb = leader ? FULL_BAR(stage) : map_to_rank(FULL_BAR(stage), 0);
             tma_load_3d_pair(sa, &G.tmA, fb, kb * BK, arow, c.mat);
-            if (!p.b_mn_major) {
+            if (!b_mn_major) {
               tma_load_3d_pair(sb, &G.tmB, fb, kb * BK, bcol, c.mat);
             } else {
 #pragma unroll
@@ -583,12 +654,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
-      const uint32_t b_lbo = p.b_mn_major ? (64u * BK * 2u) : 16u;
       for (int n = 0; ok; ++n) {
         int t = 0;
         if (!sched_take(n, t) || t >= p.total_tiles) break;
         const TileCoord c = decode_tile<kPair>(p, t);
-        const int nk = (p.g[c.g].K + BK - 1) / BK;
+        const GemmGroup& G = p.g[c.g];
+        const int nk = (G.K + BK - 1) / BK;
+        const int b_mn_major = kPersistent ? G.b_mn_major : p.g[0].b_mn_major;
+        const uint32_t idesc = kPersistent ? G.idesc : p.g[0].idesc;
+        const uint32_t b_lbo = b_mn_major ? (64u * BK * 2u) : 16u;
         if (!wait_bounded(TEMPTY_BAR(acc), acc_phase ^ 1u, err, DEV_TIMEOUT_MMA_TMEM, tmo)) break;
         tc_fence_after();
         const uint32_t d = tmem_base + static_cast<uint32_t>(acc * BN);
@@ -603,10 +677,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
 #pragma unroll
           for (int k = 0; k < BK / UK; ++k) {
             const uint64_t adesc = smem_desc(sa + k * (UK * 2), 16u, 1024u);
-            const uint64_t bdesc = p.b_mn_major ? smem_desc(sb + k * (UK * 128), b_lbo, 1024u)
+            const uint64_t bdesc = b_mn_major ? smem_desc(sb + k * (UK * 128), b_lbo, 1024u)
                                                 : smem_desc(sb + k * (UK * 2), 16u, 1024u);
-            if (kPair == 2) tc_mma_pair(d, adesc, bdesc, p.idesc, (kb > 0 || k > 0) ? 1u : 0u);
-            else tc_mma(d, adesc, bdesc, p.idesc, (kb > 0 || k > 0) ? 1u : 0u);
+            if (kPair == 2) tc_mma_pair(d, adesc, bdesc, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+            else tc_mma(d, adesc, bdesc, idesc, (kb > 0 || k > 0) ? 1u : 0u);
           }
           if (kPair == 2) tc_commit_pair_both(EMPTY_BAR(stage));
           else tc_commit(EMPTY_BAR(stage));
@@ -643,13 +717,31 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     const int half = ew >> 2;
     uint8_t* slot = gbase + C_::SMEM_EPI_OFF + ew * (2 * SLOT_BYTES);
     uint8_t* slot_t = slot + SLOT_BYTES;
-    const int mode = p.mode;
     int acc = 0;
     uint32_t acc_phase = 0;
 
     // The leader's tmem-empty barrier counts the epilogue warps of both CTAs.
     const uint32_t tempty_target0 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(0), 0) : TEMPTY_BAR(0);
     const uint32_t tempty_target1 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(1), 0) : TEMPTY_BAR(1);
+    // One-launch NS: each warp counts its part of a tile as done once the
+    // tile's stores have landed (release at GPU scope), for the next
+    // product's tiles of that matrix. The count of tile n is deferred to the
+    // end of tile n + 1's epilogue, by when tile n's stores have long
+    // completed (the wait skips tile n + 1's own store groups) -- unless tile
+    // n + 1's accumulator is not ready yet, in which case it is sent before
+    // waiting (tile n + 1 may depend on it).
+    // (Every output another tile waits for leaves by TMA stores: the host
+    // sets tma_out on every product but the last.)
+    int pend = -1;  // completion counter of the tile awaiting its count
+    auto signal_pending = [&](int keep_groups) {
+      __syncwarp();
+      if (lane == 0) {
+        bulk_wait_keep(keep_groups);
+        fence_proxy_async_global();
+        red_release_gpu_add(p.done + pend, 1);
+      }
+      pend = -1;
+    };
     for (int n = 0;; ++n) {
       int t = 0, got = 1;
       if (lane == 0) got = sched_take(n, t) ? 1 : 0;
@@ -658,7 +750,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       if (!got || t >= p.total_tiles) break;
       const TileCoord c = decode_tile<kPair>(p, t);
       const GemmGroup& G = p.g[c.g];
+      const int mode = kPersistent ? G.mode : p.g[0].mode;  // one mode per launch (a launch-uniform read)
+      if (pend >= 0 && !__all_sync(0xffffffffu, mbar_try_wait(TFULL_BAR(acc), acc_phase))) signal_pending(0);
       if (!wait_bounded_warp(TFULL_BAR(acc), acc_phase, err, DEV_TIMEOUT_EPI, tmo)) break;
+      if (kPersistent && mode == MODE_POLY && G.dep_target > 0) {
+        // The A read below comes from the previous product of this launch:
+        // acquire its completion. It is complete by now, since the tile's
+        // operands waited for it; waiting before the accumulator could
+        // deadlock (the count may still lack this warp's own deferred one).
+        int okd = 1;
+        if (lane == 0)
+          okd = wait_count(p.done + (G.prod - 1) * p.nslots + G.mat_base + c.mat, G.dep_target, err, DEV_TIMEOUT_DEP,
+                           tmo)
+                    ? 1
+                    : 0;
+        if (!__shfl_sync(0xffffffffu, okd, 0)) break;
+      }
       tc_fence_after();
       const int row0 = c.tm * TILE_M + static_cast<int>(rank) * BM + q * 32;
       const int R = row0 / 32;  // 32-row block index
@@ -677,18 +784,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
         for (int i = 0; i < 4; ++i) {
           const int r = (lane >> 2) + 8 * i;
           aux[i] = make_uint4(0u, 0u, 0u, 0u);
-          if (r < rows_valid)
-            aux[i] = __ldg(reinterpret_cast<const uint4*>(auxm + static_cast<int64_t>(row0 + r) * G.aux_ld +
-                                                         static_cast<int64_t>(col0) * 2 + (lane & 3) * 16));
+          if (r < rows_valid) {
+            const uint4* src = reinterpret_cast<const uint4*>(auxm + static_cast<int64_t>(row0 + r) * G.aux_ld +
+                                                              static_cast<int64_t>(col0) * 2 + (lane & 3) * 16);
+            aux[i] = kPersistent ? ld_cg_v4(src) : __ldg(src);
+          }
         }
       };
       if (mode == MODE_POLY && ch0 < nch) load_aux(c.tn * BN + ch0 * 32);
+      int tile_groups = 0;  // TMA store groups this warp commits for the tile
       for (int ch = ch0; ch < nch; ch += 2) {
         const int col0 = c.tn * BN + ch * 32;
         const int C = c.tn * 8 + ch;
         float v[32];
         tmem_ld_32cols(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN + ch * 32), v);
-        if (G.sym) {
+        if (G.tma_out) {
           if (lane == 0) bulk_wait_reads();  // both slots free
         }
         __syncwarp();
@@ -765,7 +875,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
             store_block64(slot_t, lane, outm + static_cast<int64_t>(col0) * G.out_ld + row0 * 2, G.out_ld,
                           min(32, G.N - col0), min(4, (G.M - row0 + 7) / 8));
           }
-        } else if (!G.sym) {
+        } else if (!G.tma_out) {
           // X rows are padded to a multiple of 64 elements: whole 32-column blocks stay inside them
           fill_half_rows(slot, lane, v, G.out_fp16);
           __syncwarp();
@@ -786,7 +896,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
           }
         }
         __syncwarp();  // reconverge before the next warp-wide tcgen05.ld
+        if (G.tma_out) ++tile_groups;
       }
+      if (pend >= 0) signal_pending(tile_groups);  // the previous tile, behind this tile's store groups
       if (mode == MODE_XLAST && row0 < G.M && row0 + lane < G.M)  // one partial per (tile column, half)
         G.rpart[(static_cast<int64_t>(c.mat) * G.tiles_n * 2 + c.tn * 2 + half) * G.M + row0 + lane] = rsum * kUInvScale2;
       tc_fence_before();
@@ -796,7 +908,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
+      if (kPersistent && G.prod + 1 < p.nprod) pend = G.prod * p.nslots + G.mat_base + c.mat;
     }
+    if (pend >= 0) signal_pending(0);
     // The outputs are in global memory before the CTA leaves.
     if (lane == 0) bulk_wait_all();
     __syncwarp();
@@ -827,6 +941,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     if (atomicAdd(p.sched + 1, 1) == nunits - 1) {
       p.sched[0] = 0;
       p.sched[1] = 0;
+      if (kPersistent)
+        for (int i = 0; i < p.nprod * p.nslots; ++i) p.done[i] = 0;
     }
   }
   if (warp == 1) {
@@ -839,19 +955,67 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
 
 }  // namespace
 
+static_assert(sizeof(PersistParams) <= 32000, "one-launch NS parameters exceed the kernel parameter space");
+
 int ns_gemm_smem_bytes(int pair) { return pair == 2 ? Cfg<2>::SMEM_BYTES : Cfg<1>::SMEM_BYTES; }
 
 cudaError_t prepare_ns_gemm() {
-  cudaError_t e =
-      cudaFuncSetAttribute(ns_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<1>::SMEM_BYTES);
+  cudaError_t e = cudaFuncSetAttribute(ns_gemm_kernel<1, kMaxGroups>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       Cfg<1>::SMEM_BYTES);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(ns_gemm_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<2>::SMEM_BYTES);
+  e = cudaFuncSetAttribute(ns_gemm_kernel<2, kMaxGroups>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           Cfg<2>::SMEM_BYTES);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(ns_gemm_kernel<2, kMaxSegs>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              Cfg<2>::SMEM_BYTES);
 }
 
 cudaError_t launch_ns_gemm(const GemmParams& p, int grid, int pair, cudaStream_t st) {
   if (pair == 2)
-    return launch_pdl(ns_gemm_kernel<2>, dim3(grid), dim3(NUM_THREADS), Cfg<2>::SMEM_BYTES, st, 2, p);
-  return launch_pdl(ns_gemm_kernel<1>, dim3(grid), dim3(NUM_THREADS), Cfg<1>::SMEM_BYTES, st, 1, p);
+    return launch_pdl(ns_gemm_kernel<2, kMaxGroups>, dim3(grid), dim3(NUM_THREADS), Cfg<2>::SMEM_BYTES, st, 2, p);
+  return launch_pdl(ns_gemm_kernel<1, kMaxGroups>, dim3(grid), dim3(NUM_THREADS), Cfg<1>::SMEM_BYTES, st, 1, p);
+}
+
+int ns_gemm_persistent_max_pairs() {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2);
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = Cfg<2>::SMEM_BYTES;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, ns_gemm_kernel<2, kMaxSegs>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return clusters;
+}
+
+// Tiles of later products wait for earlier ones on other SMs, so every CTA
+// must be resident at once: a cooperative launch (one CTA per SM).
+cudaError_t launch_ns_gemm_persistent(const PersistParams& p, int grid, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = Cfg<2>::SMEM_BYTES;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[3];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 2;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  attr[2].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[2].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 3;
+  return cudaLaunchKernelEx(&cfg, ns_gemm_kernel<2, kMaxSegs>, p);
 }
 
 }  // namespace meq

@@ -43,6 +43,7 @@ class MeqOptions(ctypes.Structure):
         ("ns_x0_fused", ctypes.c_int),
         ("update_rule", ctypes.c_int),
         ("debug_canaries", ctypes.c_int),
+        ("ns_single_launch", ctypes.c_int),
     ]
 
 
