@@ -421,12 +421,15 @@ def main():
         # Copies move in pieces of COPY_CHUNK elements (a single copy of
         # hundreds of MB runs at half the rate of the same bytes in pieces on
         # this host link), on two copy streams: the gradients of step k go up
-        # while step k - 1 runs; the parameters of step k come back after it,
-        # before step k + 1 updates them in place.
+        # while step k - 1 runs; the parameters of step k - 1 come back while
+        # step k's momentum, Newton-Schulz and statistics run
+        # (meq_step_prepare), and step k's update (meq_step_apply) waits for
+        # that copy before it writes the parameters in place.
         pieces = [(lo, min(lo + COPY_CHUNK, pbuf.numel())) for lo in range(0, pbuf.numel(), COPY_CHUNK)]
         up, down = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
         ev_in = [torch.cuda.Event() for _ in range(2)]
-        ev_step = [torch.cuda.Event() for _ in range(2)]
+        ev_prep = [torch.cuda.Event() for _ in range(2)]
+        ev_step = torch.cuda.Event()
         ev_out = torch.cuda.Event()
         torch.cuda.synchronize()
         a0 = torch.cuda.Event(enable_timing=True)
@@ -437,17 +440,19 @@ def main():
             b = k % 2
             with torch.cuda.stream(up):
                 if k >= 2:
-                    up.wait_event(ev_step[b])   # step k - 2 has read this gradient buffer
+                    up.wait_event(ev_prep[b])   # step k - 2 has read this gradient buffer
                 for lo, hi in pieces:
                     gbufs[b][0][lo:hi].copy_(hg[b][lo:hi], non_blocking=True)
                 ev_in[b].record(up)
             stream.wait_event(ev_in[b])
+            opt.step_prepare(grads[b], LR, MU, WD, EPS)
+            ev_prep[b].record(stream)
             if k >= 1:
                 stream.wait_event(ev_out)        # parameters of step k - 1 are back on the host
-            opt.step(params, grads[b], LR, MU, WD, EPS)
-            ev_step[b].record(stream)
+            opt.step_apply(params)
+            ev_step.record(stream)
             with torch.cuda.stream(down):
-                down.wait_event(ev_step[b])
+                down.wait_event(ev_step)
                 for lo, hi in pieces:
                     hp[lo:hi].copy_(pbuf[lo:hi], non_blocking=True)
                 ev_out.record(down)
@@ -460,7 +465,8 @@ def main():
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
             e2e_ms = float(t.item())
         e2e = {"value": e2e_ms, "unit": "ms/step", "h2d_bytes_per_step": 4 * numel * (world if world > 1 else 1),
-               "d2h_bytes_per_step": 4 * numel * (world if world > 1 else 1), "steps": n_e2e}
+               "d2h_bytes_per_step": 4 * numel * (world if world > 1 else 1), "steps": n_e2e,
+               "api": "meq_step_prepare + meq_step_apply (parameter read-back of step k - 1 overlaps step k's prepare)"}
     opt.sync()
 
     cpu = None

@@ -145,6 +145,26 @@ meq_status meq_step(float* const* params, const float* const* grads, meq_state* 
                     const meq_shape* shapes, int n, float lr, float momentum,
                     float weight_decay, float eps, void* cuda_stream);
 
+/* The same step in two calls, split before the parameter update, so that a
+ * caller can overlap work on the parameters of the previous step (a copy
+ * to the host, an all-gather) with this step's momentum, Newton-Schulz and
+ * statistics, which do not touch the parameters:
+ *   meq_step_prepare: Eq. (10), Eq. (5) and the statistics of Eqs. (7)-(9)
+ *     and (11) (Algorithm 1 up to the update), for the gradients and scalars
+ *     given (the arguments of meq_step without params);
+ *   meq_step_apply: the update (Eq. (14); Eqs. (12) and (13) for the other
+ *     kinds) of params with the scalars of the pending prepare.
+ * meq_step(params, grads, ...) equals meq_step_prepare(grads, ...) then
+ * meq_step_apply(params, ...), bit for bit. Each call enqueues on its
+ * cuda_stream; the apply must be ordered after its prepare and before the
+ * next prepare (for example, one stream, with a cudaStreamWaitEvent on the
+ * caller's copy before the apply). A second prepare before the apply, an
+ * apply without a prepare, or meq_step while a prepare is pending returns
+ * MEQ_ERR_INVALID_ARG. With use_graph, each part replays its own graph. */
+meq_status meq_step_prepare(const float* const* grads, meq_state* st, const meq_shape* shapes, int n,
+                            float lr, float momentum, float weight_decay, float eps, void* cuda_stream);
+meq_status meq_step_apply(float* const* params, meq_state* st, void* cuda_stream);
+
 /* Wait for the state's enqueued work and report device-side errors
  * (MEQ_ERR_TIMEOUT for an expired bounded wait, MEQ_ERR_CUDA otherwise), then
  * MEQ_ERR_NONFINITE if, in a step since the last meq_sync, the momentum of

@@ -132,6 +132,10 @@ struct meq_state {
   bool graph_ready = false;
   cudaGraph_t graph = nullptr;
   cudaGraphExec_t gexec = nullptr;
+  // meq_step_prepare / meq_step_apply: one graph each, captured on first use
+  cudaGraph_t graph_prep = nullptr, graph_apply = nullptr;
+  cudaGraphExec_t gexec_prep = nullptr, gexec_apply = nullptr;
+  bool prepared = false;  // a prepare is waiting for its apply
   cudaStream_t last_stream = nullptr;
   int kernels_per_step = 0;
   bool profiling = false;
@@ -776,7 +780,9 @@ struct NvtxRange {
   ~NvtxRange() { nvtxRangePop(); }
 };
 
-static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev = nullptr) {
+enum StepParts : int { PART_PREPARE = 1, PART_APPLY = 2, PART_ALL = 3 };
+
+static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev = nullptr, int parts = PART_ALL) {
   const LaunchCtx& C = st->ctx;
   // NVTX ranges name the stages on the host timeline (each eager enqueue, or
   // the capture of the graph); CUDA events time them on the stream.
@@ -788,6 +794,11 @@ static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev
     stage.next(i < 5 ? kStage[i] : nullptr);
   };
   cudaError_t e = cudaSuccess;
+  if (!(parts & PART_PREPARE)) {
+    mark(4);
+    e = launch_apply(C, s);
+    return e == cudaSuccess ? MEQ_OK : cuda_fail(st, e, "apply launch");
+  }
   mark(0);
   const bool fused = st->opt.ns_x0_fused != 0;
   if (st->n_hidden) {
@@ -825,13 +836,14 @@ static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev
   e = launch_stats(C, s);
   if (e != cudaSuccess) return cuda_fail(st, e, "finalize launch");
   mark(4);
+  if (!(parts & PART_APPLY)) return MEQ_OK;
   e = launch_apply(C, s);
   if (e != cudaSuccess) return cuda_fail(st, e, "apply launch");
   mark(5);
   return MEQ_OK;
 }
 
-static meq_status capture_graph(meq_state* st) {
+static meq_status capture_graph(meq_state* st, int parts, cudaGraph_t* graph, cudaGraphExec_t* gexec) {
   cudaStream_t cs = nullptr;
   cudaError_t e = cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking);
   if (e != cudaSuccess) return cuda_fail(st, e, "cudaStreamCreate");
@@ -840,7 +852,7 @@ static meq_status capture_graph(meq_state* st) {
     cudaStreamDestroy(cs);
     return cuda_fail(st, e, "cudaStreamBeginCapture");
   }
-  meq_status ms = enqueue_kernels(st, cs);
+  meq_status ms = enqueue_kernels(st, cs, nullptr, parts);
   cudaGraph_t g = nullptr;
   e = cudaStreamEndCapture(cs, &g);
   cudaStreamDestroy(cs);
@@ -855,28 +867,28 @@ static meq_status capture_graph(meq_state* st) {
     cudaGraphDestroy(g);
     return cuda_fail(st, e, "cudaGraphInstantiate");
   }
-  st->graph = g;
-  st->gexec = x;
-  st->graph_ready = true;
+  *graph = g;
+  *gexec = x;
   return MEQ_OK;
 }
 
-meq_status meq_step(float* const* params, const float* const* grads, meq_state* st, const meq_shape* shapes, int n,
-                    float lr, float momentum, float weight_decay, float eps, void* cuda_stream) {
-  NvtxRange range("meq_step");
-  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
-  if (!params || !grads || !shapes) return fail(st, MEQ_ERR_INVALID_ARG, "params, grads and shapes must be non-NULL");
+// Checks shapes and scalars and uploads the per-step block (scalars, then
+// the params and grads pointer tables; params may be NULL: that table is
+// left as it is).
+static meq_status upload_step(meq_state* st, float* const* params, const float* const* grads, const meq_shape* shapes,
+                              int n, float lr, float momentum, float weight_decay, float eps, cudaStream_t s) {
+  if (!grads || !shapes) return fail(st, MEQ_ERR_INVALID_ARG, "grads and shapes must be non-NULL");
   if (n != st->n) return fail(st, MEQ_ERR_INVALID_ARG, "n differs from the init-time shape list");
   for (int i = 0; i < n; ++i) {
     if (shapes[i].rows != st->shapes[i].rows || shapes[i].cols != st->shapes[i].cols)
       return fail(st, MEQ_ERR_INVALID_ARG, "shape of matrix " + std::to_string(i) + " differs from init");
-    if (!params[i] || !grads[i]) return fail(st, MEQ_ERR_INVALID_ARG, "NULL params/grads pointer at " + std::to_string(i));
-    if ((reinterpret_cast<uintptr_t>(params[i]) & 15u) || (reinterpret_cast<uintptr_t>(grads[i]) & 15u))
+    if ((params && !params[i]) || !grads[i])
+      return fail(st, MEQ_ERR_INVALID_ARG, "NULL params/grads pointer at " + std::to_string(i));
+    if ((params && (reinterpret_cast<uintptr_t>(params[i]) & 15u)) || (reinterpret_cast<uintptr_t>(grads[i]) & 15u))
       return fail(st, MEQ_ERR_INVALID_ARG, "params/grads pointer " + std::to_string(i) + " is not 16-byte aligned");
   }
   if (!std::isfinite(lr) || !std::isfinite(momentum) || !std::isfinite(weight_decay) || !(eps >= 0.f) || !std::isfinite(eps))
     return fail(st, MEQ_ERR_INVALID_ARG, "lr, momentum, weight_decay must be finite and eps >= 0");
-  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   StepScalars sc;
   std::memset(&sc, 0, sizeof(sc));
   sc.lr = lr, sc.mu = momentum, sc.wd = weight_decay, sc.eps = eps;
@@ -884,32 +896,93 @@ meq_status meq_step(float* const* params, const float* const* grads, meq_state* 
   sc.rule = st->opt.update_rule;
   char* h = st->step_host.data();
   std::memcpy(h, &sc, sizeof(sc));
-  std::memcpy(h + sizeof(sc), params, n * sizeof(void*));
+  if (params) std::memcpy(h + sizeof(sc), params, n * sizeof(void*));
   std::memcpy(h + sizeof(sc) + n * sizeof(void*), grads, n * sizeof(void*));
   // Pageable source: the call returns once the bytes are staged, so the
   // host buffer can be reused by the next step right away.
-  cudaError_t e = cudaMemcpyAsync(st->d_step, h, static_cast<size_t>(st->step_bytes), cudaMemcpyHostToDevice, s);
+  cudaError_t e;
+  if (params) {
+    e = cudaMemcpyAsync(st->d_step, h, static_cast<size_t>(st->step_bytes), cudaMemcpyHostToDevice, s);
+  } else {
+    e = cudaMemcpyAsync(st->d_step, h, sizeof(sc), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(st->d_step + sizeof(sc) + n * sizeof(void*), h + sizeof(sc) + n * sizeof(void*),
+                          n * sizeof(void*), cudaMemcpyHostToDevice, s);
+  }
   if (e != cudaSuccess) return cuda_fail(st, e, "step upload");
   st->last_stream = s;
+  return MEQ_OK;
+}
+
+// Runs the given parts of the step on s: eagerly, or from its graph.
+static meq_status run_parts(meq_state* st, int parts, cudaStream_t s) {
+  if (st->opt.use_graph) {
+    cudaGraph_t* g = parts == PART_ALL ? &st->graph : parts == PART_PREPARE ? &st->graph_prep : &st->graph_apply;
+    cudaGraphExec_t* x = parts == PART_ALL ? &st->gexec : parts == PART_PREPARE ? &st->gexec_prep : &st->gexec_apply;
+    if (!*x) {
+      meq_status ms = capture_graph(st, parts, g, x);
+      if (ms != MEQ_OK) return ms;
+      if (parts == PART_ALL) st->graph_ready = true;
+    }
+    cudaError_t e = cudaGraphLaunch(*x, s);
+    return e == cudaSuccess ? MEQ_OK : cuda_fail(st, e, "cudaGraphLaunch");
+  }
+  return enqueue_kernels(st, s, nullptr, parts);
+}
+
+meq_status meq_step(float* const* params, const float* const* grads, meq_state* st, const meq_shape* shapes, int n,
+                    float lr, float momentum, float weight_decay, float eps, void* cuda_stream) {
+  NvtxRange range("meq_step");
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  if (!params) return fail(st, MEQ_ERR_INVALID_ARG, "params must be non-NULL");
+  if (st->prepared) return fail(st, MEQ_ERR_INVALID_ARG, "a meq_step_prepare is waiting for its meq_step_apply");
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  meq_status ms = upload_step(st, params, grads, shapes, n, lr, momentum, weight_decay, eps, s);
+  if (ms != MEQ_OK) return ms;
   if (st->profiling) {
     std::vector<cudaEvent_t> ev(6, nullptr);
     for (auto& x : ev) {
-      e = cudaEventCreate(&x);
+      cudaError_t e = cudaEventCreate(&x);
       if (e != cudaSuccess) return cuda_fail(st, e, "cudaEventCreate");
     }
     st->prof_events.push_back(ev);
     return enqueue_kernels(st, s, st->prof_events.back().data());
   }
-  if (st->opt.use_graph) {
-    if (!st->graph_ready) {
-      meq_status ms = capture_graph(st);
-      if (ms != MEQ_OK) return ms;
-    }
-    e = cudaGraphLaunch(st->gexec, s);
-    if (e != cudaSuccess) return cuda_fail(st, e, "cudaGraphLaunch");
-    return MEQ_OK;
+  return run_parts(st, PART_ALL, s);
+}
+
+meq_status meq_step_prepare(const float* const* grads, meq_state* st, const meq_shape* shapes, int n, float lr,
+                            float momentum, float weight_decay, float eps, void* cuda_stream) {
+  NvtxRange range("meq_step");
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  if (st->prepared) return fail(st, MEQ_ERR_INVALID_ARG, "meq_step_prepare twice without meq_step_apply");
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  meq_status ms = upload_step(st, nullptr, grads, shapes, n, lr, momentum, weight_decay, eps, s);
+  if (ms != MEQ_OK) return ms;
+  ms = run_parts(st, PART_PREPARE, s);
+  if (ms == MEQ_OK) st->prepared = true;
+  return ms;
+}
+
+meq_status meq_step_apply(float* const* params, meq_state* st, void* cuda_stream) {
+  NvtxRange range("meq_step");
+  if (!st) return fail(nullptr, MEQ_ERR_INVALID_ARG, "state is NULL");
+  if (!st->prepared) return fail(st, MEQ_ERR_INVALID_ARG, "meq_step_apply without a meq_step_prepare");
+  if (!params) return fail(st, MEQ_ERR_INVALID_ARG, "params must be non-NULL");
+  for (int i = 0; i < st->n; ++i) {
+    if (!params[i]) return fail(st, MEQ_ERR_INVALID_ARG, "NULL params pointer at " + std::to_string(i));
+    if (reinterpret_cast<uintptr_t>(params[i]) & 15u)
+      return fail(st, MEQ_ERR_INVALID_ARG, "params pointer " + std::to_string(i) + " is not 16-byte aligned");
   }
-  return enqueue_kernels(st, s);
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  char* h = st->step_host.data() + sizeof(StepScalars);
+  std::memcpy(h, params, st->n * sizeof(void*));
+  cudaError_t e = cudaMemcpyAsync(st->d_step + sizeof(StepScalars), h, st->n * sizeof(void*), cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_fail(st, e, "step upload");
+  st->last_stream = s;
+  meq_status ms = run_parts(st, PART_APPLY, s);
+  if (ms == MEQ_OK) st->prepared = false;
+  return ms;
 }
 
 meq_status meq_sync(meq_state* st) {
@@ -946,6 +1019,10 @@ meq_status meq_free(meq_state* st) {
   drop_profile(st);
   if (st->gexec) cudaGraphExecDestroy(st->gexec);
   if (st->graph) cudaGraphDestroy(st->graph);
+  if (st->gexec_prep) cudaGraphExecDestroy(st->gexec_prep);
+  if (st->graph_prep) cudaGraphDestroy(st->graph_prep);
+  if (st->gexec_apply) cudaGraphExecDestroy(st->gexec_apply);
+  if (st->graph_apply) cudaGraphDestroy(st->graph_apply);
   if (st->arena) cudaFree(st->arena);
   delete st;
   return MEQ_OK;

@@ -55,6 +55,7 @@ EXPORTED = [
     "meq_init_state_kinds", "meq_state_bytes_kinds", "meq_ns_gemm_launches_per_step",
     "meq_read_direction_counts", "meq_reset_direction_counts", "meq_ns_cv_trajectory",
     "meq_check_canaries", "meq_canary_count", "meq_debug_corrupt_canary",
+    "meq_step_prepare", "meq_step_apply",
 ]
 HIDDEN, REMAINING_2D, VECTOR = 0, 1, 2  # meq_kind
 RULE_MEQMUON, RULE_MUON = 0, 1          # meq_update_rule
@@ -74,6 +75,10 @@ def _load():
     lib.meq_init_state.restype = I
     lib.meq_step.argtypes = [ctypes.POINTER(P), ctypes.POINTER(P), P, ctypes.POINTER(MeqShape), I, F, F, F, F, P]
     lib.meq_step.restype = I
+    lib.meq_step_prepare.argtypes = [ctypes.POINTER(P), P, ctypes.POINTER(MeqShape), I, F, F, F, F, P]
+    lib.meq_step_prepare.restype = I
+    lib.meq_step_apply.argtypes = [ctypes.POINTER(P), P, P]
+    lib.meq_step_apply.restype = I
     lib.meq_sync.argtypes = [P]
     lib.meq_sync.restype = I
     lib.meq_free.argtypes = [P]
@@ -249,6 +254,33 @@ class MeqMuon:
                 raise ValueError("params and grads must be contiguous fp32 CUDA tensors")
         self.step_ptrs([p.data_ptr() for p in params], [g.data_ptr() for g in grads], lr, momentum, weight_decay,
                        eps, stream)
+
+    @staticmethod
+    def _check_tensors(ts):
+        for t in ts:
+            if not t.is_cuda or t.dtype.itemsize != 4 or not t.is_contiguous():
+                raise ValueError("params and grads must be contiguous fp32 CUDA tensors")
+
+    def step_prepare(self, grads, lr, momentum, weight_decay, eps=1e-7, stream=None):
+        """First half of a step (meq_step_prepare): momentum, Newton-Schulz and
+        statistics for these gradients; the parameters are not touched."""
+        if len(grads) != len(self.shapes):
+            raise ValueError("grads must have one tensor per matrix")
+        self._check_tensors(grads)
+        n = len(self.shapes)
+        for i, g in enumerate(grads):
+            self._gp[i] = g.data_ptr()
+        self._check(lib.meq_step_prepare(self._gp, self._st, self._shape_arr, n, float(lr), float(momentum),
+                                         float(weight_decay), float(eps), _stream_handle(stream)))
+
+    def step_apply(self, params, stream=None):
+        """Second half of a step (meq_step_apply): the update of params."""
+        if len(params) != len(self.shapes):
+            raise ValueError("params must have one tensor per matrix")
+        self._check_tensors(params)
+        for i, p in enumerate(params):
+            self._pp[i] = p.data_ptr()
+        self._check(lib.meq_step_apply(self._pp, self._st, _stream_handle(stream)))
 
     def sync(self):
         self._check(lib.meq_sync(self._st))
