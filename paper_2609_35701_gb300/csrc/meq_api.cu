@@ -527,7 +527,6 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
       Q.ngroups = nseg;
       Q.total_tiles = tiles;
       Q.reverse = 0;
-      Q.persistent = 1;
       Q.ca = P0.ca, Q.cb = P0.cb, Q.cc = P0.cc;
       Q.err = st->d_err;
       Q.sched = st->d_sched;

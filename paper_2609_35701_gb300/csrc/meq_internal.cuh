@@ -117,15 +117,15 @@ struct GemmGroup {
   int32_t tma_out;        // 1: the output leaves by TMA stores through tmO (else 16-byte thread stores)
 };
 
-// One GEMM launch: kSegs segments (one product's shape groups, or every
-// product's for the one-launch NS), taken as one tile queue in segment order.
+// One GEMM launch: kSegs segments (one product's shape groups, or, with
+// kSegs = kMaxSegs, every product's for the one-launch NS), taken as one tile
+// queue in segment order.
 template <int kSegs>
 struct GemmParamsT {
   GemmGroup g[kSegs];
   int32_t ngroups;
   int32_t total_tiles;
   int32_t reverse;         // 1: tiles are taken in reverse order (alternates between launches)
-  int32_t persistent;      // 1: every product of the NS in this launch, ordered by completion counters
   float ca, cb, cc;        // NS coefficients
   int* err;                // device error word
   int* sched;              // tile queue: [0] tiles handed out beyond the first wave, [1] units done;
