@@ -290,6 +290,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--update-rule", default="meqmuon", choices=["meqmuon", "muon"],
                     help="meqmuon: Eq. (11) + Eq. (14); muon: the Eq. (6) comparison baseline (hidden weights only)")
+    ap.add_argument("--ns-single-launch", action="store_true",
+                    help="run all Newton-Schulz products in one cooperative launch (option ns_single_launch)")
     ap.add_argument("--ns-trajectory", type=int, default=0, metavar="K",
                     help="instead of the step, time the Section 3.1 CV replay of X_0..X_K (one matrix per shape)")
     args = ap.parse_args()
@@ -352,7 +354,8 @@ def main():
     grads = [[v.view(r, c) for v, (r, c) in zip(gv, shapes)] for _, gv in gbufs]
 
     rule = meq.RULE_MUON if args.update_rule == "muon" else meq.RULE_MEQMUON
-    opt = meq.MeqMuon(shapes, kinds=kinds, ns_fp16_mask=args.ns_fp16_mask, update_rule=rule)
+    opt = meq.MeqMuon(shapes, kinds=kinds, ns_fp16_mask=args.ns_fp16_mask, update_rule=rule,
+                      ns_single_launch=1 if args.ns_single_launch else 0)
     stream = torch.cuda.current_stream()
     for k in range(args.warmup):
         opt.step(params, grads[k % 2], LR, MU, WD, EPS)
@@ -493,12 +496,14 @@ def main():
                        "ns_steps": K, "ns_operands": "fp16" if args.ns_fp16_mask == 0xFFFFFFFF else hex(args.ns_fp16_mask),
                        "accumulate": "fp32", "l2": "inputs larger than L2 (params+grads+momentum %.2f GB)" % (12 * wl.numel / 1e9),
                        "parallelism": f"matrices split over {world} GPU(s)" if world > 1 else "single GPU",
-                       "update_rule": "Eq. (11) + Eq. (14)" if args.update_rule == "meqmuon" else "Eq. (6)"},
+                       "update_rule": "Eq. (11) + Eq. (14)" if args.update_rule == "meqmuon" else "Eq. (6)",
+                       "ns_launches_per_step": n_gemm_launches},
             "roofline": {
                 "bound": "tensor", "kernel": "ns_gemm_kernel",
                 "achieved": ns_tflops, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                 "frac": ns_tflops / peaks["bf16_tflops"], "peak_source": f"{peak_src} bf16 dense burst (fp16 rate = bf16 rate)",
-                "traffic": recorded_traffic(args.workload),
+                # the recorded capture is of the one-launch-per-product kernel
+                "traffic": recorded_traffic(args.workload) if n_gemm_launches > 1 else None,
                 "flops_per_launch": sym / max(n_gemm_launches, 1),
                 "avg_launch_ms": ph["ns_gemm"] / max(n_gemm_launches, 1),
                 "dense_equivalent_tflops": ns_dense_tflops,

@@ -498,8 +498,8 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
     }
   }
   // ns_single_launch: the per-product launches' groups become the segments of
-  // one tile queue in product order; a tile of product j waits until every
-  // epilogue warp of every tile of its matrix in product j - 1 has counted.
+  // one tile queue in product order; a tile of product j waits until both
+  // CTAs of every tile of its matrix in product j - 1 have counted it stored.
   st->use_persist = false;
   const int nprod = 3 * K;
   if (st->opt.ns_single_launch && pair == 2 && ng <= kMaxGroups && static_cast<int>(st->gemm.size()) == nprod &&
@@ -515,7 +515,7 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
           GemmGroup S = P.g[gi];
           S.tile_begin = tiles;
           S.prod = j;
-          S.dep_target = j == 0 ? 0 : st->gemm[j - 1].g[gi].tiles_per_mat * pair * kNsEpilogueWarps;
+          S.dep_target = j == 0 ? 0 : st->gemm[j - 1].g[gi].tiles_per_mat * pair;  // one count per CTA and tile
           // every output another tile waits for leaves by TMA stores, whose
           // completion a warp can wait for without waiting for later stores
           if (S.mode == MODE_XUPD) S.tma_out = 1;

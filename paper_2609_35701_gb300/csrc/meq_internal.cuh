@@ -23,6 +23,7 @@ enum DevErr : int {
   DEV_TIMEOUT_SCHED_PUT = 0x106, // tile scheduler waited too long for a free slot of the tile ring
   DEV_TIMEOUT_SCHED_TAKE = 0x107,// a role waited too long for its next tile index
   DEV_TIMEOUT_DEP = 0x108,       // one-launch NS: a tile waited too long for the product it reads
+  DEV_TIMEOUT_SIG = 0x109,       // one-launch NS: waited too long for a tile's stores or their report slot
   DEV_TIMEOUT_TEST = 0x1FF,      // the wait-timeout self test
 };
 

@@ -53,6 +53,14 @@ constexpr int BM = 128, BN = 256, BK = 64, UK = 16;  // per-CTA rows, tile colum
 constexpr int A_BYTES = BM * BK * 2;                 // 16 KB
 constexpr int NUM_EPI_WARPS = kNsEpilogueWarps;      // two per TMEM lane quarter
 constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
+// The one-launch NS adds two warps per CTA: one acquires each tile's
+// dependency ahead of the producer, one releases each tile's completion
+// count, so that neither GPU-scope operation sits on a producer or epilogue
+// path (a release stalls its warp for about 2 us).
+constexpr int NUM_THREADS_P = NUM_THREADS + 64;
+constexpr int DEP_WARP = 2 + NUM_EPI_WARPS, SIG_WARP = DEP_WARP + 1;
+constexpr int DEP_Q = 32;  // ring of "dependency acquired" barriers, one-launch NS
+constexpr int SIG_Q = 8;   // ring of "tile stored" barriers (and their free barriers), one-launch NS
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int SLOT_BYTES = 2048;                     // one 32 x 32 16-bit block (two per epilogue warp)
 constexpr int SCHED_D = 16;                          // entries of the tile-index ring
@@ -70,8 +78,9 @@ struct Cfg {
   static constexpr int B_BYTES = BN_LOCAL * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int STAGES = kPair == 1 ? 4 : 6;
-  // full, empty, tmem full x2, tmem empty x2, drain, tile ring full / empty
-  static constexpr int NUM_BARS = 2 * STAGES + 4 + 1 + 2 * SCHED_D;
+  // full, empty, tmem full x2, tmem empty x2, drain, tile ring full / empty,
+  // then (one-launch NS) dependency acquired, tile stored, stored slot free
+  static constexpr int NUM_BARS = 2 * STAGES + 4 + 1 + 2 * SCHED_D + DEP_Q + 2 * SIG_Q;
   static constexpr int SMEM_EPI_OFF = STAGES * STAGE_BYTES;
   static constexpr int SMEM_BAR_OFF = SMEM_EPI_OFF + NUM_EPI_WARPS * 2 * SLOT_BYTES;
   // barriers, the TMEM address word (16 bytes reserved), the tile ring
@@ -392,11 +401,10 @@ __device__ __forceinline__ void fill_half_rows(uint8_t* slot, int r, const float
   }
 }
 // The transposed block: element (row j, col r) = v[j] of lane r.
-// Transposes, in place, the 32 x 32 16-bit block a warp holds in its slot
-// (64-byte rows of four 16-byte chunks, chunk k of row r at k ^ ((r >> 1) & 3)):
+// Writes the transpose of the 32 x 32 16-bit block in `src` into `dst` (both
+// 64-byte rows of four 16-byte chunks, chunk k of row r at k ^ ((r >> 1) & 3)):
 // ldmatrix .trans reads each 8 x 8 sub-block (g, q) as its transpose and
-// stmatrix writes it back as sub-block (q, g). All reads finish before the
-// first write (the warp holds the whole block in registers in between).
+// stmatrix writes it as sub-block (q, g).
 __device__ __forceinline__ void transpose_slot(const uint8_t* src, uint8_t* dst, int lane) {
   const uint32_t base = smem_u32(src), dbase = smem_u32(dst);
   const int r8 = lane & 7, q = lane >> 3;
@@ -458,7 +466,8 @@ __device__ __forceinline__ void bulk_wait_keep(int keep) {
   }
 }
 template <int kPair, int kSegs>
-__global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_constant__ GemmParamsT<kSegs> p) {
+__global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREADS, 1)
+    ns_gemm_kernel(const __grid_constant__ GemmParamsT<kSegs> p) {
   // The one-launch NS (every product, completion counters) is the kMaxSegs
   // instantiation; the per-product launches compile without its code.
   constexpr bool kPersistent = kSegs == kMaxSegs;
@@ -480,6 +489,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
 #define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
 #define SFULL_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + (i)))
 #define SEMPTY_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + SCHED_D + (i)))
+#define DEPOK_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + 2 * SCHED_D + (i)))
+#define STORED_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + 2 * SCHED_D + DEP_Q + (i)))
+#define STFREE_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + 2 * SCHED_D + DEP_Q + SIG_Q + (i)))
   const uint32_t ring = tmem_slot + 16;  // SCHED_D tile indices
 
   const int warp = threadIdx.x >> 5;
@@ -505,8 +517,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     for (int i = 0; i < SCHED_D; ++i) {
       mbar_init(SFULL_BAR(i), 1);
       // consumers of each index: the MMA issuer and the epilogue warps of the
-      // leader, and (pair) the peer's producer and epilogue warps
-      mbar_init(SEMPTY_BAR(i), kPair * (1 + NUM_EPI_WARPS));
+      // leader, and (pair) the peer's producer and epilogue warps; the
+      // dependency and signal warps of both CTAs in the one-launch NS
+      mbar_init(SEMPTY_BAR(i), kPair * (1 + NUM_EPI_WARPS + (kPersistent ? 2 : 0)));
+    }
+    if (kPersistent) {
+      for (int i = 0; i < DEP_Q; ++i) mbar_init(DEPOK_BAR(i), 1);
+      for (int i = 0; i < SIG_Q; ++i) {
+        mbar_init(STORED_BAR(i), NUM_EPI_WARPS);
+        mbar_init(STFREE_BAR(i), 1);
+      }
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     for (int g = 0; g < p.ngroups; ++g) {
@@ -574,16 +594,34 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       bool ok = true;
       int t = unit;
       int fetched = 0;  // leader: the counter value for the next tile
+      int t_ahead = 0;  // leader, one-launch NS: index n + 1, published when tile n starts
       for (int n = 0; ok; ++n) {
-        if (n > 0 && leader) t = nunits + fetched;
-        if (leader ? !sched_put(n, t) : !sched_take(n, t)) break;
+        if (kPersistent && leader) {
+          // one tile ahead, so that the dependency warps see each index early
+          if (n == 0) {
+            if (!sched_put(0, t)) break;
+            if (t < p.total_tiles) {
+              t_ahead = nunits + atomicAdd(p.sched, 1);
+              if (!sched_put(1, t_ahead)) break;
+            }
+          } else {
+            t = t_ahead;
+            if (t < p.total_tiles) {
+              t_ahead = nunits + fetched;
+              if (!sched_put(n + 1, t_ahead)) break;
+            }
+          }
+        } else {
+          if (n > 0 && leader) t = nunits + fetched;
+          if (leader ? !sched_put(n, t) : !sched_take(n, t)) break;
+        }
         if (t >= p.total_tiles) break;
         const TileCoord c = decode_tile<kPair>(p, t);
         const GemmGroup& G = p.g[c.g];
-        if (kPersistent && G.dep_target > 0) {
-          // the previous product of this matrix is complete, and visible to TMA
-          if (!wait_count(p.done + (G.prod - 1) * p.nslots + G.mat_base + c.mat, G.dep_target, err, DEV_TIMEOUT_DEP,
-                          tmo)) {
+        if (kPersistent) {
+          // the previous product of this matrix is complete (acquired by the
+          // dependency warp), and visible to TMA
+          if (!wait_bounded(DEPOK_BAR(n % DEP_Q), (n / DEP_Q) & 1, err, DEV_TIMEOUT_DEP, tmo)) {
             ok = false;
             break;
           }
@@ -701,7 +739,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       wait_bounded(drain_bar, 0, err, DEV_TIMEOUT_DRAIN, tmo);
     }
     __syncwarp();
-  } else {
+  } else if (warp < 2 + NUM_EPI_WARPS) {
     // ------------------------------------------------------------------ epilogue
     // Warp ew (0..7) owns TMEM lanes 32*q .. +31 (q = warp % 4), i.e. rows
     // 32q .. 32q+31 of the tile, chunks ch with ch % 2 == half, and two 2 KB
@@ -723,22 +761,24 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     // The leader's tmem-empty barrier counts the epilogue warps of both CTAs.
     const uint32_t tempty_target0 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(0), 0) : TEMPTY_BAR(0);
     const uint32_t tempty_target1 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(1), 0) : TEMPTY_BAR(1);
-    // One-launch NS: each warp counts its part of a tile as done once the
-    // tile's stores have landed (release at GPU scope), for the next
-    // product's tiles of that matrix. The count of tile n is deferred to the
-    // end of tile n + 1's epilogue, by when tile n's stores have long
+    // One-launch NS: once a tile's stores have landed, each warp tells the
+    // signal warp (a CTA barrier per tile, in tile order), which releases the
+    // tile's count for the next product. The report of tile n is deferred to
+    // the end of tile n + 1's epilogue, by when tile n's stores have long
     // completed (the wait skips tile n + 1's own store groups) -- unless tile
     // n + 1's accumulator is not ready yet, in which case it is sent before
     // waiting (tile n + 1 may depend on it).
     // (Every output another tile waits for leaves by TMA stores: the host
     // sets tma_out on every product but the last.)
-    int pend = -1;  // completion counter of the tile awaiting its count
+    int pend = -1;  // ordinal of the tile whose report is deferred
     auto signal_pending = [&](int keep_groups) {
       __syncwarp();
       if (lane == 0) {
         bulk_wait_keep(keep_groups);
         fence_proxy_async_global();
-        red_release_gpu_add(p.done + pend, 1);
+        // the signal warp has consumed this slot's previous tile
+        wait_bounded(STFREE_BAR(pend % SIG_Q), ((pend / SIG_Q) & 1) ^ 1u, err, DEV_TIMEOUT_SIG, tmo);
+        mbar_arrive_local(STORED_BAR(pend % SIG_Q));  // release (CTA scope)
       }
       pend = -1;
     };
@@ -753,17 +793,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       const int mode = kPersistent ? G.mode : p.g[0].mode;  // one mode per launch (a launch-uniform read)
       if (pend >= 0 && !__all_sync(0xffffffffu, mbar_try_wait(TFULL_BAR(acc), acc_phase))) signal_pending(0);
       if (!wait_bounded_warp(TFULL_BAR(acc), acc_phase, err, DEV_TIMEOUT_EPI, tmo)) break;
-      if (kPersistent && mode == MODE_POLY && G.dep_target > 0) {
+      if (kPersistent && mode == MODE_POLY) {
         // The A read below comes from the previous product of this launch:
-        // acquire its completion. It is complete by now, since the tile's
-        // operands waited for it; waiting before the accumulator could
-        // deadlock (the count may still lack this warp's own deferred one).
+        // synchronise with the dependency warp's acquire of it (CTA scope).
+        // It is done by now, since the tile's operands waited for it; waiting
+        // before the accumulator could deadlock (the count may still lack
+        // this warp's own deferred report).
         int okd = 1;
-        if (lane == 0)
-          okd = wait_count(p.done + (G.prod - 1) * p.nslots + G.mat_base + c.mat, G.dep_target, err, DEV_TIMEOUT_DEP,
-                           tmo)
-                    ? 1
-                    : 0;
+        if (lane == 0) okd = wait_bounded(DEPOK_BAR(n % DEP_Q), (n / DEP_Q) & 1, err, DEV_TIMEOUT_DEP, tmo) ? 1 : 0;
         if (!__shfl_sync(0xffffffffu, okd, 0)) break;
       }
       tc_fence_after();
@@ -908,11 +945,45 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
-      if (kPersistent && G.prod + 1 < p.nprod) pend = G.prod * p.nslots + G.mat_base + c.mat;
+      if (kPersistent) pend = n;
     }
     if (pend >= 0) signal_pending(0);
     // The outputs are in global memory before the CTA leaves.
     if (lane == 0) bulk_wait_all();
+    __syncwarp();
+  } else if (kPersistent && warp == DEP_WARP) {
+    // ---------------------------------------------------------------- dependency warp (one-launch NS)
+    // Acquires (GPU scope) the completion count each tile depends on, one
+    // tile ahead of the producer, and hands it on by a CTA barrier that the
+    // producer and the polynomial epilogue wait on.
+    if (lane == 0) {
+      for (int n = 0;; ++n) {
+        int t = 0;
+        if (!sched_take(n, t) || t >= p.total_tiles) break;
+        const TileCoord c = decode_tile<kPair>(p, t);
+        const GemmGroup& G = p.g[c.g];
+        if (G.dep_target > 0 &&
+            !wait_count(p.done + (G.prod - 1) * p.nslots + G.mat_base + c.mat, G.dep_target, err, DEV_TIMEOUT_DEP, tmo))
+          break;
+        mbar_arrive_local(DEPOK_BAR(n % DEP_Q));  // release (CTA scope)
+      }
+    }
+    __syncwarp();
+  } else if (kPersistent && warp == SIG_WARP) {
+    // ---------------------------------------------------------------- signal warp (one-launch NS)
+    // Once every epilogue warp of this CTA reports a tile stored, adds one to
+    // the tile's matrix count (release, GPU scope) for the next product.
+    if (lane == 0) {
+      for (int n = 0;; ++n) {
+        int t = 0;
+        if (!sched_take(n, t) || t >= p.total_tiles) break;
+        const TileCoord c = decode_tile<kPair>(p, t);
+        const GemmGroup& G = p.g[c.g];
+        if (!wait_bounded(STORED_BAR(n % SIG_Q), (n / SIG_Q) & 1, err, DEV_TIMEOUT_SIG, tmo)) break;
+        if (G.prod + 1 < p.nprod) red_release_gpu_add(p.done + G.prod * p.nslots + G.mat_base + c.mat, 1);
+        mbar_arrive_local(STFREE_BAR(n % SIG_Q));
+      }
+    }
     __syncwarp();
   }
 #undef FULL_BAR
@@ -921,6 +992,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
 #undef TEMPTY_BAR
 #undef SFULL_BAR
 #undef SEMPTY_BAR
+#undef DEPOK_BAR
+#undef STORED_BAR
+#undef STFREE_BAR
 
   if (kPair == 2 && *reinterpret_cast<volatile int*>(err) != 0) {
     // After an early exit, give copies still in flight towards either CTA
@@ -979,7 +1053,7 @@ cudaError_t launch_ns_gemm(const GemmParams& p, int grid, int pair, cudaStream_t
 int ns_gemm_persistent_max_pairs() {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2);
-  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.blockDim = dim3(NUM_THREADS_P);
   cfg.dynamicSmemBytes = Cfg<2>::SMEM_BYTES;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -1001,7 +1075,7 @@ int ns_gemm_persistent_max_pairs() {
 cudaError_t launch_ns_gemm_persistent(const PersistParams& p, int grid, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.blockDim = dim3(NUM_THREADS_P);
   cfg.dynamicSmemBytes = Cfg<2>::SMEM_BYTES;
   cfg.stream = st;
   cudaLaunchAttribute attr[3];
