@@ -20,7 +20,7 @@
 // X is stored scaled by a power of two alpha so its entries stay in the
 // normal range of fp16; the epilogues undo the scale in fp32.
 //
-// Roles (320 threads, one CTA per SM):
+// Roles (320 threads, one CTA per SM; one-launch NS below):
 //   warp 0 : TMA producer (one thread), shared-memory ring of 4 stages
 //            (single CTA) or 6 (CTA pair)
 //   warp 1 : TMEM allocator and tcgen05.mma issuer (one thread; with CTA
@@ -39,6 +39,14 @@
 // swizzled shared memory; the symmetric A and P (each block stored twice)
 // leave by TMA stores, X and U by coalesced 16-byte stores from the threads
 // (the update launches keep the SM's TMA unit for their operand loads).
+//
+// The same kernel, instantiated with kMaxSegs segments and two more warps
+// (384 threads), runs every product of the iteration in one cooperative
+// launch (option ns_single_launch): the products' shape groups are segments
+// of one tile queue in product order, a dependency warp acquires for each
+// tile the completion count of its matrix in the previous product before the
+// producer may load it, and a signal warp releases a tile's count once the
+// CTA's epilogue warps report its TMA stores landed.
 //
 // Every mbarrier wait is bounded (time and iteration count). On expiry the
 // waiting role records an error code, the others see it and stop, in-flight
