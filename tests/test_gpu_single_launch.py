@@ -59,6 +59,8 @@ def _assert_same(a, b):
     ([(64, 64), (129, 385), (385, 129), (256, 1000), (1000, 64)], 3),
     # one matrix: every product waits on the previous one
     ([(256, 256)], 5),
+    # several waves of tiles per product launch (Llama-130M-sized groups)
+    ([(768, 768)] * 48 + [(768, 2048)] * 12, 5),
 ])
 def test_single_launch_bitwise(meq, shapes, ns_steps):
     wl = W.custom_workload(shapes, pattern="both", seed=11)
