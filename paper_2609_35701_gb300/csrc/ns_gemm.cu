@@ -880,11 +880,25 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
         }
         if (mode == MODE_XLAST) {
           // U is stored as fp16(kUScale U). The sums of squares are taken from
-          // those stored values (v holds them exactly) and scaled back by
-          // kUScale^-2 (a power of two) when written, so the statistics
-          // describe the U the update applies.
+          // those stored values and scaled back by kUScale^-2 (a power of
+          // two) when written, so the statistics describe the U the update
+          // applies. Each pair is rounded once: the packed halves go to the
+          // staging slot, their exact fp32 values back into v.
 #pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] = __half2float(__float2half_rn(v[j] * kUScale));
+          for (int k = 0; k < 4; ++k) {
+            uint32_t wv[4];
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+              const int j = 8 * k + 2 * h;
+              const __half2 hh = __floats2half2_rn(v[j] * kUScale, v[j + 1] * kUScale);
+              wv[h] = *reinterpret_cast<const uint32_t*>(&hh);
+              const float2 f = __half22float2(hh);
+              v[j] = f.x;
+              v[j + 1] = f.y;
+            }
+            *reinterpret_cast<uint4*>(slot + lane * 64 + ((k ^ ((lane >> 1) & 3)) << 4)) =
+                make_uint4(wv[0], wv[1], wv[2], wv[3]);
+          }
           // Column sums of squares over the warp's 32 rows: transpose-reduce
           // so that lane j ends with the sum for column col0 + j.
           float sq[32];
@@ -906,8 +920,8 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
           if (col0 + lane < G.N)
             G.cpart[(static_cast<int64_t>(c.mat) * ((G.M + 31) / 32) + R) * G.N + col0 + lane] = sq[0] * kUInvScale2;
           // 8-element chunks that start below the row length stay inside the
-          // padded row (stride = row length rounded up to 8)
-          fill_half_rows(slot, lane, v, 1);
+          // padded row (stride = row length rounded up to 8); the slot holds
+          // the block (filled above)
           __syncwarp();
           if (!G.trans) {
             // U rows = NS rows row0 + r, U columns = NS columns col0 + j
