@@ -497,6 +497,19 @@ __global__ void __launch_bounds__(kThreads) cast_x0_kernel(const MatInfo* __rest
 
 // ----------------------------------------------------------------- statistics
 // Two-pass fp32 CV of Eq. (8) over the entries of v above delta.
+// sum_{k < count} p[k * stride] with eight independent partial sums (term k
+// goes to partial k % 8) so that the loads overlap; fixed order.
+__device__ __forceinline__ float strided_sum8(const float* __restrict__ p, int64_t count, int64_t stride) {
+  float a8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  int64_t k = 0;
+  for (; k + 8 <= count; k += 8) {
+#pragma unroll
+    for (int u = 0; u < 8; ++u) a8[u] += p[(k + u) * stride];
+  }
+  for (; k < count; ++k) a8[k & 7] += p[k * stride];
+  return ((a8[0] + a8[1]) + (a8[2] + a8[3])) + ((a8[4] + a8[5]) + (a8[6] + a8[7]));
+}
+
 __device__ float block_cv(const float* v, int64_t len, float delta, float* shf) {
   float cnt = 0.f, sum = 0.f;
   for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
@@ -561,19 +574,10 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
       r[i] = rms;
       s[i] = rms > delta ? 1.0f / rms : 0.f;
     }
-    // Column sums over the slabs, eight independent partial sums per thread
-    // (slab k goes to accumulator k % 8) so loads overlap; fixed order.
+    // column sums over the slabs
     const int64_t nslabs = (M.m + kColSlab - 1) / kColSlab;
     for (int64_t j = threadIdx.x; j < M.n; j += blockDim.x) {
-      const float* pj = parts + M.cpart_off + j;
-      float a8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      int64_t k = 0;
-      for (; k + 8 <= nslabs; k += 8) {
-#pragma unroll
-        for (int u = 0; u < 8; ++u) a8[u] += pj[(k + u) * M.n];
-      }
-      for (; k < nslabs; ++k) a8[k & 7] += pj[k * M.n];
-      const float tot = ((a8[0] + a8[1]) + (a8[2] + a8[3])) + ((a8[4] + a8[5]) + (a8[6] + a8[7]));
+      const float tot = strided_sum8(parts + M.cpart_off + j, nslabs, M.n);
       const float rms = sqrtf(tot * inv_m);
       c[j] = rms;
       t[j] = rms > delta ? 1.0f / rms : 0.f;
@@ -592,14 +596,12 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
   const int64_t tiles_n = 2 * ((M.l + 255) / 256);  // two epilogue halves per 256-column tile
   const int64_t nrb = (M.s + 31) / 32;
   for (int64_t i = threadIdx.x; i < M.s; i += blockDim.x) {
-    float acc = 0.f;
-    for (int64_t t = 0; t < tiles_n; ++t) acc += parts[M.rpart_off + t * M.s + i];
+    const float acc = strided_sum8(parts + M.rpart_off + i, tiles_n, M.s);
     if (!M.trans) r[i] = sqrtf(acc * inv_n);
     else c[i] = sqrtf(acc * inv_m);
   }
   for (int64_t j = threadIdx.x; j < M.l; j += blockDim.x) {
-    float acc = 0.f;
-    for (int64_t k = 0; k < nrb; ++k) acc += parts[M.cpart_off + k * M.l + j];
+    const float acc = strided_sum8(parts + M.cpart_off + j, nrb, M.l);
     if (!M.trans) c[j] = sqrtf(acc * inv_m);
     else r[j] = sqrtf(acc * inv_n);
   }
