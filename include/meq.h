@@ -83,6 +83,13 @@ typedef struct {
                              else the step keeps one launch per product
                              (meq_ns_gemm_launches_per_step tells which). 0 (default): one
                              launch per product. */
+  int debug_skip_load;    /* 1 (tests only): in every step's first NS launch, the leader
+                             CTA of the first CTA pair arms its first operand stage but
+                             does not load its half, so that stage never completes: the
+                             MMA issuer's bounded wait expires, every role of the launch
+                             stops and drains, and meq_sync reports MEQ_ERR_TIMEOUT (the
+                             results of that step are not meaningful). Requires
+                             ns_cta_pair = 1 and ns_single_launch = 0. Default 0. */
 } meq_options;
 
 /* Update applied to the hidden 2D weights after momentum and Newton-Schulz. */

@@ -178,6 +178,11 @@ bool valid_options(const meq_options& o, std::string* why) {
   if (o.ns_x0_fused != 0 && o.ns_x0_fused != 1) { *why = "ns_x0_fused must be 0 or 1"; return false; }
   if (o.debug_canaries != 0 && o.debug_canaries != 1) { *why = "debug_canaries must be 0 or 1"; return false; }
   if (o.ns_single_launch != 0 && o.ns_single_launch != 1) { *why = "ns_single_launch must be 0 or 1"; return false; }
+  if (o.debug_skip_load != 0 && o.debug_skip_load != 1) { *why = "debug_skip_load must be 0 or 1"; return false; }
+  if (o.debug_skip_load && (!o.ns_cta_pair || o.ns_single_launch)) {
+    *why = "debug_skip_load requires ns_cta_pair = 1 and ns_single_launch = 0";
+    return false;
+  }
   if (o.update_rule != MEQ_RULE_MEQMUON && o.update_rule != MEQ_RULE_MUON) {
     *why = "update_rule must be MEQ_RULE_MEQMUON or MEQ_RULE_MUON";
     return false;
@@ -491,6 +496,7 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
         // before it (the X_0 cast writes in forward order), so it begins with
         // the outputs still resident in L2.
         P.reverse = (st->gemm.size() % 2 == 0) ? 1 : 0;
+        P.debug_skip_load = (st->opt.debug_skip_load && st->gemm.empty()) ? 1 : 0;
         st->gemm.push_back(P);
         // persistent grid: one CTA (pair) per SM (pair of SMs), never more than the tiles
         st->gemm_grid.push_back(pair * std::max(1, std::min(tiles, st->num_sms / pair)));
@@ -563,6 +569,7 @@ void meq_default_options(meq_options* o) {
   o->ns_x0_fused = 1;
   o->debug_canaries = 0;
   o->ns_single_launch = 0;
+  o->debug_skip_load = 0;
 }
 
 const char* meq_status_string(meq_status s) {

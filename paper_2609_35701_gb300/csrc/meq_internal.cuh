@@ -135,6 +135,7 @@ struct GemmParamsT {
                            // zero between launches (reset with the tile queue)
   int32_t nslots;          // slots per product row of `done`
   int32_t nprod;           // product rows of `done`
+  int32_t debug_skip_load; // tests: the first pair's leader skips its first stage's loads
   unsigned long long timeout_ns;
 };
 using GemmParams = GemmParamsT<kMaxGroups>;

@@ -140,6 +140,20 @@ __device__ bool wait_bounded(uint32_t bar, uint32_t parity, int* err, int code, 
   }
 }
 
+// Bounded wait that does not stop early on another role's error: for the
+// MMA issuer's drain, which must see its MMAs complete before TMEM is freed
+// (they always do, so the bound is a safety net only).
+__device__ bool wait_bounded_drain(uint32_t bar, uint32_t parity, int* err, int code, uint64_t timeout_ns) {
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 0;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 127u) == 127u && (global_ns() - t0 > timeout_ns || it >= (1u << 28))) {
+      atomicCAS(err, 0, code);
+      return false;
+    }
+  }
+}
+
 // Warp-uniform bounded wait (all 32 lanes call it; all get the same answer).
 __device__ bool wait_bounded_warp(uint32_t bar, uint32_t parity, int* err, int code, uint64_t timeout_ns) {
   const unsigned FULL = 0xffffffffu;
@@ -667,13 +681,18 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
             // the leader arms with the bytes of both.
             if (leader) mbar_expect_tx(FULL_BAR(stage), 2 * STAGE_BYTES);
             const uint32_t fb = leader ? FULL_BAR(stage) : map_to_rank(FULL_BAR(stage), 0);
-            tma_load_3d_pair(sa, &G.tmA, fb, kb * BK, arow, c.mat);
-            if (!b_mn_major) {
-              tma_load_3d_pair(sb, &G.tmB, fb, kb * BK, bcol, c.mat);
-            } else {
+            // tests (debug_skip_load): the stage is armed but this CTA's half never
+            // comes, so the MMA issuer's bounded wait on it expires
+            const bool skip = !kPersistent && p.debug_skip_load && leader && unit == 0 && n == 0 && kb == 0;
+            if (!skip) {
+              tma_load_3d_pair(sa, &G.tmA, fb, kb * BK, arow, c.mat);
+              if (!b_mn_major) {
+                tma_load_3d_pair(sb, &G.tmB, fb, kb * BK, bcol, c.mat);
+              } else {
 #pragma unroll
-              for (int j = 0; j < C_::BN_LOCAL / 64; ++j)
-                tma_load_3d_pair(sb + j * (64 * BK * 2), &G.tmB, fb, bcol + j * 64, kb * BK, c.mat);
+                for (int j = 0; j < C_::BN_LOCAL / 64; ++j)
+                  tma_load_3d_pair(sb + j * (64 * BK * 2), &G.tmB, fb, bcol + j * 64, kb * BK, c.mat);
+              }
             }
           }
           issued_mask |= 1u << stage;
@@ -744,7 +763,7 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
       // Drain: all MMAs issued by this thread are complete before TMEM is freed.
       if (kPair == 2) tc_commit_pair_local(drain_bar);
       else tc_commit(drain_bar);
-      wait_bounded(drain_bar, 0, err, DEV_TIMEOUT_DRAIN, tmo);
+      wait_bounded_drain(drain_bar, 0, err, DEV_TIMEOUT_DRAIN, tmo);
     }
     __syncwarp();
   } else if (warp < 2 + NUM_EPI_WARPS) {

@@ -44,6 +44,7 @@ class MeqOptions(ctypes.Structure):
         ("update_rule", ctypes.c_int),
         ("debug_canaries", ctypes.c_int),
         ("ns_single_launch", ctypes.c_int),
+        ("debug_skip_load", ctypes.c_int),
     ]
 
 

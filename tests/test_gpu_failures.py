@@ -117,3 +117,47 @@ def test_canary_check_detects_a_change(meq):
         opt.check_canaries()
     assert e.value.status == 7
     opt.close()
+
+
+def test_ns_gemm_stage_that_never_fills(meq):
+    """debug_skip_load: in the first NS launch one operand stage is armed but
+    half its bytes never come. The MMA issuer's bounded wait expires, every
+    role of every CTA stops and drains (the MMA issuer waits for its issued
+    MMAs before TMEM is freed), meq_sync reports MEQ_ERR_TIMEOUT and clears
+    it, and the GPU context stays usable: a clean state then steps exactly as
+    a clean state did before the fault."""
+    import torch
+
+    shapes = [(512, 768), (768, 512), (256, 256)]
+    wl = W.custom_workload(shapes, pattern="both", seed=23)
+
+    def clean_run():
+        opt = meq.MeqMuon(shapes)
+        params = [w.cuda() for w in W.initial_weights(wl)]
+        for t in range(2):
+            opt.step(params, [g.cuda() for g in W.gradients(wl, t)], LR, MU, WD, EPS)
+        opt.sync()
+        out = [p.cpu().numpy() for p in params]
+        opt.close()
+        return out
+
+    before = clean_run()
+    opt = meq.MeqMuon(shapes, debug_skip_load=1, wait_timeout_ms=200.0, use_graph=0)
+    params = [w.cuda() for w in W.initial_weights(wl)]
+    opt.step(params, [g.cuda() for g in W.gradients(wl, 0)], LR, MU, WD, EPS)
+    with pytest.raises(meq.MeqError) as e:
+        opt.sync()
+    assert e.value.status == 5, str(e.value)  # MEQ_ERR_TIMEOUT
+    opt.sync()  # cleared by the report
+    opt.close()
+    torch.cuda.synchronize()
+    after = clean_run()
+    for i in range(len(shapes)):
+        assert np.array_equal(before[i], after[i]), f"matrix {i} differs after the timeout"
+
+
+def test_debug_skip_load_validation(meq):
+    with pytest.raises(meq.MeqError):
+        meq.MeqMuon([(64, 64)], debug_skip_load=1, ns_cta_pair=0)
+    with pytest.raises(meq.MeqError):
+        meq.MeqMuon([(64, 64)], debug_skip_load=1, ns_single_launch=1)

@@ -101,7 +101,7 @@ def test_host_validation_errors():
     p0, w0 = meq.state_bytes([(300, 200), (1, 64)], kinds=[meq.HIDDEN, meq.VECTOR])
     p1, w1 = meq.state_bytes([(300, 200), (1, 64)], kinds=[meq.HIDDEN, meq.VECTOR], debug_canaries=1)
     assert p1 == p0 and w1 > w0  # guard bands are workspace only
-    for field in ("ns_cta_pair", "ns_x0_fused", "update_rule", "debug_canaries", "ns_single_launch"):
+    for field in ("ns_cta_pair", "ns_x0_fused", "update_rule", "debug_canaries", "ns_single_launch", "debug_skip_load"):
         with pytest.raises(meq.MeqError):
             meq.state_bytes([(4, 4)], **{field: 2})
     # Eq. (6) is the hidden-weight baseline only
