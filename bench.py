@@ -421,9 +421,8 @@ def main():
             hg.append(h)
         hp = torch.empty(pbuf.numel(), dtype=torch.float32, pin_memory=True)
         n_e2e = max(3, min(args.steps, 50))
-        # Copies move in pieces of COPY_CHUNK elements (a single copy of
-        # hundreds of MB runs at half the rate of the same bytes in pieces on
-        # this host link), on two copy streams: the gradients of step k go up
+        # Copies move in pieces of COPY_CHUNK elements on two copy streams,
+        # so that the two directions share the host link: the gradients of step k go up
         # while step k - 1 runs; the parameters of step k - 1 come back while
         # step k's momentum, Newton-Schulz and statistics run
         # (meq_step_prepare), and step k's update (meq_step_apply) waits for
