@@ -496,7 +496,6 @@ __global__ void __launch_bounds__(kThreads) cast_x0_kernel(const MatInfo* __rest
 }
 
 // ----------------------------------------------------------------- statistics
-// Two-pass fp32 CV of Eq. (8) over the entries of v above delta.
 // sum_{k < count} p[k * stride] with eight independent partial sums (term k
 // goes to partial k % 8) so that the loads overlap; fixed order.
 __device__ __forceinline__ float strided_sum8(const float* __restrict__ p, int64_t count, int64_t stride) {
@@ -510,22 +509,62 @@ __device__ __forceinline__ float strided_sum8(const float* __restrict__ p, int64
   return ((a8[0] + a8[1]) + (a8[2] + a8[3])) + ((a8[4] + a8[5]) + (a8[6] + a8[7]));
 }
 
-__device__ float block_cv(const float* v, int64_t len, float delta, float* shf) {
-  float cnt = 0.f, sum = 0.f;
-  for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
-    const float x = v[i];
-    if (x > delta) cnt += 1.f, sum += x;
+// K block sums at once: each value goes through the same warp tree and the
+// same in-order sum over warps as block_sum_f32 gives it alone, with one set
+// of barriers for all of them. sh holds at least 33 * K floats.
+template <int K>
+__device__ __forceinline__ void block_sum_multi(float (&v)[K], float* sh) {
+  const unsigned FULL = 0xffffffffu;
+#pragma unroll
+  for (int k = 0; k < K; ++k)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(FULL, v[k], o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) {
+#pragma unroll
+    for (int k = 0; k < K; ++k) sh[32 * k + w] = v[k];
   }
-  cnt = block_sum_f32(cnt, shf);
-  sum = block_sum_f32(sum, shf);
-  const float mean = cnt > 0.f ? sum / cnt : 0.f;
-  float var = 0.f;
-  for (int64_t i = threadIdx.x; i < len; i += blockDim.x) {
-    const float x = v[i];
-    if (x > delta) var += (x - mean) * (x - mean);
+  __syncthreads();
+  if (threadIdx.x < K) {
+    float r = 0.f;
+    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) r += sh[32 * threadIdx.x + i];
+    sh[32 * K + threadIdx.x] = r;
   }
-  var = block_sum_f32(var, shf);
-  return cnt > 0.f ? sqrtf(var / cnt) / mean : 0.f;
+  __syncthreads();
+#pragma unroll
+  for (int k = 0; k < K; ++k) v[k] = sh[32 * K + k];
+}
+
+// Two-pass fp32 CVs of Eq. (8) of a (length la) and b (length lb) over their
+// entries above delta, both at once: the mean pass, then the squared
+// deviations.
+__device__ void block_cv2(const float* a, int64_t la, const float* b, int64_t lb, float delta, float* sh, float* ga,
+                          float* gb) {
+  float p[4] = {0.f, 0.f, 0.f, 0.f};  // count and sum over a, then over b
+  for (int64_t i = threadIdx.x; i < la; i += blockDim.x) {
+    const float x = a[i];
+    if (x > delta) p[0] += 1.f, p[1] += x;
+  }
+  for (int64_t i = threadIdx.x; i < lb; i += blockDim.x) {
+    const float x = b[i];
+    if (x > delta) p[2] += 1.f, p[3] += x;
+  }
+  block_sum_multi<4>(p, sh);
+  const float mean_a = p[0] > 0.f ? p[1] / p[0] : 0.f;
+  const float mean_b = p[2] > 0.f ? p[3] / p[2] : 0.f;
+  float q[2] = {0.f, 0.f};
+  for (int64_t i = threadIdx.x; i < la; i += blockDim.x) {
+    const float x = a[i];
+    if (x > delta) q[0] += (x - mean_a) * (x - mean_a);
+  }
+  for (int64_t i = threadIdx.x; i < lb; i += blockDim.x) {
+    const float x = b[i];
+    if (x > delta) q[1] += (x - mean_b) * (x - mean_b);
+  }
+  block_sum_multi<2>(q, sh);
+  *ga = p[0] > 0.f ? sqrtf(q[0] / p[0]) / mean_a : 0.f;
+  *gb = p[2] > 0.f ? sqrtf(q[1] / p[2]) / mean_b : 0.f;
 }
 
 // Statistics and normalisation scales, one block per parameter.
@@ -546,7 +585,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
                                                                int* __restrict__ nonfinite) {
   pdl_allow_dependents();
   pdl_wait_predecessor();
-  __shared__ float shf[32];
+  __shared__ float shf[33 * 4];
   const MatInfo& M = mats[blockIdx.x];
   const float delta = sc->eps;
   float* r = rvec + M.vec_off;
@@ -583,8 +622,8 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
       t[j] = rms > delta ? 1.0f / rms : 0.f;
     }
     __syncthreads();
-    const float gr = block_cv(r, M.m, delta, shf);
-    const float gc = block_cv(c, M.n, delta, shf);
+    float gr, gc;
+    block_cv2(r, M.m, c, M.n, delta, shf, &gr, &gc);
     if (threadIdx.x == 0) {
       stats[blockIdx.x].gamma_r = static_cast<double>(gr);
       stats[blockIdx.x].gamma_c = static_cast<double>(gc);
@@ -608,8 +647,8 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const MatInfo* __
   __syncthreads();
   // Eq. (8) over entries > delta: two passes (mean, then squared deviations),
   // fp32 with fixed-order block reductions.
-  const float gam0 = block_cv(r, M.m, delta, shf);
-  const float gam1 = block_cv(c, M.n, delta, shf);
+  float gam0, gam1;
+  block_cv2(r, M.m, c, M.n, delta, shf, &gam0, &gam1);
   int dir;
   if (sc->rule == 1) {
     // Eq. (6): every row scaled by sqrt(max(m, n)), no equilibration
