@@ -134,7 +134,7 @@ meq_status meq_init_state(const meq_shape* shapes, int n, const meq_options* opt
 
 /* As meq_init_state, with a parameter type (meq_kind) per entry, so one state
  * runs Algorithm 1 over every trainable parameter of a model: hidden 2D
- * weights, the remaining 2D parameters and 1D parameters (shape (1, d)).
+ * weights, the other 2D parameters, and vectors (shape (1, d)).
  * kinds is copied; NULL means all MEQ_KIND_HIDDEN. */
 meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n,
                                 const meq_options* opt, void* cuda_stream, meq_state** out);

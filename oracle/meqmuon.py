@@ -32,7 +32,7 @@ Readings of points the paper leaves open (each one is listed with its
 justification in the design notes of the repository):
   * Zero input to NS: the paper defines the iteration for a nonzero input
     only (Section 2); a zero momentum matrix gives U = 0.
-  * Rows / columns whose RMS is at or below delta are "treated as zero"
+  * A row / column RMS that does not exceed delta counts as zero
     (Section 3.1): they are excluded from the CVs and their normalisation
     scale is 0, so they contribute no update.
   * Ties in Eq. (11): row is chosen when gamma_r >= gamma_c - tie_atol, with
@@ -51,7 +51,7 @@ import numpy as np
 # Section 4 (5 iterations with these coefficients).
 NS_COEFFS = (3.4445, -4.7750, 2.0315)
 NS_STEPS = 5
-# RMS threshold delta of Section 3.1 (values at or below it are treated as zero).
+# RMS threshold delta of Section 3.1 (an RMS that does not exceed it counts as zero).
 DELTA = 1e-7
 # RMS alignment coefficient rho, Section 4.
 RHO = 0.2
