@@ -466,8 +466,13 @@ def main():
             t = torch.tensor([e2e_ms], device=dev)
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
             e2e_ms = float(t.item())
-        e2e = {"value": e2e_ms, "unit": "ms/step", "h2d_bytes_per_step": 4 * numel * (world if world > 1 else 1),
-               "d2h_bytes_per_step": 4 * numel * (world if world > 1 else 1), "steps": n_e2e,
+        numel_job = numel   # elements of every rank's matrices: the whole job's copies
+        if world > 1:
+            t = torch.tensor([float(numel)], dtype=torch.float64, device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.SUM)
+            numel_job = int(t.item())
+        e2e = {"value": e2e_ms, "unit": "ms/step", "h2d_bytes_per_step": 4 * numel_job,
+               "d2h_bytes_per_step": 4 * numel_job, "steps": n_e2e,
                "api": "meq_step_prepare + meq_step_apply (parameter read-back of step k - 1 overlaps step k's prepare)"}
     opt.sync()
 
