@@ -35,6 +35,7 @@ LR, MU, WD, EPS = 0.02, 0.95, 0.1, 1e-7
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 BW_BYTES_PER_ELEM = 24  # read G, B; write B; write X_0 (2 B); read U (2 B); read + write W
 REFERENCE_BUDGET_S = 150.0   # wall-clock cap on the timed oracle samples of --impl reference
+METRIC = "MeqMuon step ms per model; NS TFLOP/s & equilibration GB/s as % of GB300 peak"
 COPY_CHUNK = 8 << 20          # elements (32 MB) per host <-> device copy of the end-to-end loop
 
 
@@ -218,7 +219,7 @@ def run_reference(args):
     sample = (f"one matrix per shape class ({', '.join(sampled)}) per step, fp64 oracle, "
               f"extrapolated by class counts to all {len(wl.shapes)} matrices")
     line = {
-        "impl": "reference", "metric": "MeqMuon optimizer step time (all hidden 2D weights)", "value": v,
+        "impl": "reference", "metric": METRIC, "value": v,
         "unit": "ms/step", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": v, "higher_is_better": False, "scaling": "strong", "vs_baseline": None, "dtype": "f64",
         "timed_steps": len(vals), "data": "synthetic", "config": {"workload": args.workload, "matrices": len(wl.shapes), "elements": wl.numel,
@@ -491,7 +492,7 @@ def main():
 
     if rank == 0:
         line = {
-            "metric": "MeqMuon optimizer step time (all hidden 2D weights)",
+            "metric": METRIC,
             "value": ms, "unit": "ms/step", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": ms, "higher_is_better": False, "scaling": "strong", "vs_baseline": None,
             "dtype": "fp16" if args.ns_fp16_mask == 0xFFFFFFFF else ("bf16" if args.ns_fp16_mask == 0 else "bf16/fp16"),
