@@ -178,6 +178,9 @@ def state_bytes(shapes, kinds=None, **opts):
 def ns_cv_trajectory(H, steps=20, eps=1e-7, stream=None, **opts):
     """(gamma_r, gamma_c) of the NS iterates X_0..X_steps of a CUDA fp32
     matrix H (meq_ns_cv_trajectory)."""
+    if H.dim() != 2:
+        raise ValueError("H must be a matrix")
+    _require_cuda(H, "float32", H.shape[0] * H.shape[1], "H")
     gr = (ctypes.c_double * (steps + 1))()
     gc = (ctypes.c_double * (steps + 1))()
     o = default_options(**opts)
@@ -193,10 +196,28 @@ def row_col_stats_noalloc(U, r, c, gammas, direction, eps=1e-7, tie_atol=1e-6, s
     r (rows), c (cols), gammas (2 x float64) and direction (1 x int32),
     without any device allocation (see include/meq.h). Returns the status."""
     rows, cols = U.shape
+    _require_cuda(U, "float32", rows * cols, "U")
+    _require_cuda(r, "float32", rows, "r", U.device.index)
+    _require_cuda(c, "float32", cols, "c", U.device.index)
+    _require_cuda(gammas, "float64", 2, "gammas", U.device.index)
+    _require_cuda(direction, "int32", 1, "direction", U.device.index)
     return lib.meq_row_col_stats_noalloc(ctypes.c_void_p(U.data_ptr()), rows, cols, float(eps), float(tie_atol),
                                          ctypes.c_void_p(r.data_ptr()), ctypes.c_void_p(c.data_ptr()),
                                          ctypes.c_void_p(gammas.data_ptr()), ctypes.c_void_p(direction.data_ptr()),
                                          _stream_handle(stream))
+
+
+def _require_cuda(t, dtype_name, numel, what, device=None):
+    """Raises unless t is a contiguous CUDA tensor of the given dtype (a
+    torch dtype name) and element count (on `device` when given): the library
+    only sees a pointer, so a tensor of the wrong size or type would be read
+    or written past its end."""
+    if not t.is_cuda or str(t.dtype) != "torch." + dtype_name or not t.is_contiguous():
+        raise ValueError(f"{what} must be a contiguous {dtype_name} CUDA tensor")
+    if t.numel() != numel:
+        raise ValueError(f"{what} has {t.numel()} elements, expected {numel}")
+    if device is not None and t.device.index != device:
+        raise ValueError(f"{what} is on cuda:{t.device.index}, the state on cuda:{device}")
 
 
 def _stream_handle(stream):
@@ -217,6 +238,9 @@ class MeqMuon:
         self.kinds = [HIDDEN] * len(self.shapes) if kinds is None else [int(k) for k in kinds]
         self._shape_arr = _shape_array(self.shapes)
         self._opts = default_options(**opts)
+        import torch
+
+        self._device = torch.cuda.current_device()  # the state lives on the current device
         self._st = ctypes.c_void_p()
         s = lib.meq_init_state_kinds(self._shape_arr, _kind_array(self.kinds, len(self.shapes)), len(self.shapes),
                                      ctypes.byref(self._opts), _stream_handle(stream), ctypes.byref(self._st))
@@ -250,24 +274,21 @@ class MeqMuon:
         """One step on lists of contiguous fp32 CUDA tensors (params updated in place)."""
         if len(params) != len(self.shapes) or len(grads) != len(self.shapes):
             raise ValueError("params / grads must have one tensor per matrix")
-        for t in list(params) + list(grads):
-            if not t.is_cuda or t.dtype.itemsize != 4 or not t.is_contiguous():
-                raise ValueError("params and grads must be contiguous fp32 CUDA tensors")
+        self._check_tensors(params, "params")
+        self._check_tensors(grads, "grads")
         self.step_ptrs([p.data_ptr() for p in params], [g.data_ptr() for g in grads], lr, momentum, weight_decay,
                        eps, stream)
 
-    @staticmethod
-    def _check_tensors(ts):
-        for t in ts:
-            if not t.is_cuda or t.dtype.itemsize != 4 or not t.is_contiguous():
-                raise ValueError("params and grads must be contiguous fp32 CUDA tensors")
+    def _check_tensors(self, ts, what):
+        for i, (t, (r, c)) in enumerate(zip(ts, self.shapes)):
+            _require_cuda(t, "float32", r * c, f"{what}[{i}]", self._device)
 
     def step_prepare(self, grads, lr, momentum, weight_decay, eps=1e-7, stream=None):
         """First half of a step (meq_step_prepare): momentum, Newton-Schulz and
         statistics for these gradients; the parameters are not touched."""
         if len(grads) != len(self.shapes):
             raise ValueError("grads must have one tensor per matrix")
-        self._check_tensors(grads)
+        self._check_tensors(grads, "grads")
         n = len(self.shapes)
         for i, g in enumerate(grads):
             self._gp[i] = g.data_ptr()
@@ -278,7 +299,7 @@ class MeqMuon:
         """Second half of a step (meq_step_apply): the update of params."""
         if len(params) != len(self.shapes):
             raise ValueError("params must have one tensor per matrix")
-        self._check_tensors(params)
+        self._check_tensors(params, "params")
         for i, p in enumerate(params):
             self._pp[i] = p.data_ptr()
         self._check(lib.meq_step_apply(self._pp, self._st, _stream_handle(stream)))
@@ -295,7 +316,8 @@ class MeqMuon:
     def write_momentum(self, i, arr):
         r, c = self.shapes[i]
         a = np.ascontiguousarray(arr, dtype=np.float32)
-        assert a.shape == (r, c)
+        if a.shape != (r, c):
+            raise ValueError(f"momentum {i} must have shape {(r, c)}, got {a.shape}")
         self._check(lib.meq_write_momentum(self._st, i, a.ctypes.data))
 
     def read_ns_output(self, i):

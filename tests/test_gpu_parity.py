@@ -320,6 +320,19 @@ def test_argument_errors(meq):
     with pytest.raises(meq.MeqError) as e:
         o.step_ptrs([0], [g[0].data_ptr()], LR, MU, WD)
     assert e.value.status == 1
+    # the binding checks what the C ABI cannot see behind a pointer
+    for bad in (torch.zeros(64, 95, device="cuda"),                      # too few elements
+                torch.zeros(64, 96, device="cuda", dtype=torch.int32),   # not fp32
+                torch.zeros(96, 64, device="cuda").t(),                  # not contiguous
+                torch.zeros(64, 96)):                                    # host memory
+        with pytest.raises(ValueError):
+            o.step([bad], g, LR, MU, WD)
+        with pytest.raises(ValueError):
+            o.step_prepare([bad], LR, MU, WD)
+        with pytest.raises(ValueError):
+            o.step_apply([bad])
+    with pytest.raises(ValueError):
+        o.write_momentum(0, np.zeros((96, 64), np.float32))
     o.close()
     with pytest.raises(meq.MeqError) as e:
         meq.MeqMuon([(4096, 4096)], workspace_limit_bytes=1 << 20)

@@ -109,3 +109,22 @@ def test_host_validation_errors():
     with pytest.raises(meq.MeqError) as e:
         meq.state_bytes([(4, 4), (1, 4)], kinds=[meq.HIDDEN, meq.VECTOR], update_rule=meq.RULE_MUON)
     assert e.value.status == 1
+
+
+def test_binding_rejects_tensors_the_library_cannot_check(lib):
+    """The library sees raw pointers only; the binding refuses host tensors,
+    other dtypes, strided views and wrong element counts before any call."""
+    import torch
+
+    from paper_2609_35701_gb300 import meq
+
+    for t, dt, n in [(torch.zeros(4, 4), "float32", 16),                     # host memory
+                     (torch.zeros(4, 4, dtype=torch.float64), "float32", 16)]:
+        with pytest.raises(ValueError):
+            meq._require_cuda(t, dt, n, "x")
+    H = torch.zeros(8, 8)
+    with pytest.raises(ValueError):
+        meq.ns_cv_trajectory(H)
+    with pytest.raises(ValueError):
+        meq.row_col_stats_noalloc(H, torch.zeros(8), torch.zeros(8), torch.zeros(2, dtype=torch.float64),
+                                  torch.zeros(1, dtype=torch.int32))
