@@ -98,6 +98,12 @@ def test_host_validation_errors():
         assert e.value.status == 1
     with pytest.raises(meq.MeqError):
         meq.state_bytes([(4, 4)], ns_steps=0)
+    # the size limits, at and just past their edges (dims 2^20, elements 2^34)
+    meq.state_bytes([(1 << 20, 1), (1, 1 << 20), (1 << 20, 1 << 14)])
+    for bad in ([(1 << 20, (1 << 14) + 1)], [((1 << 20) + 1, 1)], [(1, (1 << 20) + 1)]):
+        with pytest.raises(meq.MeqError) as e:
+            meq.state_bytes(bad)
+        assert e.value.status == 1
     p0, w0 = meq.state_bytes([(300, 200), (1, 64)], kinds=[meq.HIDDEN, meq.VECTOR])
     p1, w1 = meq.state_bytes([(300, 200), (1, 64)], kinds=[meq.HIDDEN, meq.VECTOR], debug_canaries=1)
     assert p1 == p0 and w1 > w0  # guard bands are workspace only
