@@ -63,6 +63,10 @@ def test_single256_one_step(meq):
     [(1, 7), (7, 1), (1, 1), (3, 2)],
     [(257, 513), (513, 257), (64, 1000), (1000, 64)],
     [(384, 768), (768, 384), (768, 768), (129, 385)],
+    # extreme aspect ratios: one row of the maximum length (a Gram product of
+    # 16384 k-blocks in one tile), hundreds of column tiles over 2-3 rows, and
+    # a tall one (kept small: the oracle forms the literal m x m Gram matrix)
+    [(1, 1 << 20), (3, 1 << 16), (2, 40000), (1024, 3)],
 ])
 @pytest.mark.parametrize("pair", [1, 0], ids=["cta_pair", "single_cta"])
 def test_ragged_shapes_two_steps(meq, shapes, pair):
