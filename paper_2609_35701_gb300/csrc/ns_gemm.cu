@@ -659,6 +659,10 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
         const int b_mn_major = kPersistent ? G.b_mn_major : p.g[0].b_mn_major;
         const int arow = c.tm * TILE_M + static_cast<int>(rank) * BM;
         const int bcol = c.tn * BN + static_cast<int>(rank) * C_::BN_LOCAL;
+        // A diagonal tile of a symmetric product (X X^T, A A) has each CTA's
+        // B half equal to its A half (same rows of the same buffer, same box):
+        // only A is loaded, and the MMA reads it as B too.
+        const bool b_is_a = kPair == 2 && G.sym && !b_mn_major && arow == bcol;
         for (int kb = 0; kb < nk; ++kb) {
           if (!wait_bounded(EMPTY_BAR(stage), phase ^ 1u, err, DEV_TIMEOUT_PRODUCER, tmo)) {
             ok = false;
@@ -679,14 +683,16 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
           } else {
             // Both CTAs' copies complete on the leader's full barrier, which
             // the leader arms with the bytes of both.
-            if (leader) mbar_expect_tx(FULL_BAR(stage), 2 * STAGE_BYTES);
+            if (leader) mbar_expect_tx(FULL_BAR(stage), b_is_a ? 2 * A_BYTES : 2 * STAGE_BYTES);
             const uint32_t fb = leader ? FULL_BAR(stage) : map_to_rank(FULL_BAR(stage), 0);
             // tests (debug_skip_load): the stage is armed but this CTA's half never
             // comes, so the MMA issuer's bounded wait on it expires
             const bool skip = !kPersistent && p.debug_skip_load && leader && unit == 0 && n == 0 && kb == 0;
             if (!skip) {
               tma_load_3d_pair(sa, &G.tmA, fb, kb * BK, arow, c.mat);
-              if (!b_mn_major) {
+              if (b_is_a) {
+                // B is this stage's A
+              } else if (!b_mn_major) {
                 tma_load_3d_pair(sb, &G.tmB, fb, kb * BK, bcol, c.mat);
               } else {
 #pragma unroll
@@ -728,6 +734,8 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
         const int b_mn_major = kPersistent ? G.b_mn_major : p.g[0].b_mn_major;
         const uint32_t idesc = kPersistent ? G.idesc : p.g[0].idesc;
         const uint32_t b_lbo = b_mn_major ? (64u * BK * 2u) : 16u;
+        // diagonal tile of a symmetric product: B is read from the A half (the producer loads A only)
+        const bool b_is_a = kPair == 2 && G.sym && !b_mn_major && c.tm * TILE_M == c.tn * BN;
         if (!wait_bounded(TEMPTY_BAR(acc), acc_phase ^ 1u, err, DEV_TIMEOUT_MMA_TMEM, tmo)) break;
         tc_fence_after();
         const uint32_t d = tmem_base + static_cast<uint32_t>(acc * BN);
@@ -738,7 +746,7 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
           }
           tc_fence_after();
           const uint32_t sa = base + stage * STAGE_BYTES;
-          const uint32_t sb = sa + A_BYTES;
+          const uint32_t sb = b_is_a ? sa : sa + A_BYTES;
 #pragma unroll
           for (int k = 0; k < BK / UK; ++k) {
             const uint64_t adesc = smem_desc(sa + k * (UK * 2), 16u, 1024u);
