@@ -5,12 +5,13 @@ Metric: milliseconds per optimizer step for the whole model (lower is
 better), with NS TFLOP/s and the bandwidth kernels' GB/s as fractions of the
 measured GB300 peaks.
 
-Default workload: Llama-130M hidden weights (84 matrices, 84.9M elements),
-seeded synthetic gradients (see paper_2609_35701_gb300/workloads.py); the
-state (params + grads + momentum = 1.02 GB) is larger than L2, so no flush
-is needed between steps.
+Default workload: the Llama-7B-class hidden weights (32 layers, d 4096, ffn
+11008: 224 matrices, 6.48G elements; params + grads + momentum 77.7 GB on
+one GPU), the largest single-GPU configuration; seeded synthetic gradients
+(see paper_2609_35701_gb300/workloads.py). Every workload's state is larger
+than L2, so no flush is needed between steps.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--layers L]
   python bench.py --impl reference ...   # the fp64 CPU oracle on host cores
 
 With N > 1 (torchrun), the matrices are split across ranks (flop-balanced,
@@ -34,7 +35,10 @@ sys.path.insert(0, ROOT)
 LR, MU, WD, EPS = 0.02, 0.95, 0.1, 1e-7
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 BW_BYTES_PER_ELEM = 24  # read G, B; write B; write X_0 (2 B); read U (2 B); read + write W
-REFERENCE_BUDGET_S = 150.0   # wall-clock cap on the timed oracle samples of --impl reference
+REFERENCE_BUDGET_S = 150.0   # wall-clock budget of all oracle samples of --impl reference
+CPU_BASELINE_BUDGET_S = 20.0 # wall-clock budget of the oracle sample beside the GPU line
+SUSTAINED_NS_MS = 20.0       # an NS phase this long per step runs under the power cap: sustained peak
+DEFAULT_STEPS = {"llama7b": 20, "llama1b": 50}
 METRIC = "MeqMuon step ms per model; NS TFLOP/s & equilibration GB/s as % of GB300 peak"
 COPY_CHUNK = 8 << 20          # elements (32 MB) per host <-> device copy of the end-to-end loop
 
@@ -154,11 +158,22 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def oracle_sample(wl, seed_step=0, max_per_class=1, rule="meqmuon"):
-    """Times the fp64 oracle on one matrix of every (rows, cols) class of the
-    workload and extrapolates to the whole model step (ms)."""
+def oracle_flops(r, c, kind, K=5):
+    """fp64 flops of the oracle's step for one (rows, cols) matrix: Eq. (5)
+    as written (A = X X^T on the row side, A A, then (b A + c A^2) X), or a
+    few dozen per element for the branches without Newton-Schulz."""
+    if kind != 0:
+        return 30 * r * c
+    return K * (4 * r * r * c + 2 * r ** 3)
+
+
+def oracle_sample(wl, seed_step=0, rule="meqmuon", budget_s=None):
+    """Times the fp64 oracle on one matrix of each (rows, cols, kind) class of
+    the workload, cheapest first, and extrapolates to the whole model step
+    (ms). With a budget, a class whose predicted time (the flop rate of the
+    classes timed so far) would overrun it is not run: its time is that rate
+    times its flop count. Returns (ms, timed classes, estimated classes)."""
     import numpy as np
-    import torch
 
     from oracle import meqmuon as O
     from paper_2609_35701_gb300 import workloads as W
@@ -167,11 +182,21 @@ def oracle_sample(wl, seed_step=0, max_per_class=1, rule="meqmuon"):
     kinds = wl.kind_list()
     for i, (_, r, c) in enumerate(wl.shapes):
         classes.setdefault((r, c, kinds[i]), []).append(i)
-    total_ms = 0.0
-    sampled = []
-    for (r, c, k), idx in classes.items():
-        i = idx[0]
-        G = W.gradient(wl, i, seed_step).double().numpy()
+    order = sorted(classes, key=lambda k: oracle_flops(*k))
+    total_ms, spent, flops_done = 0.0, 0.0, 0.0
+    timed, estimated = [], []
+
+    def label(r, c, k):
+        return f"{r}x{c}" + ("" if k == 0 else ("/2-sided" if k == 1 else "/vector"))
+
+    for (r, c, k) in order:
+        idx = classes[(r, c, k)]
+        f = oracle_flops(r, c, k)
+        if timed and budget_s is not None and spent > 0 and spent + f / (flops_done / spent) > budget_s:
+            total_ms += f / (flops_done / spent) * 1e3 * len(idx)
+            estimated.append(label(r, c, k))
+            continue
+        G = W.gradient(wl, idx[0], seed_step).double().numpy()
         W0 = np.zeros((r, c))
         Bp = np.zeros((r, c))
         t0 = time.perf_counter()
@@ -179,10 +204,27 @@ def oracle_sample(wl, seed_step=0, max_per_class=1, rule="meqmuon"):
             O.moonlight_step(W0, G, Bp, LR, MU, WD)
         else:
             O.param_step(k, W0, G, Bp, LR, MU, WD, eps=EPS)
-        dt = (time.perf_counter() - t0) * 1e3
-        total_ms += dt * len(idx)
-        sampled.append(f"{r}x{c}" + ("" if k == 0 else ("/2-sided" if k == 1 else "/vector")))
-    return total_ms, sampled
+        dt = time.perf_counter() - t0
+        spent += dt
+        flops_done += f
+        total_ms += dt * 1e3 * len(idx)
+        timed.append(label(r, c, k))
+    return total_ms, timed, estimated
+
+
+def sample_text(wl, timed, estimated, repeats):
+    t = (f"fp64 oracle on one matrix per shape class, timed: {', '.join(timed)}"
+         + (f"; estimated from the timed classes' flop rate x the oracle's own flop count: {', '.join(estimated)}"
+            if estimated else "")
+         + f"; {repeats} sample(s); extrapolated by class counts to all {len(wl.shapes)} matrices")
+    return t
+
+
+def workload_for(args):
+    from paper_2609_35701_gb300 import workloads as W
+
+    wl = W.get_workload(args.workload)
+    return W.first_layers(wl, args.layers) if args.layers else wl
 
 
 def cpu_cores():
@@ -201,28 +243,27 @@ def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    from paper_2609_35701_gb300 import workloads as W
-
-    wl = W.get_workload(args.workload)
-    for w in range(args.warmup):
-        oracle_sample(wl, w, rule=args.update_rule)
+    wl = workload_for(args)
+    # each sample gets an equal share of the budget (the warm-up sample too),
+    # so the whole --steps K --warmup W run stays within a few minutes
+    per = max(REFERENCE_BUDGET_S / (args.steps + 1), 2.0)
+    oracle_sample(wl, 0, rule=args.update_rule, budget_s=per)  # warm-up (BLAS threads)
     vals = []
-    sampled = None
+    timed = estimated = None
     t0 = time.perf_counter()
     for k in range(args.steps):
-        ms, sampled = oracle_sample(wl, k, rule=args.update_rule)
+        ms, timed, estimated = oracle_sample(wl, k, rule=args.update_rule, budget_s=per)
         vals.append(ms)
         if time.perf_counter() - t0 > REFERENCE_BUDGET_S:
             break  # the samples are timed on the host cores: keep the whole run to a few minutes
     v = statistics.median(vals)
     cores = cpu_cores()
-    sample = (f"one matrix per shape class ({', '.join(sampled)}) per step, fp64 oracle, "
-              f"extrapolated by class counts to all {len(wl.shapes)} matrices")
+    sample = sample_text(wl, timed, estimated, len(vals)) + " (one sample per step)"
     line = {
         "impl": "reference", "metric": METRIC, "value": v,
         "unit": "ms/step", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": v, "higher_is_better": False, "scaling": "strong", "vs_baseline": None, "dtype": "f64",
-        "timed_steps": len(vals), "data": "synthetic", "config": {"workload": args.workload, "matrices": len(wl.shapes), "elements": wl.numel,
+        "timed_steps": len(vals), "data": "synthetic", "config": {"workload": wl.name, "matrices": len(wl.shapes), "elements": wl.numel,
                                         "update_rule": "Eq. (11) + Eq. (14)" if args.update_rule == "meqmuon" else "Eq. (6)"},
         "cpu_baseline": {"value": v, "unit": "ms/step", "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": v, "unit": "ms/step", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -244,7 +285,7 @@ def run_trajectory(args):
     from paper_2609_35701_gb300 import meq
     from paper_2609_35701_gb300 import workloads as W
 
-    wl = W.get_workload(args.workload)
+    wl = workload_for(args)
     kinds = wl.kind_list()
     firsts = {}
     for i, (_, r, c) in enumerate(wl.shapes):
@@ -271,7 +312,7 @@ def run_trajectory(args):
     line = {
         "metric": f"NS CV trajectory replay, k = 0..{K} (Section 3.1)", "value": gpu_ms, "unit": "ms (all shapes)",
         "n_gpus": 1, "steps": reps, "warmup": 2, "higher_is_better": False, "dtype": "fp16", "data": "synthetic",
-        "config": {"workload": args.workload, "shapes": shapes,
+        "config": {"workload": wl.name, "shapes": shapes,
                    "method": "one state per k (ns_steps = k) through the CUDA step, k = 0 by the statistics kernel"},
         "cpu_baseline": {"value": cpu_ms, "unit": "ms (all shapes)", "cores": cpu_cores(), "kind": "oracle",
                          "sample": f"fp64 oracle replay of the same {len(Hs)} matrices"},
@@ -282,21 +323,24 @@ def run_trajectory(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
-    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=None, help="timed steps (default: 20 for llama7b, 50 for llama1b, "
+                    "200 otherwise)")
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="llama130m")
+    ap.add_argument("--workload", default="llama7b")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="use only the first L layers of the workload (a smaller case of the same kernels)")
     ap.add_argument("--ns-fp16-mask", type=lambda x: int(x, 0), default=0xFFFFFFFF)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--update-rule", default="meqmuon", choices=["meqmuon", "muon"],
                     help="meqmuon: Eq. (11) + Eq. (14); muon: the Eq. (6) comparison baseline (hidden weights only)")
-    ap.add_argument("--ns-single-launch", action="store_true",
-                    help="run all Newton-Schulz products in one cooperative launch (option ns_single_launch)")
     ap.add_argument("--ns-trajectory", type=int, default=0, metavar="K",
                     help="instead of the step, time the Section 3.1 CV replay of X_0..X_K (one matrix per shape)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    if args.steps is None:
+        args.steps = DEFAULT_STEPS.get(args.workload, 200)
     if args.impl == "reference":
         run_reference(args)
         return
@@ -320,7 +364,7 @@ def main():
     from paper_2609_35701_gb300 import meq
     from paper_2609_35701_gb300 import workloads as W
 
-    wl = W.get_workload(args.workload)
+    wl = workload_for(args)
     mine = partition([(r, c) for _, r, c in wl.shapes], world, kinds=wl.kind_list())[rank]
     shapes = [(wl.shapes[i][1], wl.shapes[i][2]) for i in mine]
     all_kinds = wl.kind_list()
@@ -355,8 +399,7 @@ def main():
     grads = [[v.view(r, c) for v, (r, c) in zip(gv, shapes)] for _, gv in gbufs]
 
     rule = meq.RULE_MUON if args.update_rule == "muon" else meq.RULE_MEQMUON
-    opt = meq.MeqMuon(shapes, kinds=kinds, ns_fp16_mask=args.ns_fp16_mask, update_rule=rule,
-                      ns_single_launch=1 if args.ns_single_launch else 0)
+    opt = meq.MeqMuon(shapes, kinds=kinds, ns_fp16_mask=args.ns_fp16_mask, update_rule=rule)
     stream = torch.cuda.current_stream()
     for k in range(args.warmup):
         opt.step(params, grads[k % 2], LR, MU, WD, EPS)
@@ -403,6 +446,10 @@ def main():
     dense = sum(ns_flops(min(r, c), max(r, c), K)[1] for r, c in hid)
     n_gemm_launches = opt.ns_gemm_launches_per_step
     peaks, peak_src = load_peaks()
+    # an NS phase that runs tens of milliseconds at a time draws the power
+    # cap: its denominator is the sustained bf16 figure, else the burst one
+    sustained = ph["ns_gemm"] >= SUSTAINED_NS_MS
+    ns_peak = peaks["bf16_tflops_sustained"] if sustained else peaks["bf16_tflops"]
     ns_tflops = sym / (ph["ns_gemm"] * 1e-3) / 1e12
     ns_dense_tflops = dense / (ph["ns_gemm"] * 1e-3) / 1e12
     numel = sum(nums)
@@ -415,11 +462,12 @@ def main():
     # ---------------- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
-        hg = []
-        for gb, _ in gbufs:
-            h = torch.empty(gb.numel(), dtype=torch.float32, pin_memory=True)
-            h.copy_(gb)
-            hg.append(h)
+        # one pinned host copy of the gradients serves both device buffers
+        # (every step uploads a whole gradient set; at Llama-7B one set is
+        # 25.9 GB, so two would pin another 26 GB of host memory)
+        h = torch.empty(gbufs[0][0].numel(), dtype=torch.float32, pin_memory=True)
+        h.copy_(gbufs[0][0])
+        hg = [h, h]
         hp = torch.empty(pbuf.numel(), dtype=torch.float32, pin_memory=True)
         n_e2e = max(3, min(args.steps, 50))
         # Copies move in pieces of COPY_CHUNK elements on two copy streams,
@@ -479,16 +527,16 @@ def main():
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        vals, sampled = [], None
+        vals = []
         t_start = time.perf_counter()
         while True:
-            v, sampled = oracle_sample(wl, len(vals), rule=args.update_rule)
+            left = CPU_BASELINE_BUDGET_S - (time.perf_counter() - t_start)
+            v, timed, estimated = oracle_sample(wl, len(vals), rule=args.update_rule, budget_s=max(left, 1.0))
             vals.append(v)
-            if time.perf_counter() - t_start > 10.0 or len(vals) >= 5:
+            if time.perf_counter() - t_start > CPU_BASELINE_BUDGET_S / 2 or len(vals) >= 5:
                 break
         cpu = {"value": statistics.median(vals), "unit": "ms/step", "cores": cpu_cores(), "kind": "oracle",
-               "sample": (f"fp64 oracle on one matrix per shape class ({', '.join(sampled)}), {len(vals)} repeats, "
-                          f"extrapolated by class counts to all {len(wl.shapes)} matrices")}
+               "sample": sample_text(wl, timed, estimated, len(vals))}
 
     if rank == 0:
         line = {
@@ -497,7 +545,7 @@ def main():
             "ms_per_step": ms, "higher_is_better": False, "scaling": "strong", "vs_baseline": None,
             "dtype": "fp16" if args.ns_fp16_mask == 0xFFFFFFFF else ("bf16" if args.ns_fp16_mask == 0 else "bf16/fp16"),
             "data": "synthetic",
-            "config": {"workload": args.workload, "matrices": len(wl.shapes), "elements": wl.numel,
+            "config": {"workload": wl.name, "matrices": len(wl.shapes), "elements": wl.numel,
                        "ns_steps": K, "ns_operands": "fp16" if args.ns_fp16_mask == 0xFFFFFFFF else hex(args.ns_fp16_mask),
                        "accumulate": "fp32", "l2": "inputs larger than L2 (params+grads+momentum %.2f GB)" % (12 * wl.numel / 1e9),
                        "parallelism": f"matrices split over {world} GPU(s)" if world > 1 else "single GPU",
@@ -505,10 +553,12 @@ def main():
                        "ns_launches_per_step": n_gemm_launches},
             "roofline": {
                 "bound": "tensor", "kernel": "ns_gemm_kernel",
-                "achieved": ns_tflops, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
-                "frac": ns_tflops / peaks["bf16_tflops"], "peak_source": f"{peak_src} bf16 dense burst (fp16 rate = bf16 rate)",
-                # the recorded capture is of the one-launch-per-product kernel
-                "traffic": recorded_traffic(args.workload) if n_gemm_launches > 1 else None,
+                "achieved": ns_tflops, "peak": ns_peak, "unit": "TFLOP/s",
+                "frac": ns_tflops / ns_peak,
+                "peak_source": (f"{peak_src} bf16 dense {'sustained' if sustained else 'burst'} (fp16 rate = bf16 rate;"
+                                f" NS phase {ph['ns_gemm']:.2f} ms per step)"),
+                "frac_of_burst": ns_tflops / peaks["bf16_tflops"],
+                "traffic": recorded_traffic(wl.name),
                 "flops_per_launch": sym / max(n_gemm_launches, 1),
                 "avg_launch_ms": ph["ns_gemm"] / max(n_gemm_launches, 1),
                 "dense_equivalent_tflops": ns_dense_tflops,

@@ -76,20 +76,13 @@ typedef struct {
   int update_rule;        /* meq_update_rule; default MEQ_RULE_MEQMUON */
   int debug_canaries;     /* 1: guard bands of a fixed byte pattern surround every workspace
                              buffer (meq_check_canaries); default 0 */
-  int ns_single_launch;   /* 1: all 3K products of Eq. (5) run in one cooperative launch of
-                             CTA pairs, each tile waiting (bounded) until the previous product
-                             of its matrix is complete; used when ns_cta_pair = 1 and the
-                             shape groups x 3K fit 48 segments (with at most 8 groups),
-                             else the step keeps one launch per product
-                             (meq_ns_gemm_launches_per_step tells which). 0 (default): one
-                             launch per product. */
   int debug_skip_load;    /* 1 (tests only): in every step's first NS launch, the leader
                              CTA of the first CTA pair arms its first operand stage but
                              does not load its half, so that stage never completes: the
                              MMA issuer's bounded wait expires, every role of the launch
                              stops and drains, and meq_sync reports MEQ_ERR_TIMEOUT (the
                              results of that step are not meaningful). Requires
-                             ns_cta_pair = 1 and ns_single_launch = 0. Default 0. */
+                             ns_cta_pair = 1. Default 0. */
 } meq_options;
 
 /* Update applied to the hidden 2D weights after momentum and Newton-Schulz. */
@@ -185,8 +178,10 @@ meq_status meq_sync(meq_state* st);
 /* Release all device memory of the state (synchronises first). NULL is a no-op. */
 meq_status meq_free(meq_state* st);
 
-/* Human-readable text of the last error of st (or of the last init failure
- * when st is NULL). Valid until the next call on the same state. */
+/* Human-readable text of the last error of st; with st NULL, of the last
+ * failed call made without a state (meq_init_state[_kinds],
+ * meq_state_bytes[_kinds], meq_ns_cv_trajectory, meq_row_col_stats_noalloc).
+ * Valid until the next such call. */
 const char* meq_last_error(const meq_state* st);
 const char* meq_status_string(meq_status s);
 
@@ -202,6 +197,16 @@ meq_status meq_write_momentum(meq_state* st, int i, const float* src);
  * significant bits); the values returned are those fp16 values, from which
  * the row and column statistics are taken and which the update applies. */
 meq_status meq_read_ns_output(meq_state* st, int i, float* dst);
+/* Copy the normalised update U~_i of the last step (rows x cols fp32) to
+ * dst (host or device): the matrix that step applied as
+ * W <- (1 - lr wd) W - rho lr U~ (Eq. (14)). Hidden weight: diag(r^-1) U or
+ * U diag(c^-1) (Eqs. (9), (11); rows or columns with RMS <= eps scaled by 0),
+ * or sqrt(max(m, n)) U under MEQ_RULE_MUON (Eq. (6)); remaining 2D
+ * parameter: N_c(N_r(B_t)) (Eq. (12)); vector: B_t / RMS(B_t) (Eq. (13)).
+ * Computed by a kernel from the operands and scale factors of the update
+ * kernel; a host dst goes through a temporary device buffer of the same size
+ * (MEQ_ERR_OOM if that allocation fails). Synchronises the state's stream. */
+meq_status meq_read_update(meq_state* st, int i, float* dst);
 /* Last step's statistics of entry i. Hidden weight: r (rows floats), c (cols
  * floats) of Eq. (7) for U, gamma_r, gamma_c of Eq. (8) and the direction of
  * Eq. (11) (0 = row, 1 = column; 4 under MEQ_RULE_MUON, whose update is
@@ -237,11 +242,15 @@ meq_status meq_debug_corrupt_canary(meq_state* st, int index);
  * gamma_c[k] are the Eq. (8) CVs (over entries > eps) of the row and column
  * RMS (Eq. (7)) of X_k, k = 0..steps, computed by this library's CUDA path
  * with the NS options of opt (NULL: defaults; its ns_steps and update_rule
- * are ignored). h: device fp32, rows x cols row-major, 16-byte aligned, read
- * only. gamma_r, gamma_c: host arrays of steps + 1 doubles. steps: 0..32.
- * Synchronous; allocates and frees its own device scratch. Errors:
+ * are ignored). k = 0 is X_0 = h / ||h||_F: its RMS values, like those of
+ * every later iterate, are compared with eps after the normalisation. h:
+ * device fp32, rows x cols row-major, 16-byte aligned, read only. gamma_r,
+ * gamma_c: host arrays of steps + 1 doubles. steps: 0..32. Synchronous;
+ * allocates and frees its own device scratch (about rows x cols x 4 bytes
+ * plus one optimizer state per k), so concurrent calls do not share memory;
+ * every shape meq_init_state accepts is accepted. Errors:
  * MEQ_ERR_INVALID_ARG (NULL, misaligned, bad sizes), MEQ_ERR_OOM, or the
- * error of the step it runs. */
+ * error of the step it runs (text in meq_last_error(NULL)). */
 meq_status meq_ns_cv_trajectory(const float* h, int64_t rows, int64_t cols, int steps, float eps,
                                 const meq_options* opt, double* gamma_r, double* gamma_c, void* cuda_stream);
 /* Number of kernels one meq_step launches (for launch accounting), and how
@@ -287,14 +296,17 @@ meq_status meq_debug_wait_selftest(meq_state* st, float timeout_ms);
  * the library, held by every GPU that loads the library until the process
  * exits. A matrix fits when rows + ceil(rows / 32) * cols <= 2,097,152 (e.g.
  * 4096 x 11008 and 11008 x 4096); larger ones, NULL pointers or
- * non-positive sizes return MEQ_ERR_INVALID_ARG before anything is enqueued.
+ * non-positive sizes return MEQ_ERR_INVALID_ARG before anything is enqueued
+ * and before any CUDA call; meq_last_error(NULL) then says why.
  * The first call on a device looks up the array's device address (once per
  * device, with that device current); make that first call before any CUDA
  * stream capture. Every call shares the one array and overwrites all of the
  * scratch it reads, so nothing needs clearing between calls, but calls whose
  * kernels overlap on the GPU (different streams without ordering) race on
- * it. Work is enqueued on cuda_stream (cudaStream_t, NULL = legacy stream);
- * MEQ_ERR_CUDA reports a failed launch or address lookup. */
+ * it. Work is enqueued on cuda_stream (cudaStream_t, NULL = legacy stream)
+ * as three kernel launches; MEQ_ERR_CUDA reports a failed launch or address
+ * lookup of this call (its own status, with the CUDA error text in
+ * meq_last_error(NULL)). */
 meq_status meq_row_col_stats_noalloc(const float* U, int64_t rows, int64_t cols, float eps,
                                      float tie_atol, float* r, float* c, double* gammas,
                                      int* direction, void* cuda_stream);

@@ -12,6 +12,8 @@
 //   rows, colpart : momentum, row and column statistics of the remaining 2D
 //                   parameters and vectors (Eqs. (12), (13)).
 //   apply         : W <- (1 - lr wd) W - rho lr U~ (Eq. (14)).
+#include <algorithm>
+
 #include "meq_elementwise.cuh"
 
 namespace meq {
@@ -764,6 +766,33 @@ __global__ void __launch_bounds__(kThreads, 8) apply_kernel(const MatInfo* __res
   }
 }
 
+// The normalised update of one entry that apply_kernel applies, W <- (1 -
+// lr wd) W - rho lr U~: U~ = diag(r^-1) U or U diag(c^-1) (Eqs. (9), (11)),
+// sqrt(max(m, n)) U under the Eq. (6) rule, N_c(N_r(B)) (Eq. (12)) or
+// B / RMS(B) (Eq. (13)), with the same scale factors and operands.
+__global__ void __launch_bounds__(kThreads) update_kernel(MatInfo M, int mi, const uint16_t* __restrict__ uslab,
+                                                          const float* __restrict__ mom,
+                                                          const float* __restrict__ svec,
+                                                          const float* __restrict__ tvec,
+                                                          const MatStats* __restrict__ stats, float* __restrict__ dst) {
+  const bool hidden = M.kind == KIND_HIDDEN;
+  const int dir = hidden ? stats[mi].direction : (M.kind == KIND_TWO_SIDED ? 2 : 0);
+  const int mode = dir == 4 ? 0 : dir;
+  const float* sv = svec + M.vec_off;
+  const float* tv = tvec + M.vec_off;
+  const uint16_t* U16 = uslab + M.u_off;
+  const float* U32 = mom + M.mom_off;
+  const float back = hidden ? 1.0f / kUScale : 1.0f;  // a power of two: exact
+  const int64_t numel = M.m * M.n;
+  for (int64_t e = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; e < numel;
+       e += static_cast<int64_t>(gridDim.x) * kThreads) {
+    const int64_t i = e / M.n, j = e - i * M.n;
+    const float u = hidden ? __half2float(__ushort_as_half(U16[i * M.un + j])) : U32[e];
+    const float f = mode == 0 ? sv[i] : (mode == 1 ? sv[j] : sv[i] * tv[j]);
+    dst[e] = (f * u) * back;
+  }
+}
+
 // Bounded-wait self test: waits on a flag nobody sets and reports a timeout.
 __global__ void wait_selftest_kernel(const volatile int* flag, int* err, unsigned long long timeout_ns) {
   unsigned long long t0;
@@ -825,6 +854,14 @@ cudaError_t launch_apply(const LaunchCtx& L, cudaStream_t st) {
                     static_cast<const uint16_t*>(L.uslab), static_cast<const float*>(L.mom),
                     static_cast<const float*>(L.svec), static_cast<const float*>(L.tvec),
                     static_cast<const MatStats*>(L.stats), L.sc);
+}
+
+cudaError_t launch_update(const LaunchCtx& L, const MatInfo& M, int mi, float* dst, cudaStream_t st) {
+  const int64_t blocks = std::min<int64_t>((M.m * M.n + kThreads - 1) / kThreads, 4096);
+  update_kernel<<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(
+      M, mi, static_cast<const uint16_t*>(L.uslab), static_cast<const float*>(L.mom),
+      static_cast<const float*>(L.svec), static_cast<const float*>(L.tvec), static_cast<const MatStats*>(L.stats), dst);
+  return cudaPeekAtLastError();
 }
 
 cudaError_t launch_wait_selftest(const int* flag, int* err, unsigned long long timeout_ns, cudaStream_t st) {

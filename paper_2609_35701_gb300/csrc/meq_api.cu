@@ -84,6 +84,8 @@ struct Layout {
 
 }  // namespace
 
+void meq::set_global_error(const std::string& msg) { g_init_error = msg; }
+
 struct meq_state {
   int n = 0;
   std::vector<meq_shape> shapes;
@@ -124,10 +126,6 @@ struct meq_state {
   // launch plan
   std::vector<GemmParams> gemm;  // in launch order
   std::vector<int> gemm_grid;
-  PersistParams persist;       // the one-launch NS (ns_single_launch), when it fits
-  int persist_grid = 0;
-  bool use_persist = false;
-  int* d_done = nullptr;       // its completion counters, [3K][n_hidden]
   LaunchCtx ctx{};
   bool graph_ready = false;
   cudaGraph_t graph = nullptr;
@@ -177,10 +175,9 @@ bool valid_options(const meq_options& o, std::string* why) {
   if (o.ns_cta_pair != 0 && o.ns_cta_pair != 1) { *why = "ns_cta_pair must be 0 or 1"; return false; }
   if (o.ns_x0_fused != 0 && o.ns_x0_fused != 1) { *why = "ns_x0_fused must be 0 or 1"; return false; }
   if (o.debug_canaries != 0 && o.debug_canaries != 1) { *why = "debug_canaries must be 0 or 1"; return false; }
-  if (o.ns_single_launch != 0 && o.ns_single_launch != 1) { *why = "ns_single_launch must be 0 or 1"; return false; }
   if (o.debug_skip_load != 0 && o.debug_skip_load != 1) { *why = "debug_skip_load must be 0 or 1"; return false; }
-  if (o.debug_skip_load && (!o.ns_cta_pair || o.ns_single_launch)) {
-    *why = "debug_skip_load requires ns_cta_pair = 1 and ns_single_launch = 0";
+  if (o.debug_skip_load && !o.ns_cta_pair) {
+    *why = "debug_skip_load requires ns_cta_pair = 1";
     return false;
   }
   if (o.update_rule != MEQ_RULE_MEQMUON && o.update_rule != MEQ_RULE_MUON) {
@@ -328,8 +325,7 @@ void plan(meq_state* st, Layout* L, int64_t* off_mom, int64_t* off_u, int64_t* o
   *off_vec4 = L->add(vec * 4 * 4);  // r, c, s, t
   *off_cpart = L->add(parts * 4);
   *off_partials = L->add(std::max({hchunks, tiles, xblks}) * 4);  // per momentum chunk or block
-  // per-matrix counters, then the one-launch NS completion counters [3K][n_hidden]
-  *off_counters = L->add(int64_t(n) * 4 + int64_t(3) * st->opt.ns_steps * st->n_hidden * 4);
+  *off_counters = L->add(int64_t(n) * 4);  // per-matrix counters
   *off_x0s = L->add(int64_t(n) * 4 * 2);  // x0scale (cast pass) and the inverse norms (fused)
   *off_stats = L->add(int64_t(n) * sizeof(MatStats) + int64_t(n) * 2 * 8);  // stats, then direction counts
   st->step_bytes = sizeof(StepScalars) + 2 * int64_t(n) * sizeof(void*);
@@ -431,7 +427,6 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
           Group& G = st->groups[g0 + gi];
           GemmGroup& Q = P.g[gi];
           Q.mode = real_mode, Q.idesc = idesc, Q.b_mn_major = b_mn_major;
-          Q.mat_base = static_cast<int32_t>(G.mbase);
           // storage scale of X_k; a fused X_0 is unscaled and its 1/||H||_F is applied per matrix
           const float ak = (k == 0) ? (fused ? 1.0f : G.alpha0) : G.alpha;
           const bool per_matrix = fused && k == 0;
@@ -468,8 +463,6 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
             ok &= encode_map(&Q.tmB, G.x[cur], 2, G.l, G.s, G.count, G.lp, 64, 64, SW128);
             if (real_mode == MODE_XUPD) {
               Q.out = G.x[nxt], Q.out_ld = x_ld, Q.out_mstride = x_ms;
-              // thread stores here; the one-launch NS switches to this map (below)
-              ok &= encode_map(&Q.tmO, G.x[nxt], 2, G.l, G.s, G.count, G.lp, 32, 32, SW64);
               Q.scale = G.alpha / ak;
               if (per_matrix) Q.minv = st->d_ginv + G.mbase, Q.minv_pow = 1;
               Q.out_fp16 = dX(k + 1);
@@ -503,47 +496,6 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
       }
     }
   }
-  // ns_single_launch: the per-product launches' groups become the segments of
-  // one tile queue in product order; a tile of product j waits until both
-  // CTAs of every tile of its matrix in product j - 1 have counted it stored.
-  st->use_persist = false;
-  const int nprod = 3 * K;
-  if (st->opt.ns_single_launch && pair == 2 && ng <= kMaxGroups && static_cast<int>(st->gemm.size()) == nprod &&
-      nprod * ng <= kMaxSegs) {
-    const int max_pairs = ns_gemm_persistent_max_pairs();
-    if (max_pairs > 0) {
-      PersistParams& Q = st->persist;
-      std::memset(&Q, 0, sizeof(Q));
-      int tiles = 0, nseg = 0;
-      for (int j = 0; j < nprod; ++j) {
-        const GemmParams& P = st->gemm[j];
-        for (int gi = 0; gi < P.ngroups; ++gi) {
-          GemmGroup S = P.g[gi];
-          S.tile_begin = tiles;
-          S.prod = j;
-          S.dep_target = j == 0 ? 0 : st->gemm[j - 1].g[gi].tiles_per_mat * pair;  // one count per CTA and tile
-          // every output another tile waits for leaves by TMA stores, whose
-          // completion a warp can wait for without waiting for later stores
-          if (S.mode == MODE_XUPD) S.tma_out = 1;
-          tiles += S.tiles_per_mat * S.count;
-          Q.g[nseg++] = S;
-        }
-      }
-      const GemmParams& P0 = st->gemm[0];
-      Q.ngroups = nseg;
-      Q.total_tiles = tiles;
-      Q.reverse = 0;
-      Q.ca = P0.ca, Q.cb = P0.cb, Q.cc = P0.cc;
-      Q.err = st->d_err;
-      Q.sched = st->d_sched;
-      Q.done = st->d_done;
-      Q.nslots = static_cast<int32_t>(st->n_hidden);
-      Q.nprod = nprod;
-      Q.timeout_ns = P0.timeout_ns;
-      st->persist_grid = pair * std::max(1, std::min({tiles, st->num_sms / pair, max_pairs}));
-      st->use_persist = true;
-    }
-  }
   return true;
 }
 
@@ -568,7 +520,6 @@ void meq_default_options(meq_options* o) {
   o->ns_cta_pair = 1;
   o->ns_x0_fused = 1;
   o->debug_canaries = 0;
-  o->ns_single_launch = 0;
   o->debug_skip_load = 0;
 }
 
@@ -680,7 +631,6 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   st->d_parts = reinterpret_cast<float*>(A + off_cpart);
   st->d_partials = reinterpret_cast<float*>(A + off_partials);
   st->d_counters = reinterpret_cast<unsigned int*>(A + off_counters);
-  st->d_done = reinterpret_cast<int*>(st->d_counters + n);
   st->d_x0scale = reinterpret_cast<float*>(A + off_x0s);
   st->d_ginv = st->d_x0scale + n;
   st->d_stats = reinterpret_cast<MatStats*>(A + off_stats);
@@ -757,7 +707,7 @@ meq_status meq_init_state_kinds(const meq_shape* shapes, const int* kinds, int n
   C.total_rblks = st->total_rblks;
   C.total_slabs = st->total_slabs;
   st->kernels_per_step = (st->n_hidden ? 2 : 0) + (st->n_rows ? 1 : 0) + (st->n_two ? 1 : 0) + 2 +
-                         (st->use_persist ? 1 : static_cast<int>(st->gemm.size()));
+                         static_cast<int>(st->gemm.size());
   st->step_host.assign(static_cast<size_t>(st->step_bytes), 0);
   st->last_stream = s;
   *out = st;
@@ -825,14 +775,9 @@ static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev
     if (e != cudaSuccess) return cuda_fail(st, e, "cast_x0 launch");
   }
   mark(2);
-  if (st->use_persist) {
-    e = launch_ns_gemm_persistent(st->persist, st->persist_grid, s);
-    if (e != cudaSuccess) return cuda_fail(st, e, "ns_gemm (single launch)");
-  } else {
-    for (size_t i = 0; i < st->gemm.size(); ++i) {
-      e = launch_ns_gemm(st->gemm[i], st->gemm_grid[i], st->opt.ns_cta_pair ? 2 : 1, s);
-      if (e != cudaSuccess) return cuda_fail(st, e, "ns_gemm launch");
-    }
+  for (size_t i = 0; i < st->gemm.size(); ++i) {
+    e = launch_ns_gemm(st->gemm[i], st->gemm_grid[i], st->opt.ns_cta_pair ? 2 : 1, s);
+    if (e != cudaSuccess) return cuda_fail(st, e, "ns_gemm launch");
   }
   mark(3);
   if (st->n_two) {
@@ -1076,6 +1021,31 @@ meq_status meq_read_ns_output(meq_state* st, int i, float* dst) {
   return e == cudaSuccess ? MEQ_OK : cuda_fail(st, e, "cudaMemcpy");
 }
 
+meq_status meq_read_update(meq_state* st, int i, float* dst) {
+  meq_status ms = check_index(st, i);
+  if (ms != MEQ_OK) return ms;
+  if (!dst) return fail(st, MEQ_ERR_INVALID_ARG, "dst is NULL");
+  const MatInfo& M = st->mats[i];
+  const size_t bytes = static_cast<size_t>(M.m * M.n) * sizeof(float);
+  cudaPointerAttributes pa{};
+  cudaError_t e = cudaPointerGetAttributes(&pa, dst);
+  if (e != cudaSuccess) return cuda_fail(st, e, "cudaPointerGetAttributes");
+  const bool on_device = (pa.type == cudaMemoryTypeDevice || pa.type == cudaMemoryTypeManaged) && pa.device == st->device;
+  float* out = dst;
+  if (!on_device) {
+    e = cudaMalloc(reinterpret_cast<void**>(&out), bytes);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      return fail(st, MEQ_ERR_OOM, "scratch allocation for meq_read_update failed");
+    }
+  }
+  e = launch_update(st->ctx, M, i, out, st->last_stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st->last_stream);
+  if (e == cudaSuccess && !on_device) e = cudaMemcpy(dst, out, bytes, cudaMemcpyDefault);
+  if (!on_device) cudaFree(out);
+  return e == cudaSuccess ? MEQ_OK : cuda_fail(st, e, "meq_read_update");
+}
+
 meq_status meq_read_stats(meq_state* st, int i, float* r, float* c, double* gamma_r, double* gamma_c, int* direction) {
   meq_status ms = check_index(st, i);
   if (ms != MEQ_OK) return ms;
@@ -1108,10 +1078,12 @@ meq_status meq_ns_cv_trajectory(const float* h, int64_t rows, int64_t cols, int 
   o.ns_steps = 1;
   if (!valid_options(o, &why)) return fail(nullptr, MEQ_ERR_INVALID_ARG, why);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  // scratch: W (rows x cols, left unchanged by lr = 0), r, c, the two CVs, the direction
+  // scratch: W (rows x cols, left unchanged by lr = 0), r, c, the two CVs and
+  // the direction, then the statistics kernels' partial sums
   const int64_t wb = round_up(rows * cols * 4, 256), rb = round_up(rows * 4, 256), cb = round_up(cols * 4, 256);
+  const int64_t pb = round_up(row_col_stats_scratch_floats(rows, cols) * 4, 256);
   char* tmp = nullptr;
-  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&tmp), static_cast<size_t>(wb + rb + cb + 256));
+  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&tmp), static_cast<size_t>(wb + rb + cb + 256 + pb));
   if (e != cudaSuccess) {
     cudaGetLastError();
     return fail(nullptr, MEQ_ERR_OOM, "scratch allocation failed");
@@ -1121,11 +1093,17 @@ meq_status meq_ns_cv_trajectory(const float* h, int64_t rows, int64_t cols, int 
   float* c = reinterpret_cast<float*>(tmp + wb + rb);
   double* g = reinterpret_cast<double*>(tmp + wb + rb + cb);
   int* d = reinterpret_cast<int*>(g + 2);
+  float* parts = reinterpret_cast<float*>(tmp + wb + rb + cb + 256);
   meq_status ms = MEQ_OK;
   e = cudaMemsetAsync(w, 0, static_cast<size_t>(rows * cols * 4), s);
   if (e != cudaSuccess) ms = cuda_fail(nullptr, e, "cudaMemsetAsync");
-  // k = 0: X_0 = H / ||H||_F has the CVs of H (Eq. (8) is scale-free)
-  if (ms == MEQ_OK) ms = meq_row_col_stats_noalloc(h, rows, cols, eps, o.tie_atol, r, c, g, d, s);
+  // k = 0: the statistics of X_0 = H / ||H||_F (the threshold eps applies to
+  // the RMS of X_0, as for every later iterate), in this call's own scratch
+  if (ms == MEQ_OK) {
+    const char* what = "";
+    e = launch_row_col_stats(h, rows, cols, eps, o.tie_atol, 1, parts, r, c, g, d, s, &what);
+    if (e != cudaSuccess) ms = cuda_fail(nullptr, e, what);
+  }
   double hg[2] = {0.0, 0.0};
   if (ms == MEQ_OK) {
     e = cudaMemcpyAsync(hg, g, sizeof(hg), cudaMemcpyDeviceToHost, s);
@@ -1229,7 +1207,7 @@ meq_status meq_read_profile(meq_state* st, double* phase_ms, int64_t* steps) {
 int meq_kernels_per_step(const meq_state* st) { return st ? st->kernels_per_step : 0; }
 
 int meq_ns_gemm_launches_per_step(const meq_state* st) {
-  return st ? (st->use_persist ? 1 : static_cast<int>(st->gemm.size())) : 0;
+  return st ? static_cast<int>(st->gemm.size()) : 0;
 }
 
 meq_status meq_debug_wait_selftest(meq_state* st, float timeout_ms) {

@@ -53,6 +53,8 @@ cudaError_t launch_colpart(const LaunchCtx& L, cudaStream_t st);   // remaining 
 cudaError_t launch_cast_x0(const LaunchCtx& L, bool fp16, cudaStream_t st);
 cudaError_t launch_stats(const LaunchCtx& L, cudaStream_t st);  // finalize of the fused statistics
 cudaError_t launch_apply(const LaunchCtx& L, cudaStream_t st);
+// U~ of entry mi (the update apply_kernel applies) into dst (device, M.m x M.n fp32).
+cudaError_t launch_update(const LaunchCtx& L, const MatInfo& M, int mi, float* dst, cudaStream_t st);
 cudaError_t launch_wait_selftest(const int* flag, int* err, unsigned long long timeout_ns, cudaStream_t st);
 
 }  // namespace meq

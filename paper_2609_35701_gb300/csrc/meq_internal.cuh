@@ -7,6 +7,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <string>
 #include <utility>
 
 namespace meq {
@@ -22,13 +23,10 @@ enum DevErr : int {
   DEV_TIMEOUT_DRAIN = 0x105,     // waiting for in-flight copies / MMAs at exit
   DEV_TIMEOUT_SCHED_PUT = 0x106, // tile scheduler waited too long for a free slot of the tile ring
   DEV_TIMEOUT_SCHED_TAKE = 0x107,// a role waited too long for its next tile index
-  DEV_TIMEOUT_DEP = 0x108,       // one-launch NS: a tile waited too long for the product it reads
-  DEV_TIMEOUT_SIG = 0x109,       // one-launch NS: waited too long for a tile's stores or their report slot
   DEV_TIMEOUT_TEST = 0x1FF,      // the wait-timeout self test
 };
 
 constexpr int kMaxGroups = 8;        // shape groups per GEMM launch
-constexpr int kMaxSegs = 48;         // (product, shape group) segments of the one-launch NS (30 KB of parameters)
 constexpr int kNsEpilogueWarps = 8;  // epilogue warps per CTA of the NS GEMM kernel
 
 // U of the hidden weights is stored as fp16(kUScale * U). Every entry of U
@@ -109,21 +107,13 @@ struct GemmGroup {
   int32_t mode;           // GemmMode of the product
   uint32_t idesc;         // tcgen05 instruction descriptor
   int32_t b_mn_major;     // 1: B operand tile is MN-major (XUPD)
-  // One-launch NS only: this segment's product index (row of the completion
-  // counters), its matrices' first counter slot, and the count each of its
-  // matrices waits for in the previous product's row (0: none).
-  int32_t prod;
-  int32_t mat_base;
-  int32_t dep_target;
   int32_t tma_out;        // 1: the output leaves by TMA stores through tmO (else 16-byte thread stores)
 };
 
-// One GEMM launch: kSegs segments (one product's shape groups, or, with
-// kSegs = kMaxSegs, every product's for the one-launch NS), taken as one tile
-// queue in segment order.
-template <int kSegs>
-struct GemmParamsT {
-  GemmGroup g[kSegs];
+// One GEMM launch: one product's shape groups, taken as one tile queue in
+// group order.
+struct GemmParams {
+  GemmGroup g[kMaxGroups];
   int32_t ngroups;
   int32_t total_tiles;
   int32_t reverse;         // 1: tiles are taken in reverse order (alternates between launches)
@@ -131,15 +121,9 @@ struct GemmParamsT {
   int* err;                // device error word
   int* sched;              // tile queue: [0] tiles handed out beyond the first wave, [1] units done;
                            // zero between launches (the last unit to finish resets both)
-  int* done;               // one-launch NS: [product][slot] epilogue-warp completions per matrix,
-                           // zero between launches (reset with the tile queue)
-  int32_t nslots;          // slots per product row of `done`
-  int32_t nprod;           // product rows of `done`
   int32_t debug_skip_load; // tests: the first pair's leader skips its first stage's loads
   unsigned long long timeout_ns;
 };
-using GemmParams = GemmParamsT<kMaxGroups>;
-using PersistParams = GemmParamsT<kMaxSegs>;
 
 // Programmatic dependent launch: a kernel lets the next one in the stream be
 // scheduled as soon as it starts, and waits for its predecessor's results
@@ -177,10 +161,18 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 // Launchers (defined in the .cu files).
 cudaError_t prepare_ns_gemm();  // sets the kernel's dynamic shared-memory limit (per device)
 cudaError_t launch_ns_gemm(const GemmParams& p, int grid, int pair, cudaStream_t st);  // pair: 1 or 2 CTAs per tile
-// Every NS product in one cooperative launch of CTA pairs (grid = 2 x pairs).
-cudaError_t launch_ns_gemm_persistent(const PersistParams& p, int grid, cudaStream_t st);
-// CTA pairs of the one-launch NS that can be resident at once (0 if it cannot run).
-int ns_gemm_persistent_max_pairs();
 int ns_gemm_smem_bytes(int pair);
+
+// Row / column statistics of one fp32 matrix (Eqs. (7), (8), (11)) with
+// caller-given scratch of row_col_stats_scratch_floats(rows, cols) floats;
+// frob = 1 describes U / ||U||_F instead of U. On failure *failed names the
+// launch.
+int64_t row_col_stats_scratch_floats(int64_t rows, int64_t cols);
+cudaError_t launch_row_col_stats(const float* U, int64_t rows, int64_t cols, float eps, float tie_atol, int frob,
+                                 float* scratch, float* r, float* c, double* gammas, int* direction, cudaStream_t st,
+                                 const char** failed);
+
+// Error text of the last failed call made without a state (meq_last_error(NULL)).
+void set_global_error(const std::string& msg);
 
 }  // namespace meq

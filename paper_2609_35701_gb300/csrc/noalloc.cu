@@ -10,10 +10,13 @@
 // file-scope __device__ array of fixed size that every GPU which loads the
 // library holds until the process exits.
 //
-// It sums squares over 32-row slabs and forms the CVs in two passes, all in
+// It sums squares over 32-row slabs, folds the column partials with one
+// thread per column (slabs in order), and forms the CVs in two passes, all in
 // fp32 like the full step's statistics, so results agree with meq_read_stats
-// up to fp32 summation order.
+// up to fp32 summation order. The same kernels, given scratch that the caller
+// allocated, give the first point of the CV trajectory (meq_ns_cv_trajectory).
 #include <mutex>
+#include <string>
 
 #include "../../include/meq.h"
 #include "meq_elementwise.cuh"
@@ -22,6 +25,7 @@ namespace {
 
 constexpr int kNaThreads = 256;
 constexpr int kNaSlab = 32;
+constexpr int kNaFoldThreads = 256;
 constexpr int kNaFinThreads = 1024;
 constexpr int kMaxDevices = 64;
 
@@ -98,25 +102,49 @@ __global__ void __launch_bounds__(kNaThreads) na_stats_kernel(const float* __res
   }
 }
 
-// r, c (Eq. (7)), gamma_r, gamma_c (Eq. (8)) and the side (Eq. (11)), all fp32.
-__global__ void __launch_bounds__(kNaFinThreads) na_finalize_kernel(int64_t m, int64_t n, float delta, float tie_atol,
-                                                                    const float* __restrict__ scratch,
-                                                                    float* __restrict__ r, float* __restrict__ c,
-                                                                    double* __restrict__ gammas,
-                                                                    int* __restrict__ direction) {
-  __shared__ float shf[32];
+// r (Eq. (7)) from the row sums of squares and c from the column partials,
+// one thread per row / column; each column sums its slabs in slab order.
+__global__ void __launch_bounds__(kNaFoldThreads) na_fold_kernel(int64_t m, int64_t n, const float* __restrict__ scratch,
+                                                                 float* __restrict__ r, float* __restrict__ c) {
+  const int64_t t = static_cast<int64_t>(blockIdx.x) * kNaFoldThreads + threadIdx.x;
   const int64_t nslabs = (m + kNaSlab - 1) / kNaSlab;
   const float* rowss = scratch;
   const float* cpart = scratch + m;
-  const float inv_n = 1.0f / static_cast<float>(n);
-  const float inv_m = 1.0f / static_cast<float>(m);
-  for (int64_t i = threadIdx.x; i < m; i += blockDim.x) r[i] = sqrtf(rowss[i] * inv_n);
-  for (int64_t j = threadIdx.x; j < n; j += blockDim.x) {
+  if (t < m) r[t] = sqrtf(rowss[t] * (1.0f / static_cast<float>(n)));
+  if (t < n) {
     float acc = 0.f;
-    for (int64_t k = 0; k < nslabs; ++k) acc += cpart[k * n + j];
-    c[j] = sqrtf(acc * inv_m);
+    int64_t k = 0;
+    for (; k + 4 <= nslabs; k += 4) {  // four loads in flight, added in slab order
+      const float a0 = cpart[k * n + t], a1 = cpart[(k + 1) * n + t];
+      const float a2 = cpart[(k + 2) * n + t], a3 = cpart[(k + 3) * n + t];
+      acc += a0;
+      acc += a1;
+      acc += a2;
+      acc += a3;
+    }
+    for (; k < nslabs; ++k) acc += cpart[k * n + t];
+    c[t] = sqrtf(acc * (1.0f / static_cast<float>(m)));
   }
-  __syncthreads();
+}
+
+// gamma_r, gamma_c (Eq. (8), over entries > delta) and the side (Eq. (11)),
+// all fp32, in one block. With frob set, r and c are first divided by
+// ||U||_F (from the row sums of squares, fixed order), so that they and the
+// threshold describe X = U / ||U||_F; a zero U gives zeros.
+__global__ void __launch_bounds__(kNaFinThreads) na_cv_kernel(int64_t m, int64_t n, float delta, float tie_atol, int frob,
+                                                              const float* __restrict__ scratch, float* __restrict__ r,
+                                                              float* __restrict__ c, double* __restrict__ gammas,
+                                                              int* __restrict__ direction) {
+  __shared__ float shf[32];
+  if (frob) {
+    float tot = 0.f;
+    for (int64_t i = threadIdx.x; i < m; i += blockDim.x) tot += scratch[i];
+    tot = na_block_sum_f32(tot, shf);
+    const float inv = tot > 0.f ? 1.0f / sqrtf(tot) : 0.f;
+    for (int64_t i = threadIdx.x; i < m; i += blockDim.x) r[i] *= inv;
+    for (int64_t j = threadIdx.x; j < n; j += blockDim.x) c[j] *= inv;
+    __syncthreads();
+  }
   float gam[2];
   for (int side = 0; side < 2; ++side) {
     const float* v = side == 0 ? r : c;
@@ -144,38 +172,89 @@ __global__ void __launch_bounds__(kNaFinThreads) na_finalize_kernel(int64_t m, i
   }
 }
 
+// Plain launch (no attributes) that returns this launch's own status.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_plain(void (*kernel)(KArgs...), unsigned grid, unsigned block, cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.stream = st;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 // Device address of the scratch array on the current device, looked up once
 // per device (the host-side symbol is only a stand-in, not a device address).
-meq_status scratch_address(float** out) {
+cudaError_t scratch_address(float** out) {
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MEQ_ERR_CUDA;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lock(g_setup_mu);
   if (!g_scratch_addr[dev]) {
     void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_stats_scratch) != cudaSuccess || p == nullptr) return MEQ_ERR_CUDA;
+    e = cudaGetSymbolAddress(&p, g_stats_scratch);
+    if (e != cudaSuccess) return e;
+    if (p == nullptr) return cudaErrorInvalidSymbol;
     g_scratch_addr[dev] = static_cast<float*>(p);
   }
   *out = g_scratch_addr[dev];
-  return MEQ_OK;
+  return cudaSuccess;
+}
+
+meq_status na_fail(meq_status s, const std::string& msg) {
+  meq::set_global_error(msg);
+  return s;
 }
 
 }  // namespace
 
+namespace meq {
+
+int64_t row_col_stats_scratch_floats(int64_t rows, int64_t cols) {
+  return rows + (rows + kNaSlab - 1) / kNaSlab * cols;
+}
+
+cudaError_t launch_row_col_stats(const float* U, int64_t rows, int64_t cols, float eps, float tie_atol, int frob,
+                                 float* scratch, float* r, float* c, double* gammas, int* direction, cudaStream_t st,
+                                 const char** failed) {
+  const int64_t nslabs = (rows + kNaSlab - 1) / kNaSlab;
+  *failed = "statistics launch";
+  cudaError_t e = launch_plain(na_stats_kernel, static_cast<unsigned>(nslabs), kNaThreads, st, U, rows, cols, scratch);
+  if (e != cudaSuccess) return e;
+  *failed = "column fold launch";
+  const int64_t len = rows > cols ? rows : cols;
+  e = launch_plain(na_fold_kernel, static_cast<unsigned>((len + kNaFoldThreads - 1) / kNaFoldThreads), kNaFoldThreads,
+                   st, rows, cols, static_cast<const float*>(scratch), r, c);
+  if (e != cudaSuccess) return e;
+  *failed = "CV launch";
+  return launch_plain(na_cv_kernel, 1u, kNaFinThreads, st, rows, cols, eps, tie_atol, frob,
+                      static_cast<const float*>(scratch), r, c, gammas, direction);
+}
+
+}  // namespace meq
+
 extern "C" meq_status meq_row_col_stats_noalloc(const float* U, int64_t rows, int64_t cols, float eps, float tie_atol,
                                                 float* r, float* c, double* gammas, int* direction,
                                                 void* cuda_stream) {
-  if (!U || !r || !c || !gammas || !direction) return MEQ_ERR_INVALID_ARG;
-  if (rows <= 0 || cols <= 0 || rows > (int64_t(1) << 20) || cols > (int64_t(1) << 20)) return MEQ_ERR_INVALID_ARG;
-  if (!(eps >= 0.f) || !(tie_atol >= 0.f)) return MEQ_ERR_INVALID_ARG;
-  const int64_t nslabs = (rows + kNaSlab - 1) / kNaSlab;
-  if (rows + nslabs * cols > kScratchFloats) return MEQ_ERR_INVALID_ARG;  // beyond the fixed scratch
+  if (!U || !r || !c || !gammas || !direction)
+    return na_fail(MEQ_ERR_INVALID_ARG, "meq_row_col_stats_noalloc: U, r, c, gammas and direction must not be NULL");
+  if (rows <= 0 || cols <= 0 || rows > (int64_t(1) << 20) || cols > (int64_t(1) << 20))
+    return na_fail(MEQ_ERR_INVALID_ARG, "meq_row_col_stats_noalloc: rows and cols must be in 1..2^20");
+  if (!(eps >= 0.f) || !(tie_atol >= 0.f))
+    return na_fail(MEQ_ERR_INVALID_ARG, "meq_row_col_stats_noalloc: eps and tie_atol must be >= 0");
+  const int64_t need = meq::row_col_stats_scratch_floats(rows, cols);
+  if (need > kScratchFloats)
+    return na_fail(MEQ_ERR_INVALID_ARG, "meq_row_col_stats_noalloc: " + std::to_string(rows) + " x " +
+                                            std::to_string(cols) + " needs " + std::to_string(need) +
+                                            " floats of scratch, above the fixed " + std::to_string(kScratchFloats));
   float* scratch = nullptr;
-  meq_status s = scratch_address(&scratch);
-  if (s != MEQ_OK) return s;
-  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
-  na_stats_kernel<<<static_cast<unsigned>(nslabs), kNaThreads, 0, st>>>(U, rows, cols, scratch);
-  if (cudaGetLastError() != cudaSuccess) return MEQ_ERR_CUDA;
-  na_finalize_kernel<<<1, kNaFinThreads, 0, st>>>(rows, cols, eps, tie_atol, scratch, r, c, gammas, direction);
-  if (cudaGetLastError() != cudaSuccess) return MEQ_ERR_CUDA;
+  cudaError_t e = scratch_address(&scratch);
+  if (e != cudaSuccess)
+    return na_fail(MEQ_ERR_CUDA, std::string("meq_row_col_stats_noalloc: scratch address lookup: ") + cudaGetErrorString(e));
+  const char* what = "";
+  e = meq::launch_row_col_stats(U, rows, cols, eps, tie_atol, 0, scratch, r, c, gammas, direction,
+                                static_cast<cudaStream_t>(cuda_stream), &what);
+  if (e != cudaSuccess)
+    return na_fail(MEQ_ERR_CUDA, std::string("meq_row_col_stats_noalloc: ") + what + ": " + cudaGetErrorString(e));
   return MEQ_OK;
 }

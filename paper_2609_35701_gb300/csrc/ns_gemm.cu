@@ -20,7 +20,7 @@
 // X is stored scaled by a power of two alpha so its entries stay in the
 // normal range of fp16; the epilogues undo the scale in fp32.
 //
-// Roles (320 threads, one CTA per SM; one-launch NS below):
+// Roles (320 threads, one CTA per SM):
 //   warp 0 : TMA producer (one thread), shared-memory ring of 4 stages
 //            (single CTA) or 6 (CTA pair)
 //   warp 1 : TMEM allocator and tcgen05.mma issuer (one thread; with CTA
@@ -40,14 +40,6 @@
 // leave by TMA stores, X and U by coalesced 16-byte stores from the threads
 // (the update launches keep the SM's TMA unit for their operand loads).
 //
-// The same kernel, instantiated with kMaxSegs segments and two more warps
-// (384 threads), runs every product of the iteration in one cooperative
-// launch (option ns_single_launch): the products' shape groups are segments
-// of one tile queue in product order, a dependency warp acquires for each
-// tile the completion count of its matrix in the previous product before the
-// producer may load it, and a signal warp releases a tile's count once the
-// CTA's epilogue warps report its TMA stores landed.
-//
 // Every mbarrier wait is bounded (time and iteration count). On expiry the
 // waiting role records an error code, the others see it and stop, in-flight
 // TMA copies and MMAs are drained with bounded waits, TMEM is freed and the
@@ -61,14 +53,6 @@ constexpr int BM = 128, BN = 256, BK = 64, UK = 16;  // per-CTA rows, tile colum
 constexpr int A_BYTES = BM * BK * 2;                 // 16 KB
 constexpr int NUM_EPI_WARPS = kNsEpilogueWarps;      // two per TMEM lane quarter
 constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
-// The one-launch NS adds two warps per CTA: one acquires each tile's
-// dependency ahead of the producer, one releases each tile's completion
-// count, so that neither GPU-scope operation sits on a producer or epilogue
-// path (a release stalls its warp for about 2 us).
-constexpr int NUM_THREADS_P = NUM_THREADS + 64;
-constexpr int DEP_WARP = 2 + NUM_EPI_WARPS, SIG_WARP = DEP_WARP + 1;
-constexpr int DEP_Q = 32;  // ring of "dependency acquired" barriers, one-launch NS
-constexpr int SIG_Q = 8;   // ring of "tile stored" barriers (and their free barriers), one-launch NS
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int SLOT_BYTES = 2048;                     // one 32 x 32 16-bit block (two per epilogue warp)
 constexpr int SCHED_D = 16;                          // entries of the tile-index ring
@@ -86,9 +70,8 @@ struct Cfg {
   static constexpr int B_BYTES = BN_LOCAL * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int STAGES = kPair == 1 ? 4 : 6;
-  // full, empty, tmem full x2, tmem empty x2, drain, tile ring full / empty,
-  // then (one-launch NS) dependency acquired, tile stored, stored slot free
-  static constexpr int NUM_BARS = 2 * STAGES + 4 + 1 + 2 * SCHED_D + DEP_Q + 2 * SIG_Q;
+  // full, empty, tmem full x2, tmem empty x2, drain, tile ring full / empty
+  static constexpr int NUM_BARS = 2 * STAGES + 4 + 1 + 2 * SCHED_D;
   static constexpr int SMEM_EPI_OFF = STAGES * STAGE_BYTES;
   static constexpr int SMEM_BAR_OFF = SMEM_EPI_OFF + NUM_EPI_WARPS * 2 * SLOT_BYTES;
   // barriers, the TMEM address word (16 bytes reserved), the tile ring
@@ -192,42 +175,6 @@ __device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap
       "l"(reinterpret_cast<uint64_t>(tm)), "r"(bar_cluster), "r"(x), "r"(y), "r"(z)
       : "memory");
 }
-// Completion counters of the one-launch NS (global memory, GPU scope).
-__device__ __forceinline__ int ld_acquire_gpu(const int* ptr) {
-  int v;
-  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(ptr) : "memory");
-  return v;
-}
-__device__ __forceinline__ void red_release_gpu_add(int* ptr, int v) {
-  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(ptr), "r"(v) : "memory");
-}
-// Orders this thread's generic-proxy view of global memory with its TMA
-// (async-proxy) accesses, in both directions.
-__device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
-// 16-byte load through L2 only (the data may have been written by another SM
-// during this launch, so neither L1 nor the read-only path may serve it).
-__device__ __forceinline__ uint4 ld_cg_v4(const void* ptr) {
-  uint4 v;
-  asm volatile("ld.global.cg.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(ptr));
-  return v;
-}
-// Bounded wait (one thread) until *ptr >= target, with acquire at GPU scope.
-__device__ bool wait_count(const int* ptr, int target, int* err, int code, uint64_t timeout_ns) {
-  if (ld_acquire_gpu(ptr) >= target) return true;
-  const uint64_t t0 = global_ns();
-  for (uint32_t it = 1;; ++it) {
-    __nanosleep(128);
-    if (ld_acquire_gpu(ptr) >= target) return true;
-    if ((it & 15u) == 0) {
-      if (*reinterpret_cast<volatile int*>(err) != 0) return false;
-      if (global_ns() - t0 > timeout_ns || it >= (1u << 26)) {
-        atomicCAS(err, 0, code);
-        return false;
-      }
-    }
-  }
-}
-
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
@@ -348,8 +295,7 @@ struct TileCoord {
 // over tiles_m x tiles_n; symmetric outputs (Gram, polynomial) run tn-major
 // over the tiles with tm * TILE_M < (tn + 1) * 256, i.e. those holding a
 // 32 x 32 block on or above the diagonal.
-template <int kSegs>
-__device__ __forceinline__ int find_segment(const GemmParamsT<kSegs>& p, int t) {
+__device__ __forceinline__ int find_segment(const GemmParams& p, int t) {
   int lo = 0, hi = p.ngroups - 1;  // the last segment whose tile_begin <= t
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
@@ -358,8 +304,8 @@ __device__ __forceinline__ int find_segment(const GemmParamsT<kSegs>& p, int t) 
   }
   return lo;
 }
-template <int kPair, int kSegs>
-__device__ __forceinline__ TileCoord decode_tile(const GemmParamsT<kSegs>& p, int t) {
+template <int kPair>
+__device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
   if (p.reverse) t = p.total_tiles - 1 - t;
   const int g = find_segment(p, t);
   const GemmGroup& G = p.g[g];
@@ -477,22 +423,8 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_reads() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 // Every committed store has completed.
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-// Every committed store but those of the `keep` most recent groups (0..4) has completed.
-__device__ __forceinline__ void bulk_wait_keep(int keep) {
-  switch (keep) {
-    case 0: asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); break;
-    case 1: asm volatile("cp.async.bulk.wait_group 1;" ::: "memory"); break;
-    case 2: asm volatile("cp.async.bulk.wait_group 2;" ::: "memory"); break;
-    case 3: asm volatile("cp.async.bulk.wait_group 3;" ::: "memory"); break;
-    default: asm volatile("cp.async.bulk.wait_group 4;" ::: "memory"); break;
-  }
-}
-template <int kPair, int kSegs>
-__global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREADS, 1)
-    ns_gemm_kernel(const __grid_constant__ GemmParamsT<kSegs> p) {
-  // The one-launch NS (every product, completion counters) is the kMaxSegs
-  // instantiation; the per-product launches compile without its code.
-  constexpr bool kPersistent = kSegs == kMaxSegs;
+template <int kPair>
+__global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_constant__ GemmParams p) {
   using C_ = Cfg<kPair>;
   constexpr int STAGES = C_::STAGES;
   constexpr int STAGE_BYTES = C_::STAGE_BYTES;
@@ -511,9 +443,6 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
 #define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
 #define SFULL_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + (i)))
 #define SEMPTY_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + SCHED_D + (i)))
-#define DEPOK_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + 2 * SCHED_D + (i)))
-#define STORED_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + 2 * SCHED_D + DEP_Q + (i)))
-#define STFREE_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + 2 * SCHED_D + DEP_Q + SIG_Q + (i)))
   const uint32_t ring = tmem_slot + 16;  // SCHED_D tile indices
 
   const int warp = threadIdx.x >> 5;
@@ -539,16 +468,8 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
     for (int i = 0; i < SCHED_D; ++i) {
       mbar_init(SFULL_BAR(i), 1);
       // consumers of each index: the MMA issuer and the epilogue warps of the
-      // leader, and (pair) the peer's producer and epilogue warps; the
-      // dependency and signal warps of both CTAs in the one-launch NS
-      mbar_init(SEMPTY_BAR(i), kPair * (1 + NUM_EPI_WARPS + (kPersistent ? 2 : 0)));
-    }
-    if (kPersistent) {
-      for (int i = 0; i < DEP_Q; ++i) mbar_init(DEPOK_BAR(i), 1);
-      for (int i = 0; i < SIG_Q; ++i) {
-        mbar_init(STORED_BAR(i), NUM_EPI_WARPS);
-        mbar_init(STFREE_BAR(i), 1);
-      }
+      // leader, and (pair) the peer's producer and epilogue warps
+      mbar_init(SEMPTY_BAR(i), kPair * (1 + NUM_EPI_WARPS));
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     for (int g = 0; g < p.ngroups; ++g) {
@@ -616,47 +537,20 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
       bool ok = true;
       int t = unit;
       int fetched = 0;  // leader: the counter value for the next tile
-      int t_ahead = 0;  // leader, one-launch NS: index n + 1, published when tile n starts
       for (int n = 0; ok; ++n) {
-        if (kPersistent && leader) {
-          // one tile ahead, so that the dependency warps see each index early
-          if (n == 0) {
-            if (!sched_put(0, t)) break;
-            if (t < p.total_tiles) {
-              t_ahead = nunits + atomicAdd(p.sched, 1);
-              if (!sched_put(1, t_ahead)) break;
-            }
-          } else {
-            t = t_ahead;
-            if (t < p.total_tiles) {
-              t_ahead = nunits + fetched;
-              if (!sched_put(n + 1, t_ahead)) break;
-            }
-          }
-        } else {
-          if (n > 0 && leader) t = nunits + fetched;
-          if (leader ? !sched_put(n, t) : !sched_take(n, t)) break;
-        }
+        if (n > 0 && leader) t = nunits + fetched;
+        if (leader ? !sched_put(n, t) : !sched_take(n, t)) break;
         if (t >= p.total_tiles) break;
         const TileCoord c = decode_tile<kPair>(p, t);
         const GemmGroup& G = p.g[c.g];
-        if (kPersistent) {
-          // the previous product of this matrix is complete (acquired by the
-          // dependency warp), and visible to TMA
-          if (!wait_bounded(DEPOK_BAR(n % DEP_Q), (n / DEP_Q) & 1, err, DEV_TIMEOUT_DEP, tmo)) {
-            ok = false;
-            break;
-          }
-          fence_proxy_async_global();
-        }
         // The next index is fetched while this tile's operands are requested;
         // its value is first read at the top of the next iteration.
         if (leader) fetched = atomicAdd(p.sched, 1);
         const int nk = (G.K + BK - 1) / BK;
-        // Mode, descriptor and B layout are per segment in the one-launch NS
-        // and per launch otherwise, where reading them at a fixed index keeps
-        // them launch-uniform for the compiler (measured: 2% of the step).
-        const int b_mn_major = kPersistent ? G.b_mn_major : p.g[0].b_mn_major;
+        // Mode, descriptor and B layout are per launch: reading them at a
+        // fixed index keeps them launch-uniform for the compiler (measured:
+        // 2% of the step).
+        const int b_mn_major = p.g[0].b_mn_major;
         const int arow = c.tm * TILE_M + static_cast<int>(rank) * BM;
         const int bcol = c.tn * BN + static_cast<int>(rank) * C_::BN_LOCAL;
         // A diagonal tile of a symmetric product (X X^T, A A) has each CTA's
@@ -687,7 +581,7 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
             const uint32_t fb = leader ? FULL_BAR(stage) : map_to_rank(FULL_BAR(stage), 0);
             // tests (debug_skip_load): the stage is armed but this CTA's half never
             // comes, so the MMA issuer's bounded wait on it expires
-            const bool skip = !kPersistent && p.debug_skip_load && leader && unit == 0 && n == 0 && kb == 0;
+            const bool skip = p.debug_skip_load && leader && unit == 0 && n == 0 && kb == 0;
             if (!skip) {
               tma_load_3d_pair(sa, &G.tmA, fb, kb * BK, arow, c.mat);
               if (b_is_a) {
@@ -731,8 +625,8 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
         const TileCoord c = decode_tile<kPair>(p, t);
         const GemmGroup& G = p.g[c.g];
         const int nk = (G.K + BK - 1) / BK;
-        const int b_mn_major = kPersistent ? G.b_mn_major : p.g[0].b_mn_major;
-        const uint32_t idesc = kPersistent ? G.idesc : p.g[0].idesc;
+        const int b_mn_major = p.g[0].b_mn_major;
+        const uint32_t idesc = p.g[0].idesc;
         const uint32_t b_lbo = b_mn_major ? (64u * BK * 2u) : 16u;
         // diagonal tile of a symmetric product: B is read from the A half (the producer loads A only)
         const bool b_is_a = kPair == 2 && G.sym && !b_mn_major && c.tm * TILE_M == c.tn * BN;
@@ -796,27 +690,6 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
     // The leader's tmem-empty barrier counts the epilogue warps of both CTAs.
     const uint32_t tempty_target0 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(0), 0) : TEMPTY_BAR(0);
     const uint32_t tempty_target1 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(1), 0) : TEMPTY_BAR(1);
-    // One-launch NS: once a tile's stores have landed, each warp tells the
-    // signal warp (a CTA barrier per tile, in tile order), which releases the
-    // tile's count for the next product. The report of tile n is deferred to
-    // the end of tile n + 1's epilogue, by when tile n's stores have long
-    // completed (the wait skips tile n + 1's own store groups) -- unless tile
-    // n + 1's accumulator is not ready yet, in which case it is sent before
-    // waiting (tile n + 1 may depend on it).
-    // (Every output another tile waits for leaves by TMA stores: the host
-    // sets tma_out on every product but the last.)
-    int pend = -1;  // ordinal of the tile whose report is deferred
-    auto signal_pending = [&](int keep_groups) {
-      __syncwarp();
-      if (lane == 0) {
-        bulk_wait_keep(keep_groups);
-        fence_proxy_async_global();
-        // the signal warp has consumed this slot's previous tile
-        wait_bounded(STFREE_BAR(pend % SIG_Q), ((pend / SIG_Q) & 1) ^ 1u, err, DEV_TIMEOUT_SIG, tmo);
-        mbar_arrive_local(STORED_BAR(pend % SIG_Q));  // release (CTA scope)
-      }
-      pend = -1;
-    };
     for (int n = 0;; ++n) {
       int t = 0, got = 1;
       if (lane == 0) got = sched_take(n, t) ? 1 : 0;
@@ -825,19 +698,8 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
       if (!got || t >= p.total_tiles) break;
       const TileCoord c = decode_tile<kPair>(p, t);
       const GemmGroup& G = p.g[c.g];
-      const int mode = kPersistent ? G.mode : p.g[0].mode;  // one mode per launch (a launch-uniform read)
-      if (pend >= 0 && !__all_sync(0xffffffffu, mbar_try_wait(TFULL_BAR(acc), acc_phase))) signal_pending(0);
+      const int mode = p.g[0].mode;  // one mode per launch (a launch-uniform read)
       if (!wait_bounded_warp(TFULL_BAR(acc), acc_phase, err, DEV_TIMEOUT_EPI, tmo)) break;
-      if (kPersistent && mode == MODE_POLY) {
-        // The A read below comes from the previous product of this launch:
-        // synchronise with the dependency warp's acquire of it (CTA scope).
-        // It is done by now, since the tile's operands waited for it; waiting
-        // before the accumulator could deadlock (the count may still lack
-        // this warp's own deferred report).
-        int okd = 1;
-        if (lane == 0) okd = wait_bounded(DEPOK_BAR(n % DEP_Q), (n / DEP_Q) & 1, err, DEV_TIMEOUT_DEP, tmo) ? 1 : 0;
-        if (!__shfl_sync(0xffffffffu, okd, 0)) break;
-      }
       tc_fence_after();
       const int row0 = c.tm * TILE_M + static_cast<int>(rank) * BM + q * 32;
       const int R = row0 / 32;  // 32-row block index
@@ -859,12 +721,11 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
           if (r < rows_valid) {
             const uint4* src = reinterpret_cast<const uint4*>(auxm + static_cast<int64_t>(row0 + r) * G.aux_ld +
                                                               static_cast<int64_t>(col0) * 2 + (lane & 3) * 16);
-            aux[i] = kPersistent ? ld_cg_v4(src) : __ldg(src);
+            aux[i] = __ldg(src);
           }
         }
       };
       if (mode == MODE_POLY && ch0 < nch) load_aux(c.tn * BN + ch0 * 32);
-      int tile_groups = 0;  // TMA store groups this warp commits for the tile
       for (int ch = ch0; ch < nch; ch += 2) {
         const int col0 = c.tn * BN + ch * 32;
         const int C = c.tn * 8 + ch;
@@ -982,9 +843,7 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
           }
         }
         __syncwarp();  // reconverge before the next warp-wide tcgen05.ld
-        if (G.tma_out) ++tile_groups;
       }
-      if (pend >= 0) signal_pending(tile_groups);  // the previous tile, behind this tile's store groups
       if (mode == MODE_XLAST && row0 < G.M && row0 + lane < G.M)  // one partial per (tile column, half)
         G.rpart[(static_cast<int64_t>(c.mat) * G.tiles_n * 2 + c.tn * 2 + half) * G.M + row0 + lane] = rsum * kUInvScale2;
       tc_fence_before();
@@ -994,45 +853,9 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
       }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
-      if (kPersistent) pend = n;
     }
-    if (pend >= 0) signal_pending(0);
     // The outputs are in global memory before the CTA leaves.
     if (lane == 0) bulk_wait_all();
-    __syncwarp();
-  } else if (kPersistent && warp == DEP_WARP) {
-    // ---------------------------------------------------------------- dependency warp (one-launch NS)
-    // Acquires (GPU scope) the completion count each tile depends on, one
-    // tile ahead of the producer, and hands it on by a CTA barrier that the
-    // producer and the polynomial epilogue wait on.
-    if (lane == 0) {
-      for (int n = 0;; ++n) {
-        int t = 0;
-        if (!sched_take(n, t) || t >= p.total_tiles) break;
-        const TileCoord c = decode_tile<kPair>(p, t);
-        const GemmGroup& G = p.g[c.g];
-        if (G.dep_target > 0 &&
-            !wait_count(p.done + (G.prod - 1) * p.nslots + G.mat_base + c.mat, G.dep_target, err, DEV_TIMEOUT_DEP, tmo))
-          break;
-        mbar_arrive_local(DEPOK_BAR(n % DEP_Q));  // release (CTA scope)
-      }
-    }
-    __syncwarp();
-  } else if (kPersistent && warp == SIG_WARP) {
-    // ---------------------------------------------------------------- signal warp (one-launch NS)
-    // Once every epilogue warp of this CTA reports a tile stored, adds one to
-    // the tile's matrix count (release, GPU scope) for the next product.
-    if (lane == 0) {
-      for (int n = 0;; ++n) {
-        int t = 0;
-        if (!sched_take(n, t) || t >= p.total_tiles) break;
-        const TileCoord c = decode_tile<kPair>(p, t);
-        const GemmGroup& G = p.g[c.g];
-        if (!wait_bounded(STORED_BAR(n % SIG_Q), (n / SIG_Q) & 1, err, DEV_TIMEOUT_SIG, tmo)) break;
-        if (G.prod + 1 < p.nprod) red_release_gpu_add(p.done + G.prod * p.nslots + G.mat_base + c.mat, 1);
-        mbar_arrive_local(STFREE_BAR(n % SIG_Q));
-      }
-    }
     __syncwarp();
   }
 #undef FULL_BAR
@@ -1041,9 +864,6 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
 #undef TEMPTY_BAR
 #undef SFULL_BAR
 #undef SEMPTY_BAR
-#undef DEPOK_BAR
-#undef STORED_BAR
-#undef STFREE_BAR
 
   if (kPair == 2 && *reinterpret_cast<volatile int*>(err) != 0) {
     // After an early exit, give copies still in flight towards either CTA
@@ -1064,8 +884,6 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
     if (atomicAdd(p.sched + 1, 1) == nunits - 1) {
       p.sched[0] = 0;
       p.sched[1] = 0;
-      if (kPersistent)
-        for (int i = 0; i < p.nprod * p.nslots; ++i) p.done[i] = 0;
     }
   }
   if (warp == 1) {
@@ -1078,67 +896,17 @@ __global__ void __launch_bounds__(kSegs == kMaxSegs ? NUM_THREADS_P : NUM_THREAD
 
 }  // namespace
 
-static_assert(sizeof(PersistParams) <= 32000, "one-launch NS parameters exceed the kernel parameter space");
-
 int ns_gemm_smem_bytes(int pair) { return pair == 2 ? Cfg<2>::SMEM_BYTES : Cfg<1>::SMEM_BYTES; }
 
 cudaError_t prepare_ns_gemm() {
-  cudaError_t e = cudaFuncSetAttribute(ns_gemm_kernel<1, kMaxGroups>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       Cfg<1>::SMEM_BYTES);
+  cudaError_t e = cudaFuncSetAttribute(ns_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<1>::SMEM_BYTES);
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(ns_gemm_kernel<2, kMaxGroups>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           Cfg<2>::SMEM_BYTES);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(ns_gemm_kernel<2, kMaxSegs>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              Cfg<2>::SMEM_BYTES);
+  return cudaFuncSetAttribute(ns_gemm_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<2>::SMEM_BYTES);
 }
 
 cudaError_t launch_ns_gemm(const GemmParams& p, int grid, int pair, cudaStream_t st) {
-  if (pair == 2)
-    return launch_pdl(ns_gemm_kernel<2, kMaxGroups>, dim3(grid), dim3(NUM_THREADS), Cfg<2>::SMEM_BYTES, st, 2, p);
-  return launch_pdl(ns_gemm_kernel<1, kMaxGroups>, dim3(grid), dim3(NUM_THREADS), Cfg<1>::SMEM_BYTES, st, 1, p);
-}
-
-int ns_gemm_persistent_max_pairs() {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(2);
-  cfg.blockDim = dim3(NUM_THREADS_P);
-  cfg.dynamicSmemBytes = Cfg<2>::SMEM_BYTES;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  int clusters = 0;
-  if (cudaOccupancyMaxActiveClusters(&clusters, ns_gemm_kernel<2, kMaxSegs>, &cfg) != cudaSuccess) {
-    cudaGetLastError();
-    return 0;
-  }
-  return clusters;
-}
-
-// Tiles of later products wait for earlier ones on other SMs, so every CTA
-// must be resident at once: a cooperative launch (one CTA per SM).
-cudaError_t launch_ns_gemm_persistent(const PersistParams& p, int grid, cudaStream_t st) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(NUM_THREADS_P);
-  cfg.dynamicSmemBytes = Cfg<2>::SMEM_BYTES;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[3];
-  attr[0].id = cudaLaunchAttributeCooperative;
-  attr[0].val.cooperative = 1;
-  attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = 2;
-  attr[1].val.clusterDim.y = 1;
-  attr[1].val.clusterDim.z = 1;
-  attr[2].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[2].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 3;
-  return cudaLaunchKernelEx(&cfg, ns_gemm_kernel<2, kMaxSegs>, p);
+  if (pair == 2) return launch_pdl(ns_gemm_kernel<2>, dim3(grid), dim3(NUM_THREADS), Cfg<2>::SMEM_BYTES, st, 2, p);
+  return launch_pdl(ns_gemm_kernel<1>, dim3(grid), dim3(NUM_THREADS), Cfg<1>::SMEM_BYTES, st, 1, p);
 }
 
 }  // namespace meq

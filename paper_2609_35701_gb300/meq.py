@@ -43,7 +43,6 @@ class MeqOptions(ctypes.Structure):
         ("ns_x0_fused", ctypes.c_int),
         ("update_rule", ctypes.c_int),
         ("debug_canaries", ctypes.c_int),
-        ("ns_single_launch", ctypes.c_int),
         ("debug_skip_load", ctypes.c_int),
     ]
 
@@ -56,7 +55,7 @@ EXPORTED = [
     "meq_init_state_kinds", "meq_state_bytes_kinds", "meq_ns_gemm_launches_per_step",
     "meq_read_direction_counts", "meq_reset_direction_counts", "meq_ns_cv_trajectory",
     "meq_check_canaries", "meq_canary_count", "meq_debug_corrupt_canary",
-    "meq_step_prepare", "meq_step_apply",
+    "meq_step_prepare", "meq_step_apply", "meq_read_update",
 ]
 HIDDEN, REMAINING_2D, VECTOR = 0, 1, 2  # meq_kind
 RULE_MEQMUON, RULE_MUON = 0, 1          # meq_update_rule
@@ -94,6 +93,8 @@ def _load():
     lib.meq_write_momentum.restype = I
     lib.meq_read_ns_output.argtypes = [P, I, P]
     lib.meq_read_ns_output.restype = I
+    lib.meq_read_update.argtypes = [P, I, P]
+    lib.meq_read_update.restype = I
     lib.meq_read_stats.argtypes = [P, I, P, P, ctypes.POINTER(D), ctypes.POINTER(D), ctypes.POINTER(I)]
     lib.meq_read_stats.restype = I
     lib.meq_kernels_per_step.argtypes = [P]
@@ -324,6 +325,13 @@ class MeqMuon:
         r, c = self.shapes[i]
         out = np.empty((r, c), np.float32)
         self._check(lib.meq_read_ns_output(self._st, i, out.ctypes.data))
+        return out
+
+    def read_update(self, i):
+        """The normalised update U~ the last step applied to entry i (meq_read_update)."""
+        r, c = self.shapes[i]
+        out = np.empty((r, c), np.float32)
+        self._check(lib.meq_read_update(self._st, i, out.ctypes.data))
         return out
 
     def read_stats(self, i):

@@ -138,6 +138,18 @@ def get_workload(name):
     return WORKLOADS[name]
 
 
+def first_layers(w: Workload, layers: int):
+    """The same workload over its first `layers` layers only (entries that
+    belong to no layer are kept): a smaller case of the same kernels, e.g. to
+    profile a model too large to capture whole."""
+    keep = [k for k, (n, _, _) in enumerate(w.shapes)
+            if not n.startswith("layers.") or int(n.split(".")[1]) < layers]
+    kinds = None if w.kinds is None else [w.kinds[k] for k in keep]
+    return Workload(f"{w.name}[:{layers} layers]", [w.shapes[k] for k in keep], w.base_sigma, w.pattern,
+                    scale_lo=w.scale_lo, scale_hi=w.scale_hi, steps=w.steps, lr=w.lr, momentum=w.momentum,
+                    weight_decay=w.weight_decay, eps=w.eps, seed=w.seed, extra=dict(w.extra), kinds=kinds)
+
+
 def custom_workload(shapes, pattern="both", base_sigma=0.01, seed=0, **kw):
     """A workload over an arbitrary list of (rows, cols) shapes (tests)."""
     sh = [(f"m{i}", int(r), int(c)) for i, (r, c) in enumerate(shapes)]

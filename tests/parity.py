@@ -9,6 +9,8 @@ the matrix): an element that is the difference of two O(RMS) fp32 terms
 carries an absolute rounding error of order 1e-7 * RMS, so a pure
 elementwise relative bound is not meaningful where the terms cancel.
   UPDATE_TOL    1e-2   final normalised update vs the oracle's, Frobenius
+  READBACK_TOL  1e-5   the update meq_read_update reports vs the one the
+                       parameters received (Eq. (14) solved for U~), Frobenius
   NEAR_TIE      0.1    relative CV gap under which the two sides may pick
                        different directions; the oracle's update under the
                        GPU's direction must then meet UPDATE_TOL
@@ -24,6 +26,7 @@ STATS_TOL = 1e-4
 PARAM_TOL = 1e-5
 UPDATE_TOL = 1e-2
 NEAR_TIE = 0.1
+READBACK_TOL = 1e-5
 
 
 def rel_frob(a, b):
@@ -68,7 +71,7 @@ def check_staged_stats(Ug, st_gpu, eps, out):
 
 
 def check_muon_step(W0, G, B_prev, W1_gpu, B_gpu, U_gpu, st_gpu, lr, mu, wd, eps=O.DELTA, nesterov=False,
-                    update_tol=UPDATE_TOL):
+                    update_tol=UPDATE_TOL, Ut_gpu=None):
     """All checks of one matrix after one GPU step under the Muon rule,
     Eq. (6): momentum end to end, statistics and params staged on the GPU's
     own U, and the applied update U against the oracle's."""
@@ -84,14 +87,21 @@ def check_muon_step(W0, G, B_prev, W1_gpu, B_gpu, U_gpu, st_gpu, lr, mu, wd, eps
     out["params_staged"] = max_rel(W1_gpu, O.moonlight_update(W0, Ug, lr, wd), floor_frac=1.0)
     assert out["params_staged"] <= PARAM_TOL, out
     applied = ((1.0 - lr * wd) * W0 - np.asarray(W1_gpu, np.float64)) / (lr * O.RHO * np.sqrt(max(m, n)))
+    if Ut_gpu is not None:
+        # meq_read_update reports sqrt(max(m, n)) U, the matrix Eq. (14) applied
+        out["readback"] = rel_frob(np.asarray(Ut_gpu, np.float64) / np.sqrt(max(m, n)), applied)
+        assert out["readback"] <= READBACK_TOL, out
+        applied = np.asarray(Ut_gpu, np.float64) / np.sqrt(max(m, n))
     out["update"] = rel_frob(applied, U_ora)
     assert out["update"] <= update_tol, out
     return out, W1_ora, B_ora
 
 
 def check_step(W0, G, B_prev, W1_gpu, B_gpu, U_gpu, st_gpu, lr, mu, wd, eps=O.DELTA, nesterov=False,
-               update_tol=UPDATE_TOL, report=None):
-    """All checks of one matrix after one GPU step. Returns a dict of errors."""
+               update_tol=UPDATE_TOL, report=None, Ut_gpu=None):
+    """All checks of one matrix after one GPU step. Returns a dict of errors.
+    Ut_gpu: the update meq_read_update reported; it must equal the one the
+    parameters received and is then the one compared with the oracle."""
     W0 = np.asarray(W0, np.float64)
     W1_ora, B_ora, info = O.hidden_step(W0, np.asarray(G, np.float64), np.asarray(B_prev, np.float64), lr, mu, wd,
                                         eps=eps, nesterov=nesterov)
@@ -110,7 +120,12 @@ def check_step(W0, G, B_prev, W1_gpu, B_gpu, U_gpu, st_gpu, lr, mu, wd, eps=O.DE
     out["params_staged"] = max_rel(W1_gpu, W1_staged, floor_frac=1.0)
     assert out["params_staged"] <= PARAM_TOL, out
     # final update vs the oracle (end to end), with the near-tie rule
-    Ut_gpu = gpu_update_from_params(W0, W1_gpu, lr, wd)
+    applied = gpu_update_from_params(W0, W1_gpu, lr, wd)
+    if Ut_gpu is None:
+        Ut_gpu = applied
+    else:
+        out["readback"] = rel_frob(Ut_gpu, applied)
+        assert out["readback"] <= READBACK_TOL, out
     ref = info["U_tilde"]
     out["flip"] = 0
     if st_gpu["direction"] != info["direction"]:

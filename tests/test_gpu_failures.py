@@ -159,5 +159,3 @@ def test_ns_gemm_stage_that_never_fills(meq):
 def test_debug_skip_load_validation(meq):
     with pytest.raises(meq.MeqError):
         meq.MeqMuon([(64, 64)], debug_skip_load=1, ns_cta_pair=0)
-    with pytest.raises(meq.MeqError):
-        meq.MeqMuon([(64, 64)], debug_skip_load=1, ns_single_launch=1)

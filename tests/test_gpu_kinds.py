@@ -45,7 +45,7 @@ def run_kinds(meq, wl, steps, pick=None, **opts):
             st = opt.read_stats(i)
             if kinds[i] == O.HIDDEN:
                 out, _, _, _ = PT.check_step(W0[i], G[i].double().numpy(), Bp[i], W1, B, opt.read_ns_output(i), st,
-                                             LR, MU, WD, EPS)
+                                             LR, MU, WD, EPS, Ut_gpu=opt.read_update(i))
                 err = out["update"]
             else:
                 Wn, Bo, Ut = O.param_step(kinds[i], W0[i], G[i].double().numpy(), Bp[i], LR, MU, WD, eps=EPS)
@@ -64,6 +64,8 @@ def run_kinds(meq, wl, steps, pick=None, **opts):
                 err = PT.max_rel(W1, Wn, floor_frac=1.0)
                 assert err <= PT.PARAM_TOL, (i, kinds[i], err)
                 assert PT.rel_frob(PT.gpu_update_from_params(W0[i], W1, LR, WD), Ut) <= 1e-5
+                # Eq. (12) / (13) as meq_read_update reports it
+                assert PT.rel_frob(opt.read_update(i), Ut) <= PT.READBACK_TOL
             worst[kinds[i]] = max(worst.get(kinds[i], 0.0), err)
             Bp[i] = B
     opt.close()

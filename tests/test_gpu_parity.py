@@ -46,7 +46,8 @@ def run_staged(meq, wl, steps, check_idx=None, report=None, update_tol=PT.UPDATE
             B = opt.read_momentum(i)
             PT.check_step(W0[i], Gs[i].double().numpy(), B_prev[i], params[i].cpu().numpy(), B,
                           opt.read_ns_output(i), opt.read_stats(i), LR, MU, WD, EPS,
-                          nesterov=bool(opts.get("nesterov", 0)), update_tol=update_tol, report=report)
+                          nesterov=bool(opts.get("nesterov", 0)), update_tol=update_tol, report=report,
+                          Ut_gpu=opt.read_update(i))
             B_prev[i] = B
     opt.close()
 

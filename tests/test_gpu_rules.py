@@ -46,7 +46,8 @@ def test_muon_rule_matches_oracle(meq, nesterov):
         for i in range(len(shapes)):
             B = opt.read_momentum(i)
             PT.check_muon_step(W0[i], Gs[i].double().numpy(), B_prev[i], params[i].cpu().numpy(), B,
-                               opt.read_ns_output(i), opt.read_stats(i), LR, MU, WD, EPS, nesterov=bool(nesterov))
+                               opt.read_ns_output(i), opt.read_stats(i), LR, MU, WD, EPS, nesterov=bool(nesterov),
+                               Ut_gpu=opt.read_update(i))
             B_prev[i] = B
             assert opt.read_direction_counts(i) == (0, 0)
     opt.close()
@@ -142,4 +143,53 @@ def test_ns_cv_trajectory_matches_oracle(meq):
             assert gc[20] < 0.1 * gc[0] and gc[20] < 0.2 * gr[20], (m, n, gr[[0, 20]], gc[[0, 20]])
         else:
             assert gr[20] < 0.1 * gr[0] and gc[20] < 0.1 * gc[0], (m, n, gr[[0, 20]], gc[[0, 20]])
+    torch.cuda.synchronize()
+
+
+def test_ns_cv_trajectory_threshold_applies_to_x0(meq):
+    """Section 3.1 replays Eq. (5) from X_0 = H / ||H||_F, and Eq. (8)
+    counts the rows and columns whose RMS exceeds delta: the threshold is on
+    X_0's RMS, not H's. H here has a large norm, one row at 3 delta and one
+    at delta / 10 in X_0, and one column at delta / 10 (still below delta
+    after one iteration, whose slope at zero is a = 3.4445); the oracle's
+    CVs (that row and column left out) must be reproduced, and reading the
+    threshold on H instead would be caught."""
+    import torch
+
+    rng = np.random.default_rng(3)
+    m, n = 64, 96
+    H = rng.standard_normal((m, n)) * 1e3 * np.exp(rng.uniform(-1, 1, (m, 1)))
+    H[5] = H[6] = 0.0
+    H[:, 7] = 0.0
+    nrm = np.sqrt((H * H).sum())
+    u = rng.standard_normal(n)
+    H[5] = u / np.linalg.norm(u) * 3e-7 * np.sqrt(n) * nrm
+    H[6] = u / np.linalg.norm(u) * 1e-8 * np.sqrt(n) * nrm
+    v = rng.standard_normal(m)
+    v[[5, 6]] = 0.0
+    H[:, 7] = v / np.linalg.norm(v) * 1e-8 * np.sqrt(m) * nrm
+    H = H.astype(np.float32).astype(np.float64)
+    orr, oc = O.ns_cv_trajectory(H, steps=1)
+    r_h, c_h = O.row_col_rms(H)
+    # the other reading differs well beyond the tolerance
+    assert abs(O.coefficient_of_variation(r_h) - orr[0]) > 1e-2 * orr[0]
+    assert abs(O.coefficient_of_variation(c_h) - oc[0]) > 1e-2 * oc[0]
+    gr, gc = meq.ns_cv_trajectory(torch.from_numpy(H.astype(np.float32)).cuda(), steps=1)
+    assert abs(gr[0] - orr[0]) <= 1e-4 * orr[0], (gr[0], orr[0])
+    assert abs(gc[0] - oc[0]) <= 1e-4 * oc[0], (gc[0], oc[0])
+    assert abs(gr[1] - orr[1]) <= 5e-3 + 2e-2 * orr[1] and abs(gc[1] - oc[1]) <= 5e-3 + 2e-2 * oc[1]
+
+
+def test_ns_cv_trajectory_large_matrix(meq):
+    """8192 x 8192 (beyond the allocation-free entry point's fixed scratch:
+    the replay has its own), k = 0 and 1 against the oracle."""
+    import torch
+
+    gen = torch.Generator().manual_seed(11)
+    m = n = 8192
+    H = torch.randn(m, n, generator=gen) * torch.exp(torch.empty(1, n).uniform_(-2.0, 2.0, generator=gen))
+    gr, gc = meq.ns_cv_trajectory(H.cuda(), steps=1)
+    orr, oc = O.ns_cv_trajectory(H.double().numpy(), steps=1)
+    assert abs(gr[0] - orr[0]) <= 1e-4 * max(orr[0], 1e-6) and abs(gc[0] - oc[0]) <= 1e-4 * oc[0], (gr, gc, orr, oc)
+    assert np.all(np.abs(gr - orr) <= 5e-3 + 2e-2 * orr) and np.all(np.abs(gc - oc) <= 5e-3 + 2e-2 * oc)
     torch.cuda.synchronize()

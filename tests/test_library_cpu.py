@@ -107,7 +107,7 @@ def test_host_validation_errors():
     p0, w0 = meq.state_bytes([(300, 200), (1, 64)], kinds=[meq.HIDDEN, meq.VECTOR])
     p1, w1 = meq.state_bytes([(300, 200), (1, 64)], kinds=[meq.HIDDEN, meq.VECTOR], debug_canaries=1)
     assert p1 == p0 and w1 > w0  # guard bands are workspace only
-    for field in ("ns_cta_pair", "ns_x0_fused", "update_rule", "debug_canaries", "ns_single_launch", "debug_skip_load"):
+    for field in ("ns_cta_pair", "ns_x0_fused", "update_rule", "debug_canaries", "debug_skip_load"):
         with pytest.raises(meq.MeqError):
             meq.state_bytes([(4, 4)], **{field: 2})
     # Eq. (6) is the hidden-weight baseline only
@@ -134,3 +134,27 @@ def test_binding_rejects_tensors_the_library_cannot_check(lib):
     with pytest.raises(ValueError):
         meq.row_col_stats_noalloc(H, torch.zeros(8), torch.zeros(8), torch.zeros(2, dtype=torch.float64),
                                   torch.zeros(1, dtype=torch.int32))
+
+
+def test_noalloc_size_checks_come_before_any_cuda_call():
+    """meq_row_col_stats_noalloc refuses bad arguments and shapes beyond its
+    fixed scratch on the host, with a message, before it looks for a device:
+    here, with no GPU at all, every refusal is MEQ_ERR_INVALID_ARG (a call
+    that got as far as the device would return MEQ_ERR_CUDA instead)."""
+    from paper_2609_35701_gb300 import meq
+
+    fn = meq.lib.meq_row_col_stats_noalloc
+    fake = 4096  # never dereferenced: the checks are host-only
+    cases = [
+        (fake, 8192, 8192, 1e-7, 1e-6, b"scratch"),          # 8192 + 256 * 8192 floats > 2^21
+        (fake, 1 << 20, 1 << 12, 1e-7, 1e-6, b"scratch"),
+        (fake, (1 << 20) + 1, 4, 1e-7, 1e-6, b"rows and cols"),
+        (fake, 0, 4, 1e-7, 1e-6, b"rows and cols"),
+        (None, 4, 4, 1e-7, 1e-6, b"NULL"),
+        (fake, 4, 4, -1.0, 1e-6, b"eps"),
+    ]
+    for U, m, n, eps, tie, text in cases:
+        assert fn(U, m, n, eps, tie, fake, fake, fake, fake, None) == 1, (m, n)
+        assert text in meq.lib.meq_last_error(None), (m, n, meq.lib.meq_last_error(None))
+    # the largest Llama-7B hidden shapes fit: 11008 + 344 * 4096 and 4096 + 128 * 11008 floats
+    assert 11008 + 344 * 4096 <= 1 << 21 and 4096 + 128 * 11008 <= 1 << 21
