@@ -294,8 +294,9 @@ meq_status meq_debug_wait_selftest(meq_state* st, float timeout_ms);
  *
  * It allocates nothing. Its scratch is a fixed 8 MiB __device__ array inside
  * the library, held by every GPU that loads the library until the process
- * exits. A matrix fits when rows + ceil(rows / 32) * cols <= 2,097,152 (e.g.
- * 4096 x 11008 and 11008 x 4096); larger ones, NULL pointers or
+ * exits. A matrix fits when rows * ceil(cols / 1024) + ceil(rows / 32) * cols
+ * <= 2,097,152 floats (e.g. 4096 x 11008 and 11008 x 4096, but not 8192 x
+ * 8192); larger ones, NULL pointers or
  * non-positive sizes return MEQ_ERR_INVALID_ARG before anything is enqueued
  * and before any CUDA call; meq_last_error(NULL) then says why.
  * The first call on a device looks up the array's device address (once per

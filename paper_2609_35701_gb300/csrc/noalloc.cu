@@ -10,8 +10,9 @@
 // file-scope __device__ array of fixed size that every GPU which loads the
 // library holds until the process exits.
 //
-// It sums squares over 32-row slabs, folds the column partials with one
-// thread per column (slabs in order), and forms the CVs in two passes, all in
+// It sums squares over blocks of 32 rows x 1024 columns, folds the partials
+// with one thread per row and per column (blocks in order), and forms the
+// CVs in two passes, all in
 // fp32 like the full step's statistics, so results agree with meq_read_stats
 // up to fp32 summation order. The same kernels, given scratch that the caller
 // allocated, give the first point of the CV trajectory (meq_ns_cv_trajectory).
@@ -24,13 +25,14 @@
 namespace {
 
 constexpr int kNaThreads = 256;
-constexpr int kNaSlab = 32;
+constexpr int kNaSlab = 32;        // rows per block
+constexpr int kNaChunk = 1024;     // columns per block (four per thread)
 constexpr int kNaFoldThreads = 256;
 constexpr int kNaFinThreads = 1024;
 constexpr int kMaxDevices = 64;
 
-// 8 MiB of scratch: row sums of squares (rows floats) followed by the column
-// partial sums (ceil(rows / 32) x cols floats).
+// 8 MiB of scratch: the row partial sums of squares (ceil(cols / 1024) x
+// rows floats) followed by the column partial sums (ceil(rows / 32) x cols).
 constexpr long long kScratchFloats = 2ll * 1024 * 1024;
 static __device__ __align__(256) float g_stats_scratch[kScratchFloats];
 
@@ -54,21 +56,24 @@ __device__ __forceinline__ float na_block_sum_f32(float v, float* sh) {
   return sh[0];
 }
 
-// One block per 32-row slab: column partial sums of squares for the slab and
-// the slab's row sums of squares.
+// One block per 32-row slab (blockIdx.x) and 1024-column chunk (blockIdx.y):
+// the slab's column partial sums of squares over the chunk's columns, and
+// the chunk's partial sums of squares of the slab's rows.
 __global__ void __launch_bounds__(kNaThreads) na_stats_kernel(const float* __restrict__ U, int64_t m, int64_t n,
                                                               float* __restrict__ scratch) {
   __shared__ float shr[kNaThreads / 32][32];
-  const int64_t slab = blockIdx.x;
+  const int64_t slab = blockIdx.x, chunk = blockIdx.y;
   const int64_t r0 = slab * kNaSlab;
   const int nr = static_cast<int>(m - r0 < kNaSlab ? m - r0 : kNaSlab);
+  const int64_t c1 = (chunk + 1) * kNaChunk < n ? (chunk + 1) * kNaChunk : n;
+  const int64_t nchunks = (n + kNaChunk - 1) / kNaChunk;
   const float* Us = U + r0 * n;
-  float* rowss = scratch;
-  float* cp = scratch + m + slab * n;
+  float* rowss = scratch + chunk * m;
+  float* cp = scratch + nchunks * m + slab * n;
   float racc[kNaSlab];
 #pragma unroll
   for (int r = 0; r < kNaSlab; ++r) racc[r] = 0.f;
-  for (int64_t c = threadIdx.x; c < n; c += kNaThreads) {
+  for (int64_t c = chunk * kNaChunk + threadIdx.x; c < c1; c += kNaThreads) {
     float cacc = 0.f;
 #pragma unroll
     for (int r = 0; r < kNaSlab; ++r) {
@@ -102,15 +107,21 @@ __global__ void __launch_bounds__(kNaThreads) na_stats_kernel(const float* __res
   }
 }
 
-// r (Eq. (7)) from the row sums of squares and c from the column partials,
-// one thread per row / column; each column sums its slabs in slab order.
-__global__ void __launch_bounds__(kNaFoldThreads) na_fold_kernel(int64_t m, int64_t n, const float* __restrict__ scratch,
+// r (Eq. (7)) from the row partials and c from the column partials, one
+// thread per row / column, each summing its partials in block order; the
+// row sums of squares are kept (first row of the scratch) for the CV kernel.
+__global__ void __launch_bounds__(kNaFoldThreads) na_fold_kernel(int64_t m, int64_t n, float* __restrict__ scratch,
                                                                  float* __restrict__ r, float* __restrict__ c) {
   const int64_t t = static_cast<int64_t>(blockIdx.x) * kNaFoldThreads + threadIdx.x;
   const int64_t nslabs = (m + kNaSlab - 1) / kNaSlab;
-  const float* rowss = scratch;
-  const float* cpart = scratch + m;
-  if (t < m) r[t] = sqrtf(rowss[t] * (1.0f / static_cast<float>(n)));
+  const int64_t nchunks = (n + kNaChunk - 1) / kNaChunk;
+  const float* cpart = scratch + nchunks * m;
+  if (t < m) {
+    float acc = 0.f;
+    for (int64_t k = 0; k < nchunks; ++k) acc += scratch[k * m + t];
+    scratch[t] = acc;  // only this thread reads or writes row t's partials
+    r[t] = sqrtf(acc * (1.0f / static_cast<float>(n)));
+  }
   if (t < n) {
     float acc = 0.f;
     int64_t k = 0;
@@ -174,9 +185,9 @@ __global__ void __launch_bounds__(kNaFinThreads) na_cv_kernel(int64_t m, int64_t
 
 // Plain launch (no attributes) that returns this launch's own status.
 template <typename... KArgs, typename... Args>
-cudaError_t launch_plain(void (*kernel)(KArgs...), unsigned grid, unsigned block, cudaStream_t st, Args&&... args) {
+cudaError_t launch_plain(void (*kernel)(KArgs...), dim3 grid, unsigned block, cudaStream_t st, Args&&... args) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
+  cfg.gridDim = grid;
   cfg.blockDim = dim3(block);
   cfg.stream = st;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
@@ -211,23 +222,25 @@ meq_status na_fail(meq_status s, const std::string& msg) {
 namespace meq {
 
 int64_t row_col_stats_scratch_floats(int64_t rows, int64_t cols) {
-  return rows + (rows + kNaSlab - 1) / kNaSlab * cols;
+  return (cols + kNaChunk - 1) / kNaChunk * rows + (rows + kNaSlab - 1) / kNaSlab * cols;
 }
 
 cudaError_t launch_row_col_stats(const float* U, int64_t rows, int64_t cols, float eps, float tie_atol, int frob,
                                  float* scratch, float* r, float* c, double* gammas, int* direction, cudaStream_t st,
                                  const char** failed) {
   const int64_t nslabs = (rows + kNaSlab - 1) / kNaSlab;
+  const int64_t nchunks = (cols + kNaChunk - 1) / kNaChunk;
   *failed = "statistics launch";
-  cudaError_t e = launch_plain(na_stats_kernel, static_cast<unsigned>(nslabs), kNaThreads, st, U, rows, cols, scratch);
+  cudaError_t e = launch_plain(na_stats_kernel, dim3(static_cast<unsigned>(nslabs), static_cast<unsigned>(nchunks)),
+                               kNaThreads, st, U, rows, cols, scratch);
   if (e != cudaSuccess) return e;
-  *failed = "column fold launch";
+  *failed = "fold launch";
   const int64_t len = rows > cols ? rows : cols;
-  e = launch_plain(na_fold_kernel, static_cast<unsigned>((len + kNaFoldThreads - 1) / kNaFoldThreads), kNaFoldThreads,
-                   st, rows, cols, static_cast<const float*>(scratch), r, c);
+  e = launch_plain(na_fold_kernel, dim3(static_cast<unsigned>((len + kNaFoldThreads - 1) / kNaFoldThreads)),
+                   kNaFoldThreads, st, rows, cols, scratch, r, c);
   if (e != cudaSuccess) return e;
   *failed = "CV launch";
-  return launch_plain(na_cv_kernel, 1u, kNaFinThreads, st, rows, cols, eps, tie_atol, frob,
+  return launch_plain(na_cv_kernel, dim3(1), kNaFinThreads, st, rows, cols, eps, tie_atol, frob,
                       static_cast<const float*>(scratch), r, c, gammas, direction);
 }
 

@@ -146,7 +146,7 @@ def test_noalloc_size_checks_come_before_any_cuda_call():
     fn = meq.lib.meq_row_col_stats_noalloc
     fake = 4096  # never dereferenced: the checks are host-only
     cases = [
-        (fake, 8192, 8192, 1e-7, 1e-6, b"scratch"),          # 8192 + 256 * 8192 floats > 2^21
+        (fake, 8192, 8192, 1e-7, 1e-6, b"scratch"),          # 8192 * 8 + 256 * 8192 floats > 2^21
         (fake, 1 << 20, 1 << 12, 1e-7, 1e-6, b"scratch"),
         (fake, (1 << 20) + 1, 4, 1e-7, 1e-6, b"rows and cols"),
         (fake, 0, 4, 1e-7, 1e-6, b"rows and cols"),
@@ -156,5 +156,5 @@ def test_noalloc_size_checks_come_before_any_cuda_call():
     for U, m, n, eps, tie, text in cases:
         assert fn(U, m, n, eps, tie, fake, fake, fake, fake, None) == 1, (m, n)
         assert text in meq.lib.meq_last_error(None), (m, n, meq.lib.meq_last_error(None))
-    # the largest Llama-7B hidden shapes fit: 11008 + 344 * 4096 and 4096 + 128 * 11008 floats
-    assert 11008 + 344 * 4096 <= 1 << 21 and 4096 + 128 * 11008 <= 1 << 21
+    # the largest Llama-7B hidden shapes fit: 11008 * 4 + 344 * 4096 and 4096 * 11 + 128 * 11008 floats
+    assert 11008 * 4 + 344 * 4096 <= 1 << 21 and 4096 * 11 + 128 * 11008 <= 1 << 21

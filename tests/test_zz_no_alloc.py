@@ -110,7 +110,7 @@ def test_noalloc_llama7b_shapes_and_size_limit():
         print(f"noalloc stats {m}x{n}: {e0.elapsed_time(e1) / reps * 1e3:.1f} us per call")
         _check_against_oracle(U_h.double().numpy(), r, c, g, d, (m, n))
         del U
-    # 8192 x 8192 needs 8192 + 256 * 8192 floats of scratch, above 2^21
+    # 8192 x 8192 needs 8192 * 8 + 256 * 8192 floats of scratch, above 2^21
     m = n = 8192
     U = torch.zeros(m, n, dtype=torch.float32, device="cuda")
     r, c, g, d = _outputs(torch, m, n)
