@@ -40,7 +40,8 @@ CPU_BASELINE_BUDGET_S = 20.0 # wall-clock budget of the oracle sample beside the
 SUSTAINED_NS_MS = 20.0       # an NS phase this long per step runs under the power cap: sustained peak
 DEFAULT_STEPS = {"llama7b": 20, "llama1b": 50}
 METRIC = "MeqMuon step ms per model; NS TFLOP/s & equilibration GB/s as % of GB300 peak"
-COPY_CHUNK = 8 << 20          # elements (32 MB) per host <-> device copy of the end-to-end loop
+COPY_CHUNK = 8 << 20          # smallest piece (elements, 32 MB) of a host <-> device copy in the end-to-end loop
+COPY_PIECES = 64              # at most this many pieces per direction per step
 
 
 def source_fingerprint(path):
@@ -470,24 +471,23 @@ def main():
         hg = [h, h]
         hp = torch.empty(pbuf.numel(), dtype=torch.float32, pin_memory=True)
         n_e2e = max(3, min(args.steps, 50))
-        # Copies move in pieces of COPY_CHUNK elements on two copy streams,
-        # so that the two directions share the host link: the gradients of step k go up
-        # while step k - 1 runs; the parameters of step k - 1 come back while
-        # step k's momentum, Newton-Schulz and statistics run
-        # (meq_step_prepare), and step k's update (meq_step_apply) waits for
-        # that copy before it writes the parameters in place.
-        pieces = [(lo, min(lo + COPY_CHUNK, pbuf.numel())) for lo in range(0, pbuf.numel(), COPY_CHUNK)]
+        # Copies move in pieces on two copy streams, so that the two
+        # directions share the host link: the gradients of step k + 1 go up
+        # while step k runs (enqueued right after step k's prepare); the
+        # parameters of step k - 1 come back while step k's momentum,
+        # Newton-Schulz and statistics run (meq_step_prepare), and step k's
+        # update (meq_step_apply) waits for that copy before it writes the
+        # parameters in place. At most COPY_PIECES pieces per direction keep
+        # the host from blocking on a full queue of pending copies.
+        chunk = max(COPY_CHUNK, -(-pbuf.numel() // COPY_PIECES))
+        pieces = [(lo, min(lo + chunk, pbuf.numel())) for lo in range(0, pbuf.numel(), chunk)]
         up, down = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
         ev_in = [torch.cuda.Event() for _ in range(2)]
         ev_prep = [torch.cuda.Event() for _ in range(2)]
         ev_step = torch.cuda.Event()
         ev_out = torch.cuda.Event()
-        torch.cuda.synchronize()
-        a0 = torch.cuda.Event(enable_timing=True)
-        a1 = torch.cuda.Event(enable_timing=True)
-        a0.record(stream)
-        up.wait_event(a0)
-        for k in range(n_e2e):
+
+        def upload(k):
             b = k % 2
             with torch.cuda.stream(up):
                 if k >= 2:
@@ -495,9 +495,20 @@ def main():
                 for lo, hi in pieces:
                     gbufs[b][0][lo:hi].copy_(hg[b][lo:hi], non_blocking=True)
                 ev_in[b].record(up)
+
+        torch.cuda.synchronize()
+        a0 = torch.cuda.Event(enable_timing=True)
+        a1 = torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        up.wait_event(a0)
+        upload(0)
+        for k in range(n_e2e):
+            b = k % 2
             stream.wait_event(ev_in[b])
             opt.step_prepare(grads[b], LR, MU, WD, EPS)
             ev_prep[b].record(stream)
+            if k + 1 < n_e2e:
+                upload(k + 1)
             if k >= 1:
                 stream.wait_event(ev_out)        # parameters of step k - 1 are back on the host
             opt.step_apply(params)
