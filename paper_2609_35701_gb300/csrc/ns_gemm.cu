@@ -29,11 +29,18 @@
 //               every other 32-column chunk (two warps per lane quarter, so
 //               each SM sub-partition can hide one warp's latencies behind
 //               the other's work)
+//   warp 10 : tile scheduler (one thread, leader CTA)
 // Tiles are handed out dynamically: each unit (CTA or CTA pair) starts on
-// its own index and then draws from an atomic counter, and the leader's
-// producer passes every index to the other roles through a ring in shared
-// memory, so a launch ends within about one tile on every unit whatever the
-// mix of tile sizes and SM speeds.
+// its own index and then draws from an atomic counter, so a launch ends
+// within about one tile on every unit whatever the mix of tile sizes and SM
+// speeds. The leader's scheduler thread claims each index one tile ahead of
+// the producer, decodes it (group, matrix, tile row and column, k-block
+// count) and passes the decoded entry to every role of both CTAs through a
+// ring in shared memory. The producer and the MMA issuer run ahead of the
+// tensor pipe by only a few k-blocks, so neither can afford the decode, a
+// dependent integer chain of one thread: measured at 0.35-0.6 us per tile,
+// it left the tensor pipe idle for about 0.5 us between tiles when they did
+// it themselves.
 // Two 128x256 fp32 accumulators (512 TMEM columns) let the epilogue of one
 // tile overlap the MMAs of the next. The epilogue stages 32 x 32 blocks in
 // swizzled shared memory; the symmetric A and P (each block stored twice)
@@ -52,10 +59,11 @@ namespace {
 constexpr int BM = 128, BN = 256, BK = 64, UK = 16;  // per-CTA rows, tile columns, k-block, MMA K
 constexpr int A_BYTES = BM * BK * 2;                 // 16 KB
 constexpr int NUM_EPI_WARPS = kNsEpilogueWarps;      // two per TMEM lane quarter
-constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
+constexpr int SCHED_WARP = 2 + NUM_EPI_WARPS;
+constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS + 32;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int SLOT_BYTES = 2048;                     // one 32 x 32 16-bit block (two per epilogue warp)
-constexpr int SCHED_D = 16;                          // entries of the tile-index ring
+constexpr int SCHED_D = 16;                          // entries of the tile ring (16 bytes each)
 constexpr float kUInvScale2 = 1.0f / (kUScale * kUScale);  // exact: kUScale is a power of two
 
 // kPair = 1: one CTA computes a 128 x 256 tile (tcgen05 cta_group::1).
@@ -70,12 +78,14 @@ struct Cfg {
   static constexpr int B_BYTES = BN_LOCAL * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int STAGES = kPair == 1 ? 4 : 6;
-  // full, empty, tmem full x2, tmem empty x2, drain, tile ring full / empty
-  static constexpr int NUM_BARS = 2 * STAGES + 4 + 1 + 2 * SCHED_D;
+  // full, empty, tmem full x2, tmem empty x2, drain, tile ring full / empty,
+  // entry taken by the producer
+  static constexpr int NUM_BARS = 2 * STAGES + 4 + 1 + 2 * SCHED_D + 1;
   static constexpr int SMEM_EPI_OFF = STAGES * STAGE_BYTES;
   static constexpr int SMEM_BAR_OFF = SMEM_EPI_OFF + NUM_EPI_WARPS * 2 * SLOT_BYTES;
   // barriers, the TMEM address word (16 bytes reserved), the tile ring
-  static constexpr int SMEM_BYTES = SMEM_BAR_OFF + NUM_BARS * 8 + 16 + 4 * SCHED_D + 1024;
+  // (16-byte aligned), alignment slack of the dynamic shared memory
+  static constexpr int SMEM_BYTES = SMEM_BAR_OFF + NUM_BARS * 8 + 16 + 15 + 16 * SCHED_D + 1024;
   static_assert(SMEM_BYTES <= 232448, "shared memory budget of one sm_103a CTA");
 };
 
@@ -196,27 +206,31 @@ __device__ __forceinline__ void cluster_sync_all() {
 __device__ __forceinline__ void mbar_arrive_relaxed_cluster(uint32_t bar_cluster) {
   asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
-// Writes a 32-bit value into the peer CTA's shared memory and completes it
-// as a 4-byte transaction on the peer's barrier, which this call also arms
-// (one arrival). A waiter on that barrier then sees the value, as after a TMA
-// load; no fence of the writer's other memory operations is involved.
-__device__ __forceinline__ void st_async_peer_u32(uint32_t addr_cluster, uint32_t bar_cluster, uint32_t v) {
-  asm volatile("mbarrier.arrive.expect_tx.relaxed.cluster.shared::cluster.b64 _, [%0], 4;" ::"r"(bar_cluster)
+// Writes a 16-byte tile-ring entry into the peer CTA's shared memory and
+// completes it as a 16-byte transaction on the peer's barrier, which this
+// call also arms (one arrival). A waiter on that barrier then sees the value,
+// as after a TMA load; no fence of the writer's other memory operations is
+// involved.
+__device__ __forceinline__ void st_async_peer_v4(uint32_t addr_cluster, uint32_t bar_cluster, uint4 v) {
+  asm volatile("mbarrier.arrive.expect_tx.relaxed.cluster.shared::cluster.b64 _, [%0], 16;" ::"r"(bar_cluster)
                : "memory");
-  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.u32 [%0], %1, [%2];" ::"r"(addr_cluster), "r"(v),
-               "r"(bar_cluster)
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+                   addr_cluster),
+               "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "r"(bar_cluster)
                : "memory");
+}
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint4 v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr)
+               : "memory");
+  return v;
 }
 __device__ __forceinline__ void mbar_arrive_local(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ void st_shared_u32(uint32_t addr, uint32_t v) {
-  asm volatile("st.shared.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
-}
-__device__ __forceinline__ uint32_t ld_shared_u32(uint32_t addr) {
-  uint32_t v;
-  asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
-  return v;
 }
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* tm) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
@@ -332,6 +346,18 @@ __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
   return c;
 }
 
+// A decoded tile as the scheduler publishes it: x = tile index, y = matrix,
+// z = group | tm << 4 | tn << 18, w = k-blocks | (diagonal tile whose B half
+// is its A half) << 16.
+__device__ __forceinline__ TileCoord entry_coord(uint4 e) {
+  TileCoord c;
+  c.g = static_cast<int>(e.z & 15u);
+  c.mat = static_cast<int>(e.y);
+  c.tm = static_cast<int>((e.z >> 4) & 0x3FFFu);
+  c.tn = static_cast<int>(e.z >> 18);
+  return c;
+}
+
 __device__ __forceinline__ uint32_t pack_half2(float a, float b, int fp16) {
   if (fp16) {
     __half2 h = __floats2half2_rn(a, b);
@@ -443,7 +469,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
 #define TEMPTY_BAR(a) (bar0 + 8u * (2 * STAGES + 2 + (a)))
 #define SFULL_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + (i)))
 #define SEMPTY_BAR(i) (bar0 + 8u * (2 * STAGES + 5 + SCHED_D + (i)))
-  const uint32_t ring = tmem_slot + 16;  // SCHED_D tile indices
+#define PTAKEN_BAR (bar0 + 8u * (2 * STAGES + 5 + 2 * SCHED_D))
+  const uint32_t ring = (tmem_slot + 16u + 15u) & ~15u;  // SCHED_D entries of 16 bytes
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -467,10 +494,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     mbar_init(drain_bar, 1);
     for (int i = 0; i < SCHED_D; ++i) {
       mbar_init(SFULL_BAR(i), 1);
-      // consumers of each index: the MMA issuer and the epilogue warps of the
-      // leader, and (pair) the peer's producer and epilogue warps
-      mbar_init(SEMPTY_BAR(i), kPair * (1 + NUM_EPI_WARPS));
+      // consumers of each entry: the producer and epilogue warps of each
+      // CTA, and the leader's MMA issuer
+      mbar_init(SEMPTY_BAR(i), 1 + kPair * (1 + NUM_EPI_WARPS));
     }
+    mbar_init(PTAKEN_BAR, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     for (int g = 0; g < p.ngroups; ++g) {
       prefetch_tmap(&p.g[g].tmA);
@@ -501,29 +529,29 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
   // Each unit (CTA pair) starts on tile `unit`; further tiles are handed out
   // by the launch's atomic counter, so units that finish early take more and
   // the launch ends within about one tile on every unit. The leader's
-  // producer fetches each index and publishes it in the tile ring of both
-  // CTAs (the peer's copy by st.async, which completes on the peer's barrier
-  // like a TMA load, so the producer never waits on a memory fence); every
-  // other role reads the ring in the same order. A reader hands its slot
-  // back with a relaxed arrive (a release would first wait for the
-  // epilogue's outstanding global stores). Its read has completed long
-  // before the slot can be written again: the producer writes index n + 16
-  // only after loading tile n + 15, by which time every role has used index
-  // n (the epilogue warps to release tile n's accumulator, the peer's
-  // producer to load its half of tile n) -- the operand ring holds at most
-  // 6 k-blocks and the accumulators 2 tiles.
-  auto sched_put = [&](int n, int t) -> bool {
+  // scheduler claims entry n + 1 once the producer has taken entry n (the
+  // claim stays one tile ahead, as the load balance needs), decodes it and
+  // publishes it in the tile ring of both CTAs (the peer's copy by st.async,
+  // which completes on the peer's barrier like a TMA load, so no memory
+  // fence is waited on); every other role reads the ring in the same order.
+  // A reader hands its slot back with a relaxed arrive (a release would
+  // first wait for the epilogue's outstanding global stores). Its read has
+  // completed long before the slot can be written again: entry n + 16 is
+  // written after the producer took entry n + 15, by which time every role
+  // has used entry n -- the operand ring holds at most 6 k-blocks and the
+  // accumulators 2 tiles.
+  auto sched_put = [&](int n, uint4 e) -> bool {
     const int i = n & (SCHED_D - 1);
     if (!wait_bounded(SEMPTY_BAR(i), ((n / SCHED_D) & 1) ^ 1u, err, DEV_TIMEOUT_SCHED_PUT, tmo)) return false;
-    if (kPair == 2) st_async_peer_u32(map_to_rank(ring + 4u * i, 1), map_to_rank(SFULL_BAR(i), 1), static_cast<uint32_t>(t));
-    st_shared_u32(ring + 4u * i, static_cast<uint32_t>(t));
+    if (kPair == 2) st_async_peer_v4(map_to_rank(ring + 16u * i, 1), map_to_rank(SFULL_BAR(i), 1), e);
+    st_shared_v4(ring + 16u * i, e);
     mbar_arrive_local(SFULL_BAR(i));  // release (CTA scope) of the store above
     return true;
   };
-  auto sched_take = [&](int n, int& t) -> bool {
+  auto sched_take = [&](int n, uint4& e) -> bool {
     const int i = n & (SCHED_D - 1);
     if (!wait_bounded(SFULL_BAR(i), (n / SCHED_D) & 1, err, DEV_TIMEOUT_SCHED_TAKE, tmo)) return false;
-    t = static_cast<int>(ld_shared_u32(ring + 4u * i));
+    e = ld_shared_v4(ring + 16u * i);
     mbar_arrive_relaxed_cluster((kPair == 2 && !leader) ? map_to_rank(SEMPTY_BAR(i), 0) : SEMPTY_BAR(i));
     return true;
   };
@@ -535,18 +563,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       uint32_t phase = 0;
       uint32_t issued_mask = 0, issued_parity = 0;  // bit s: stage s was filled / parity of its last fill
       bool ok = true;
-      int t = unit;
-      int fetched = 0;  // leader: the counter value for the next tile
       for (int n = 0; ok; ++n) {
-        if (n > 0 && leader) t = nunits + fetched;
-        if (leader ? !sched_put(n, t) : !sched_take(n, t)) break;
-        if (t >= p.total_tiles) break;
-        const TileCoord c = decode_tile<kPair>(p, t);
+        uint4 e;
+        if (!sched_take(n, e)) break;
+        if (leader) mbar_arrive_local(PTAKEN_BAR);  // the scheduler may claim the next tile
+        if (static_cast<int>(e.x) >= p.total_tiles) break;
+        const TileCoord c = entry_coord(e);
         const GemmGroup& G = p.g[c.g];
-        // The next index is fetched while this tile's operands are requested;
-        // its value is first read at the top of the next iteration.
-        if (leader) fetched = atomicAdd(p.sched, 1);
-        const int nk = (G.K + BK - 1) / BK;
+        const int nk = static_cast<int>(e.w & 0xFFFFu);
         // Mode, descriptor and B layout are per launch: reading them at a
         // fixed index keeps them launch-uniform for the compiler (measured:
         // 2% of the step).
@@ -556,7 +580,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
         // A diagonal tile of a symmetric product (X X^T, A A) has each CTA's
         // B half equal to its A half (same rows of the same buffer, same box):
         // only A is loaded, and the MMA reads it as B too.
-        const bool b_is_a = kPair == 2 && G.sym && !b_mn_major && arow == bcol;
+        const bool b_is_a = (e.w >> 16) & 1u;
         for (int kb = 0; kb < nk; ++kb) {
           if (!wait_bounded(EMPTY_BAR(stage), phase ^ 1u, err, DEV_TIMEOUT_PRODUCER, tmo)) {
             ok = false;
@@ -620,16 +644,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       uint32_t acc_phase = 0;
       bool ok = true;
       for (int n = 0; ok; ++n) {
-        int t = 0;
-        if (!sched_take(n, t) || t >= p.total_tiles) break;
-        const TileCoord c = decode_tile<kPair>(p, t);
-        const GemmGroup& G = p.g[c.g];
-        const int nk = (G.K + BK - 1) / BK;
+        uint4 e;
+        if (!sched_take(n, e) || static_cast<int>(e.x) >= p.total_tiles) break;
+        const int nk = static_cast<int>(e.w & 0xFFFFu);
         const int b_mn_major = p.g[0].b_mn_major;
         const uint32_t idesc = p.g[0].idesc;
         const uint32_t b_lbo = b_mn_major ? (64u * BK * 2u) : 16u;
         // diagonal tile of a symmetric product: B is read from the A half (the producer loads A only)
-        const bool b_is_a = kPair == 2 && G.sym && !b_mn_major && c.tm * TILE_M == c.tn * BN;
+        const bool b_is_a = (e.w >> 16) & 1u;
         if (!wait_bounded(TEMPTY_BAR(acc), acc_phase ^ 1u, err, DEV_TIMEOUT_MMA_TMEM, tmo)) break;
         tc_fence_after();
         const uint32_t d = tmem_base + static_cast<uint32_t>(acc * BN);
@@ -691,12 +713,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     const uint32_t tempty_target0 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(0), 0) : TEMPTY_BAR(0);
     const uint32_t tempty_target1 = (kPair == 2 && !leader) ? map_to_rank(TEMPTY_BAR(1), 0) : TEMPTY_BAR(1);
     for (int n = 0;; ++n) {
-      int t = 0, got = 1;
-      if (lane == 0) got = sched_take(n, t) ? 1 : 0;
+      uint4 e = make_uint4(0u, 0u, 0u, 0u);
+      int got = 1;
+      if (lane == 0) got = sched_take(n, e) ? 1 : 0;
       got = __shfl_sync(0xffffffffu, got, 0);
-      t = __shfl_sync(0xffffffffu, t, 0);
-      if (!got || t >= p.total_tiles) break;
-      const TileCoord c = decode_tile<kPair>(p, t);
+      e.x = __shfl_sync(0xffffffffu, e.x, 0);
+      e.y = __shfl_sync(0xffffffffu, e.y, 0);
+      e.z = __shfl_sync(0xffffffffu, e.z, 0);
+      if (!got || static_cast<int>(e.x) >= p.total_tiles) break;
+      const TileCoord c = entry_coord(e);
       const GemmGroup& G = p.g[c.g];
       const int mode = p.g[0].mode;  // one mode per launch (a launch-uniform read)
       if (!wait_bounded_warp(TFULL_BAR(acc), acc_phase, err, DEV_TIMEOUT_EPI, tmo)) break;
@@ -857,6 +882,33 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     // The outputs are in global memory before the CTA leaves.
     if (lane == 0) bulk_wait_all();
     __syncwarp();
+  } else if (warp == SCHED_WARP) {
+    if (lane == 0 && leader) {
+      // ---------------------------------------------------------------- tile scheduler
+      int t = unit;
+      int fetched = 0;  // the counter value for the next tile
+      for (int n = 0;; ++n) {
+        if (n > 0) {
+          // the producer has taken entry n - 1 (its phase n - 1 is complete)
+          if (!wait_bounded(PTAKEN_BAR, static_cast<uint32_t>(n - 1) & 1u, err, DEV_TIMEOUT_SCHED_PUT, tmo)) break;
+          t = nunits + fetched;
+        }
+        uint4 e = make_uint4(static_cast<uint32_t>(t), 0u, 0u, 0u);
+        if (t < p.total_tiles) {
+          const TileCoord c = decode_tile<kPair>(p, t);
+          const GemmGroup& G = p.g[c.g];
+          const int nk = (G.K + BK - 1) / BK;
+          const bool b_is_a = kPair == 2 && G.sym && !p.g[0].b_mn_major && c.tm * TILE_M == c.tn * BN;
+          e.y = static_cast<uint32_t>(c.mat);
+          e.z = static_cast<uint32_t>(c.g) | (static_cast<uint32_t>(c.tm) << 4) | (static_cast<uint32_t>(c.tn) << 18);
+          e.w = static_cast<uint32_t>(nk) | (b_is_a ? 0x10000u : 0u);
+        }
+        if (!sched_put(n, e)) break;
+        if (t >= p.total_tiles) break;
+        fetched = atomicAdd(p.sched, 1);  // read when the producer has taken this entry
+      }
+    }
+    __syncwarp();
   }
 #undef FULL_BAR
 #undef EMPTY_BAR
@@ -864,6 +916,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
 #undef TEMPTY_BAR
 #undef SFULL_BAR
 #undef SEMPTY_BAR
+#undef PTAKEN_BAR
 
   if (kPair == 2 && *reinterpret_cast<volatile int*>(err) != 0) {
     // After an early exit, give copies still in flight towards either CTA
