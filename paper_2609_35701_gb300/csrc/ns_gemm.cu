@@ -299,16 +299,22 @@ __device__ __forceinline__ void tmem_ld_32cols(uint32_t taddr, float* v) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+constexpr int kBand = 8;  // tile rows per band of the dense products' tile order
+
 struct TileCoord {
   int g, mat, tm, tn;
 };
 
 // Tiles of a group are numbered matrix by matrix (walked backwards when
 // p.reverse is set, so a launch starts on the matrices its predecessor wrote
-// last, which are still in L2). Dense outputs run tm-major
-// over tiles_m x tiles_n; symmetric outputs (Gram, polynomial) run tn-major
-// over the tiles with tm * TILE_M < (tn + 1) * 256, i.e. those holding a
-// 32 x 32 block on or above the diagonal.
+// last, which are still in L2). Dense outputs (X' = P X) with more than
+// kBand tile rows run in bands of kBand tile rows, each band column by column: the tiles in flight at once
+// (one per CTA pair) then share a few row panels of P and column panels of
+// X, where a row-by-row walk re-read every column panel of a wide X once per
+// tile row (measured at 4096 x 11008: 4.5 times the launch's algorithmic
+// bytes from DRAM). Symmetric outputs (Gram, polynomial) run tn-major over
+// the tiles with tm * TILE_M < (tn + 1) * 256, i.e. those holding a 32 x 32
+// block on or above the diagonal.
 __device__ __forceinline__ int find_segment(const GemmParams& p, int t) {
   int lo = 0, hi = p.ngroups - 1;  // the last segment whose tile_begin <= t
   while (lo < hi) {
@@ -329,9 +335,15 @@ __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
   TileCoord c;
   c.g = g;
   c.mat = mat;
-  if (!G.sym) {
+  if (!G.sym && G.tiles_m <= kBand) {
     c.tm = r / G.tiles_n;
     c.tn = r - c.tm * G.tiles_n;
+  } else if (!G.sym) {
+    const int band = r / (kBand * G.tiles_n);
+    const int in = r - band * kBand * G.tiles_n;
+    const int rows = min(kBand, G.tiles_m - band * kBand);
+    c.tm = band * kBand + in % rows;
+    c.tn = in / rows;
   } else {
     int tn = 0;
     for (;;) {
