@@ -259,8 +259,11 @@ int meq_kernels_per_step(const meq_state* st);
 int meq_ns_gemm_launches_per_step(const meq_state* st);
 
 /* Per-phase timing with CUDA events on the launch stream. While enabled,
- * meq_step launches its kernels directly (not from the CUDA graph) and
- * records an event between phases. meq_read_profile synchronises and returns
+ * meq_step runs the same kernels with an event recorded between phases:
+ * with use_graph, by replaying a second graph that holds event-record nodes
+ * between the phases, then waiting for the stream and adding up that step's
+ * phase times (so profiled steps are not pipelined with the host); without
+ * use_graph, by launching directly. meq_read_profile synchronises and returns
  * the summed milliseconds of each phase since profiling was enabled:
  *   phase_ms[0] momentum update + norms (all kinds), [1] X_0 cast,
  *   [2] all NS GEMMs, [3] statistics + direction / scales, [4] apply;

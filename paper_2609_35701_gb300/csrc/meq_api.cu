@@ -137,7 +137,14 @@ struct meq_state {
   cudaStream_t last_stream = nullptr;
   int kernels_per_step = 0;
   bool profiling = false;
-  std::vector<std::vector<cudaEvent_t>> prof_events;  // 6 events per profiled step
+  std::vector<std::vector<cudaEvent_t>> prof_events;  // eager launches: 6 events per profiled step
+  // graph replay: one graph with event-record nodes between the phases, its
+  // 6 events, and the summed phase times of the replays read so far
+  cudaGraph_t graph_prof = nullptr;
+  cudaGraphExec_t gexec_prof = nullptr;
+  std::vector<cudaEvent_t> prof_graph_events;
+  double prof_sum[5] = {0, 0, 0, 0, 0};
+  int64_t prof_graph_steps = 0;
   std::string last_error;
   int64_t persistent_bytes = 0;
   std::vector<std::pair<int64_t, int64_t>> guard_ranges;  // arena guard bands (debug_canaries)
@@ -719,6 +726,14 @@ static void drop_profile(meq_state* st) {
   for (auto& v : st->prof_events)
     for (auto x : v) cudaEventDestroy(x);
   st->prof_events.clear();
+  if (st->gexec_prof) cudaGraphExecDestroy(st->gexec_prof);
+  if (st->graph_prof) cudaGraphDestroy(st->graph_prof);
+  st->gexec_prof = nullptr;
+  st->graph_prof = nullptr;
+  for (auto x : st->prof_graph_events) cudaEventDestroy(x);
+  st->prof_graph_events.clear();
+  for (double& x : st->prof_sum) x = 0;
+  st->prof_graph_steps = 0;
 }
 
 // One open NVTX range at a time (closed on the next stage and on scope exit).
@@ -738,7 +753,8 @@ struct NvtxRange {
 
 enum StepParts : int { PART_PREPARE = 1, PART_APPLY = 2, PART_ALL = 3 };
 
-static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev = nullptr, int parts = PART_ALL) {
+static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev = nullptr, int parts = PART_ALL,
+                                  bool capturing = false) {
   const LaunchCtx& C = st->ctx;
   // NVTX ranges name the stages on the host timeline (each eager enqueue, or
   // the capture of the graph); CUDA events time them on the stream.
@@ -746,7 +762,9 @@ static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev
   static const char* const kStage[5] = {"momentum", "cast_x0", "ns_gemm", "statistics", "apply"};
   NvtxStages stage;
   auto mark = [&](int i) {
-    if (ev) cudaEventRecord(ev[i], s);
+    // under stream capture, only an external record becomes a node that
+    // records the event on each replay (a plain one just orders the capture)
+    if (ev) cudaEventRecordWithFlags(ev[i], s, capturing ? cudaEventRecordExternal : cudaEventRecordDefault);
     stage.next(i < 5 ? kStage[i] : nullptr);
   };
   cudaError_t e = cudaSuccess;
@@ -794,7 +812,8 @@ static meq_status enqueue_kernels(meq_state* st, cudaStream_t s, cudaEvent_t* ev
   return MEQ_OK;
 }
 
-static meq_status capture_graph(meq_state* st, int parts, cudaGraph_t* graph, cudaGraphExec_t* gexec) {
+static meq_status capture_graph(meq_state* st, int parts, cudaGraph_t* graph, cudaGraphExec_t* gexec,
+                                cudaEvent_t* ev = nullptr) {
   cudaStream_t cs = nullptr;
   cudaError_t e = cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking);
   if (e != cudaSuccess) return cuda_fail(st, e, "cudaStreamCreate");
@@ -803,7 +822,7 @@ static meq_status capture_graph(meq_state* st, int parts, cudaGraph_t* graph, cu
     cudaStreamDestroy(cs);
     return cuda_fail(st, e, "cudaStreamBeginCapture");
   }
-  meq_status ms = enqueue_kernels(st, cs, nullptr, parts);
+  meq_status ms = enqueue_kernels(st, cs, ev, parts, true);
   cudaGraph_t g = nullptr;
   e = cudaStreamEndCapture(cs, &g);
   cudaStreamDestroy(cs);
@@ -890,6 +909,29 @@ meq_status meq_step(float* const* params, const float* const* grads, meq_state* 
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   meq_status ms = upload_step(st, params, grads, shapes, n, lr, momentum, weight_decay, eps, s);
   if (ms != MEQ_OK) return ms;
+  if (st->profiling && st->opt.use_graph) {
+    // the step's own graph, with an event-record node between its phases;
+    // each replay is waited for and its phase times added up
+    if (!st->gexec_prof) {
+      st->prof_graph_events.assign(6, nullptr);
+      for (auto& x : st->prof_graph_events) {
+        cudaError_t e = cudaEventCreate(&x);
+        if (e != cudaSuccess) return cuda_fail(st, e, "cudaEventCreate");
+      }
+      meq_status cs = capture_graph(st, PART_ALL, &st->graph_prof, &st->gexec_prof, st->prof_graph_events.data());
+      if (cs != MEQ_OK) return cs;
+    }
+    cudaError_t e = cudaGraphLaunch(st->gexec_prof, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    for (int p = 0; e == cudaSuccess && p < 5; ++p) {
+      float ms = 0.f;
+      e = cudaEventElapsedTime(&ms, st->prof_graph_events[p], st->prof_graph_events[p + 1]);
+      st->prof_sum[p] += ms;
+    }
+    if (e != cudaSuccess) return cuda_fail(st, e, "profiled graph replay");
+    ++st->prof_graph_steps;
+    return MEQ_OK;
+  }
   if (st->profiling) {
     std::vector<cudaEvent_t> ev(6, nullptr);
     for (auto& x : ev) {
@@ -1191,6 +1233,7 @@ meq_status meq_read_profile(meq_state* st, double* phase_ms, int64_t* steps) {
   cudaError_t e = cudaStreamSynchronize(st->last_stream);
   if (e != cudaSuccess) return cuda_fail(st, e, "cudaStreamSynchronize");
   double acc[5] = {0, 0, 0, 0, 0};
+  for (int p = 0; p < 5; ++p) acc[p] = st->prof_sum[p];
   for (auto& v : st->prof_events)
     for (int p = 0; p < 5; ++p) {
       float ms = 0.f;
@@ -1200,7 +1243,7 @@ meq_status meq_read_profile(meq_state* st, double* phase_ms, int64_t* steps) {
     }
   if (phase_ms)
     for (int p = 0; p < 5; ++p) phase_ms[p] = acc[p];
-  if (steps) *steps = static_cast<int64_t>(st->prof_events.size());
+  if (steps) *steps = static_cast<int64_t>(st->prof_events.size()) + st->prof_graph_steps;
   return MEQ_OK;
 }
 

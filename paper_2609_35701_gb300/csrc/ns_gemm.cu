@@ -736,8 +736,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
       const TileCoord c = entry_coord(e);
       const GemmGroup& G = p.g[c.g];
       const int mode = p.g[0].mode;  // one mode per launch (a launch-uniform read)
-      if (!wait_bounded_warp(TFULL_BAR(acc), acc_phase, err, DEV_TIMEOUT_EPI, tmo)) break;
-      tc_fence_after();
       const int row0 = c.tm * TILE_M + static_cast<int>(rank) * BM + q * 32;
       const int R = row0 / 32;  // 32-row block index
       const int rows_valid = min(32, G.M - row0);
@@ -762,7 +760,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
           }
         }
       };
+      // What needs no accumulator is requested before waiting for it: the
+      // polynomial's first A block, and the output scale (iteration 0 reads
+      // its matrix's 1/||H||_F from global memory).
       if (mode == MODE_POLY && ch0 < nch) load_aux(c.tn * BN + ch0 * 32);
+      float sc = G.scale;
+      if (mode != MODE_POLY && G.minv_pow) {
+        const float iv = G.minv[c.mat];
+        sc *= G.minv_pow == 2 ? iv * iv : iv;
+      }
+      if (!wait_bounded_warp(TFULL_BAR(acc), acc_phase, err, DEV_TIMEOUT_EPI, tmo)) break;
+      tc_fence_after();
       for (int ch = ch0; ch < nch; ch += 2) {
         const int col0 = c.tn * BN + ch * 32;
         const int C = c.tn * 8 + ch;
@@ -795,11 +803,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
           }
           __syncwarp();  // slot free for the output block
         } else {
-          float sc = G.scale;
-          if (G.minv_pow) {
-            const float iv = G.minv[c.mat];
-            sc *= G.minv_pow == 2 ? iv * iv : iv;
-          }
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] *= sc;
         }

@@ -228,6 +228,34 @@ def test_graph_and_direct_launch_bitwise(meq):
         assert np.array_equal(x, y)
 
 
+def test_profiled_steps_bitwise_and_phase_times(meq):
+    """Per-phase profiling runs the same kernels (a graph with event-record
+    nodes between the phases, or direct launches without use_graph): the
+    parameters match an unprofiled state bit for bit, and every phase that
+    has work reports a positive time."""
+    wl = W.custom_workload([(192, 320), (320, 192), (256, 256)], pattern="both", seed=9)
+    shapes = [(r, c) for _, r, c in wl.shapes]
+    out = {}
+    for name, graph, prof in (("plain", 1, False), ("graph", 1, True), ("eager", 0, True)):
+        opt = meq.MeqMuon(shapes, use_graph=graph)
+        if prof:
+            opt.set_profiling(True)
+        params = _to_dev(W.initial_weights(wl))
+        for t in range(3):
+            opt.step(params, _to_dev(W.gradients(wl, t)), LR, MU, WD, EPS)
+        opt.sync()
+        out[name] = [p.cpu().numpy() for p in params]
+        if prof:
+            ph, n = opt.read_profile()
+            assert n == 3, (name, n)
+            for k in ("momentum", "ns_gemm", "stats", "apply"):
+                assert ph[k] > 0, (name, ph)
+        opt.close()
+    for name in ("graph", "eager"):
+        for a, b in zip(out["plain"], out[name]):
+            assert np.array_equal(a, b), name
+
+
 def test_scale_invariance_bitwise(meq):
     """From B = 0, gradients scaled by 2^6 give the same update bit for bit
     (Frobenius pre-normalisation of Eq. (5) and scale-free CVs, Section 3.1)."""
