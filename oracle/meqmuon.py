@@ -28,8 +28,7 @@ Equation numbers are the paper's:
   Eq. (14) parameter update with decoupled decay     (Section 3.2)
   Algorithm 1 (MeqMuon), hidden-weight branch        (Section 3.2)
 
-Readings of points the paper leaves open (each one is listed with its
-justification in the design notes of the repository):
+Readings of points the paper leaves open, each with the reason stated:
   * Zero input to NS: the paper defines the iteration for a nonzero input
     only (Section 2); a zero momentum matrix gives U = 0.
   * A row / column RMS that does not exceed delta counts as zero
