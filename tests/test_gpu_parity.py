@@ -81,6 +81,22 @@ def test_ragged_shapes_two_steps(meq, shapes, pair):
 
 
 @pytest.mark.parametrize("pair", [1, 0], ids=["cta_pair", "single_cta"])
+def test_more_shape_groups_than_one_launch_holds(meq, pair):
+    """Ten shape groups (ten distinct oriented shapes): each product of Eq. (5)
+    takes two launches (eight groups, then two), two steps, staged against
+    the oracle."""
+    shapes = [(64, 96), (96, 64), (128, 128), (100, 200), (200, 100), (33, 65), (65, 33), (256, 80), (80, 256),
+              (48, 48)]
+    wl = W.custom_workload(shapes, pattern="both", base_sigma=0.01, seed=37)
+    opt = meq.MeqMuon(shapes, ns_cta_pair=pair)
+    assert opt.ns_gemm_launches_per_step == 2 * 3 * 5
+    opt.close()
+    rep = []
+    run_staged(meq, wl, 2, report=rep, ns_cta_pair=pair)
+    assert len(rep) == 2 * len(shapes) and all(r["update"] <= PT.UPDATE_TOL for r in rep)
+
+
+@pytest.mark.parametrize("pair", [1, 0], ids=["cta_pair", "single_cta"])
 def test_separate_x0_cast(meq, pair):
     """X_0 normalised and cast by its own pass (ns_x0_fused = 0: momentum +
     norm kernel, then the cast kernel) instead of inside the first NS
