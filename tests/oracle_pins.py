@@ -310,6 +310,36 @@ def check_equilibration_invariants(O):
     assert i4["direction"] != i1["direction"] and np.abs(U1 - U4.T).max() < 1e-11
 
 
+def check_rms_threshold_scale_zero(O):
+    """Reading of Eq. (9) (the paper rescales only nonzero rows / columns and
+    sets delta for Eq. (8)): a row or column whose RMS does not exceed delta
+    gets scale 0, in N_r, N_c, both stages of Eq. (12) and Eq. (13), while
+    one just above delta is rescaled to unit RMS like any other."""
+    rng = np.random.default_rng(14)
+    X = rng.standard_normal((6, 10))
+    X[2] = 5e-8 * np.sign(rng.standard_normal(10))      # RMS 5e-8 <= delta
+    X[3] = 3e-7 * np.sign(rng.standard_normal(10))      # RMS 3e-7 > delta
+    Nr = O.row_normalize(X)
+    assert np.all(Nr[2] == 0.0)
+    assert abs(math.sqrt((Nr[3] ** 2).mean()) - 1.0) < 1e-12 and abs(Nr[3, 0] - X[3, 0] / 3e-7) < 1e-6
+    Nc = O.col_normalize(X.T)
+    assert np.all(Nc[:, 2] == 0.0) and abs(math.sqrt((Nc[:, 3] ** 2).mean()) - 1.0) < 1e-12
+    # Eq. (12): the small row is dropped by N_r, so it is zero after N_c too;
+    # a column that is tiny in every row is dropped by the second stage
+    B = rng.standard_normal((7, 5))
+    B[4] = 2e-8
+    B[:, 1] = 1e-12
+    T = O.two_sided_normalize(B)
+    assert np.all(T[4] == 0.0)
+    Rn = O.row_normalize(B)
+    c1 = math.sqrt((Rn[:, 1] ** 2).mean())
+    assert 0.0 < c1 <= O.DELTA and np.all(T[:, 1] == 0.0)
+    # Eq. (13): a vector with RMS <= delta is not rescaled
+    assert np.all(O.vector_normalize(np.full(9, 4e-8)) == 0.0)
+    w = O.vector_normalize(np.full(9, -2e-7))
+    assert np.allclose(w, -1.0, atol=1e-12)
+
+
 def check_orthogonality_constraint(O):
     """Section 3.1: exact Orth of a tall full-rank matrix has Y^T Y = I, so
     gamma_c = 0 and row is chosen; a wide one has gamma_r = 0 and picks column."""
@@ -516,7 +546,7 @@ def check_constants(O):
 ALL_CHECKS = [
     check_constants, check_ns_known_svd, check_ns_band, check_ns_hadamard, check_ns_diag_4x3,
     check_ns_zero_rows_cols, check_ns_exact_integer, check_row_col_rms_rank_one,
-    check_cv_hand_values, check_selection_rule, check_equilibration_invariants,
+    check_cv_hand_values, check_selection_rule, check_equilibration_invariants, check_rms_threshold_scale_zero,
     check_orthogonality_constraint, check_two_sided_and_vector, check_momentum_closed_form,
     check_apply_closed_form, check_hidden_step_composition, check_param_step_branches,
     check_moonlight_update, check_moonlight_step, check_ns_cv_trajectory,

@@ -90,3 +90,47 @@ def test_ragged_mixed_kinds(meq):
     kinds = [O.REMAINING_2D, O.VECTOR, O.VECTOR, O.HIDDEN, O.REMAINING_2D, O.HIDDEN, O.VECTOR]
     wl = W.custom_workload(shapes, pattern="both", seed=31, kinds=kinds)
     run_kinds(meq, wl, 2)
+
+
+def test_rows_columns_and_vectors_at_the_rms_threshold(meq):
+    """The reading of Eq. (9) for rows / columns whose RMS does not exceed
+    delta (scale 0, no update from them), on the branches without
+    Newton-Schulz, where the momentum's rows are the gradient's: a remaining
+    2D parameter with a row at RMS 5e-8 and one at 3e-7 (rescaled to unit
+    RMS), a column that is tiny in every row (dropped by the second stage of
+    Eq. (12)), and vectors at RMS 4e-8 and 2e-7 (Eq. (13)). One step from
+    B = 0, parameters and statistics against the oracle."""
+    import torch
+
+    rng = np.random.default_rng(23)
+    G = rng.standard_normal((96, 40)) * 0.01
+    G[7] = 5e-8 * np.sign(rng.standard_normal(40))
+    G[8] = 3e-7 * np.sign(rng.standard_normal(40))
+    G[:, 11] = 1e-12
+    G[8, 11] = 0.0   # else row 8's rescaling (about 3e6) would lift column 11 above delta
+    gv1 = np.full((1, 64), 4e-8)
+    gv2 = np.full((1, 64), -2e-7)
+    Gs = [G.astype(np.float32), gv1.astype(np.float32), gv2.astype(np.float32)]
+    kinds = [O.REMAINING_2D, O.VECTOR, O.VECTOR]
+    shapes = [g.shape for g in Gs]
+    W0 = [rng.standard_normal(s).astype(np.float32) * 0.02 for s in shapes]
+    opt = meq.MeqMuon(shapes, kinds=kinds)
+    params = [torch.from_numpy(w.copy()).cuda() for w in W0]
+    opt.step(params, [torch.from_numpy(g).cuda() for g in Gs], LR, MU, WD, EPS)
+    opt.sync()
+    for i, k in enumerate(kinds):
+        W1 = params[i].cpu().numpy()
+        Wn, _, Ut = O.param_step(k, W0[i].astype(np.float64), Gs[i].astype(np.float64), np.zeros(shapes[i]), LR, MU,
+                                 WD, eps=EPS)
+        assert PT.max_rel(W1, Wn, floor_frac=1.0) <= PT.PARAM_TOL, i
+        assert PT.rel_frob(opt.read_update(i), Ut) <= PT.READBACK_TOL, i
+    Ut0 = opt.read_update(0)
+    assert np.all(Ut0[7] == 0.0) and np.all(Ut0[:, 11] == 0.0)
+    assert np.all(np.isfinite(Ut0[8])) and np.sqrt((Ut0[8] ** 2).mean()) > 0.1   # rescaled by about 1 / 3e-7
+    assert np.all(opt.read_update(1) == 0.0)
+    assert np.allclose(opt.read_update(2), -1.0, atol=1e-5)
+    # decay only where nothing was rescaled
+    d = (1 - LR * WD)
+    assert np.array_equal(params[1].cpu().numpy(), (d * W0[1]).astype(np.float32)) or \
+        PT.max_rel(params[1].cpu().numpy(), d * W0[1].astype(np.float64), floor_frac=1.0) <= PT.PARAM_TOL
+    opt.close()

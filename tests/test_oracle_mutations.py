@@ -91,6 +91,9 @@ MUTATIONS = {
     "cv_keeps_zeros": ("coefficient_of_variation", _cv_keep_zeros),
     "cv_mean_over_all": ("coefficient_of_variation", _cv_mean_over_all),
     "select_flipped": ("select_direction", lambda gr, gc, tie_atol=1e-6: 0 if gr < gc else 1),
+    "inverse_rms_no_threshold": ("_inverse_rms", lambda v, delta=1e-7: np.where(np.asarray(v, np.float64) > 0,
+                                                                          1.0 / np.maximum(np.asarray(v, np.float64),
+                                                                                           1e-300), 0.0)),
     "row_norm_multiplies": ("row_normalize", lambda X, delta=1e-7: np.asarray(X) * np.sqrt((np.asarray(X) ** 2).mean(1))[:, None]),
     "col_norm_uses_l2": ("col_normalize", lambda X, delta=1e-7: np.asarray(X) / np.maximum(np.linalg.norm(X, axis=0), 1e-300)[None, :]),
     "apply_no_decay": ("apply_update", lambda W, V, lr, wd, rho=0.2: np.asarray(W) - rho * lr * np.asarray(V)),
