@@ -20,7 +20,7 @@
 // X is stored scaled by a power of two alpha so its entries stay in the
 // normal range of fp16; the epilogues undo the scale in fp32.
 //
-// Roles (320 threads, one CTA per SM):
+// Roles (352 threads, one CTA per SM):
 //   warp 0 : TMA producer (one thread), shared-memory ring of 4 stages
 //            (single CTA) or 6 (CTA pair)
 //   warp 1 : TMEM allocator and tcgen05.mma issuer (one thread; with CTA
