@@ -203,9 +203,11 @@ meq_status meq_read_ns_output(meq_state* st, int i, float* dst);
  * U diag(c^-1) (Eqs. (9), (11); rows or columns with RMS <= eps scaled by 0),
  * or sqrt(max(m, n)) U under MEQ_RULE_MUON (Eq. (6)); remaining 2D
  * parameter: N_c(N_r(B_t)) (Eq. (12)); vector: B_t / RMS(B_t) (Eq. (13)).
- * Computed by a kernel from the operands and scale factors of the update
- * kernel; a host dst goes through a temporary device buffer of the same size
- * (MEQ_ERR_OOM if that allocation fails). Synchronises the state's stream. */
+ * Computed by a kernel on the state's device (whichever device is current;
+ * the current device is restored) from the operands and scale factors of
+ * the update kernel; a host dst goes through a temporary device buffer of the
+ * same size (MEQ_ERR_OOM if that allocation fails). Synchronises the state's
+ * stream. */
 meq_status meq_read_update(meq_state* st, int i, float* dst);
 /* Last step's statistics of entry i. Hidden weight: r (rows floats), c (cols
  * floats) of Eq. (7) for U, gamma_r, gamma_c of Eq. (8) and the direction of

@@ -1069,8 +1069,19 @@ meq_status meq_read_update(meq_state* st, int i, float* dst) {
   if (!dst) return fail(st, MEQ_ERR_INVALID_ARG, "dst is NULL");
   const MatInfo& M = st->mats[i];
   const size_t bytes = static_cast<size_t>(M.m * M.n) * sizeof(float);
+  // the kernel runs (and any temporary lives) on the state's device, whichever is current
+  int prev_dev = st->device;
+  cudaError_t e = cudaGetDevice(&prev_dev);
+  if (e == cudaSuccess && prev_dev != st->device) e = cudaSetDevice(st->device);
+  if (e != cudaSuccess) return cuda_fail(st, e, "selecting the state's device");
+  struct Restore {
+    int dev, cur;
+    ~Restore() {
+      if (dev != cur) cudaSetDevice(dev);
+    }
+  } restore{prev_dev, st->device};
   cudaPointerAttributes pa{};
-  cudaError_t e = cudaPointerGetAttributes(&pa, dst);
+  e = cudaPointerGetAttributes(&pa, dst);
   if (e != cudaSuccess) return cuda_fail(st, e, "cudaPointerGetAttributes");
   const bool on_device = (pa.type == cudaMemoryTypeDevice || pa.type == cudaMemoryTypeManaged) && pa.device == st->device;
   float* out = dst;
