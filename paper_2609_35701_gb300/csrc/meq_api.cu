@@ -486,6 +486,11 @@ bool build_gemm_plan(meq_state* st, std::string* why) {
           Q.tiles_m = (int32_t)((Q.M + tile_m - 1) / tile_m);
           Q.tiles_n = (int32_t)((Q.N + 255) / 256);
           Q.tiles_per_mat = Q.sym ? sym_tiles(Q.tiles_m, Q.tiles_n, tile_m) : Q.tiles_m * Q.tiles_n;
+          // Dense products walk bands of tile rows column by column; a band's
+          // row panels of P (band * tile_m * K 16-bit values) stay within 32 MB,
+          // about a quarter of L2, so every P panel is read from DRAM once.
+          Q.band = static_cast<int32_t>(
+              std::max<int64_t>(1, std::min<int64_t>(Q.tiles_m, (int64_t(32) << 20) / (int64_t(tile_m) * Q.K * 2))));
           Q.tile_begin = tiles;
           const int64_t t = int64_t(Q.tiles_per_mat) * Q.count;
           if (tiles + t > (int64_t(1) << 30)) { *why = "too many GEMM tiles in one launch"; return false; }

@@ -88,6 +88,7 @@ struct GemmGroup {
   int32_t count;          // matrices in the group
   int32_t tiles_m, tiles_n;
   int32_t tiles_per_mat;  // tiles_m * tiles_n, or the upper-triangle count when sym
+  int32_t band;           // dense outputs: tile rows per band of the tile order
   int32_t tile_begin;     // first tile of this group in the launch
   int32_t sym;            // 1: symmetric s x s output (upper-triangle tiles, mirrored stores)
   int32_t trans;          // XLAST: 1 when the weight is the transpose of the NS layout

@@ -299,20 +299,19 @@ __device__ __forceinline__ void tmem_ld_32cols(uint32_t taddr, float* v) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-constexpr int kBand = 8;  // tile rows per band of the dense products' tile order
-
 struct TileCoord {
   int g, mat, tm, tn;
 };
 
 // Tiles of a group are numbered matrix by matrix (walked backwards when
 // p.reverse is set, so a launch starts on the matrices its predecessor wrote
-// last, which are still in L2). Dense outputs (X' = P X) with more than
-// kBand tile rows run in bands of kBand tile rows, each band column by column: the tiles in flight at once
-// (one per CTA pair) then share a few row panels of P and column panels of
-// X, where a row-by-row walk re-read every column panel of a wide X once per
-// tile row (measured at 4096 x 11008: 4.5 times the launch's algorithmic
-// bytes from DRAM). Symmetric outputs (Gram, polynomial) run tn-major over
+// last, which are still in L2). Dense outputs (X' = P X) run in bands of
+// G.band tile rows, each band column by column (the host sizes a band so
+// its row panels of P fit in a quarter of L2): the tiles in flight at once
+// (one per CTA pair) then share one or a few column panels of X and the
+// band's panels of P, where a row-by-row walk re-read every column panel of
+// a wide X once per tile row (measured at 4096 x 11008: 4.5 times the
+// launch's algorithmic bytes from DRAM). Symmetric outputs (Gram, polynomial) run tn-major over
 // the tiles with tm * TILE_M < (tn + 1) * 256, i.e. those holding a 32 x 32
 // block on or above the diagonal.
 __device__ __forceinline__ int find_segment(const GemmParams& p, int t) {
@@ -335,14 +334,11 @@ __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
   TileCoord c;
   c.g = g;
   c.mat = mat;
-  if (!G.sym && G.tiles_m <= kBand) {
-    c.tm = r / G.tiles_n;
-    c.tn = r - c.tm * G.tiles_n;
-  } else if (!G.sym) {
-    const int band = r / (kBand * G.tiles_n);
-    const int in = r - band * kBand * G.tiles_n;
-    const int rows = min(kBand, G.tiles_m - band * kBand);
-    c.tm = band * kBand + in % rows;
+  if (!G.sym) {
+    const int band = r / (G.band * G.tiles_n);
+    const int in = r - band * G.band * G.tiles_n;
+    const int rows = min(G.band, G.tiles_m - band * G.band);
+    c.tm = band * G.band + in % rows;
     c.tn = in / rows;
   } else {
     int tn = 0;
@@ -535,7 +531,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot_ptr;
   pdl_allow_dependents();
-  pdl_wait_predecessor();  // operands come from the previous kernel of the step
+  // The wait for the previous kernel of the step (griddepcontrol.wait, per
+  // thread) is taken by the roles that touch global memory, each before its
+  // first access: the producer, the epilogue warps and the scheduler (after
+  // it has published the unit's first tile). The MMA issuer works on shared
+  // memory and TMEM only.
 
   // ------------------------------------------------------------------ tile queue
   // Each unit (CTA pair) starts on tile `unit`; further tiles are handed out
@@ -571,6 +571,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
   if (warp == 0) {
     if (lane == 0) {
       // ---------------------------------------------------------------- TMA producer
+      pdl_wait_predecessor();  // operands come from the previous kernel of the step
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued_mask = 0, issued_parity = 0;  // bit s: stage s was filled / parity of its last fill
@@ -704,6 +705,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
     __syncwarp();
   } else if (warp < 2 + NUM_EPI_WARPS) {
     // ------------------------------------------------------------------ epilogue
+    pdl_wait_predecessor();  // reads A (polynomial) and overwrites buffers of earlier kernels
     // Warp ew (0..7) owns TMEM lanes 32*q .. +31 (q = warp % 4), i.e. rows
     // 32q .. 32q+31 of the tile, chunks ch with ch % 2 == half, and two 2 KB
     // shared-memory slots: `slot` takes the polynomial's A block (prefetched
@@ -920,6 +922,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) ns_gemm_kernel(const __grid_co
         }
         if (!sched_put(n, e)) break;
         if (t >= p.total_tiles) break;
+        // Entry 0, the unit's own tile, depends only on the launch parameters
+        // and is published while the previous kernel may still run; the
+        // queue counter, which that kernel's last unit resets, only after it.
+        if (n == 0) pdl_wait_predecessor();
         fetched = atomicAdd(p.sched, 1);  // read when the producer has taken this entry
       }
     }
