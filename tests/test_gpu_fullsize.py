@@ -37,15 +37,15 @@ def _release():
     torch.cuda.empty_cache()
 
 
-def _run(meq, name, steps, check_steps, check_names, property_names=()):
+def _run(meq, name, steps, check_steps, check_names, property_names=(), ns_out=None, **opts):
     import torch
 
-    wl = W.get_workload(name)
+    wl = W.get_workload(name) if isinstance(name, str) else name
     names = [n for n, _, _ in wl.shapes]
     staged = [names.index(n) for n in check_names]
     pick = staged + [names.index(n) for n in property_names]
     shapes = [(r, c) for _, r, c in wl.shapes]
-    opt = meq.MeqMuon(shapes)
+    opt = meq.MeqMuon(shapes, **opts)
     params = W.initial_weights(wl, device="cuda")
     scales = W.scale_table(wl, device="cuda")
     B_prev = {i: np.zeros(shapes[i]) for i in pick}
@@ -64,6 +64,8 @@ def _run(meq, name, steps, check_steps, check_names, property_names=()):
         if checking:
             for i in pick:
                 U = opt.read_ns_output(i)
+                if ns_out is not None:
+                    ns_out[(t, i)] = U
                 st = opt.read_stats(i)
                 W1 = params[i].cpu().numpy()
                 B = opt.read_momentum(i)
@@ -134,3 +136,22 @@ def test_llama7b_full_size_sampled(meq):
     staged = [r for r in rep if "update" in r]
     assert len(rep) == 20 and len(staged) == 4
     assert max(r["update"] for r in staged) <= PT.UPDATE_TOL
+
+
+def test_dense_product_bands_with_a_ragged_band(meq):
+    """At s = 4352 the update product X' = P X walks bands of tile rows column
+    by column, a band holding as many tile rows as keep its row panels of P
+    within 32 MB: bands of 15 and 2 tile rows of 256 (the pair variant), of
+    30 and 4 tile rows of 128 (the single-CTA variant). A wide and a tall
+    matrix (one oriented group, 18 ragged tile columns) against the fp64
+    oracle at step 1, and the single-CTA variant's NS output against the
+    pair variant's."""
+    wl = W.custom_workload([(4352, 4400), (4400, 4352)], pattern="both", seed=31)
+    names = [n for n, _, _ in wl.shapes]
+    outs = [{}, {}]
+    rep = _run(meq, wl, 2, {1}, names, ns_out=outs[0])
+    _report("bands", rep)
+    assert len(rep) == 2 and max(r["update"] for r in rep) <= PT.UPDATE_TOL
+    _run(meq, wl, 2, {1}, (), property_names=names, ns_out=outs[1], ns_cta_pair=0)
+    for key in outs[0]:
+        assert PT.rel_frob(outs[0][key], outs[1][key]) < 2e-3, key
