@@ -39,6 +39,23 @@ __device__ __forceinline__ int find_mat(const MatInfo* mats, int nmat, int64_t k
   return lo;
 }
 
+// Row i and column j of flat element e of a matrix with n columns. Every
+// model weight has fewer than 2^32 elements, where a 32-bit division is
+// several times cheaper than a 64-bit one (measured: about 0.5% of the
+// Llama-130M and 350M steps); small32 is uniform over a block, so the
+// branch does not diverge.
+__device__ __forceinline__ void row_col(int64_t e, int64_t n, bool small32, int64_t& i, int64_t& j) {
+  if (small32) {
+    const uint32_t eu = static_cast<uint32_t>(e), nu = static_cast<uint32_t>(n);
+    const uint32_t iu = eu / nu;
+    i = iu;
+    j = eu - iu * nu;
+  } else {
+    i = e / n;
+    j = e - i * n;
+  }
+}
+
 __device__ __forceinline__ float block_sum_f32(float v, float* sh) {
   const unsigned FULL = 0xffffffffu;
 #pragma unroll
@@ -176,6 +193,7 @@ __global__ void __launch_bounds__(kThreads, 8) momentum_x0_kernel(const MatInfo*
   if (!M.trans) {
     const int64_t e0 = lt * kChunk;
     const int64_t e1 = min(e0 + kChunk, M.m * M.n);
+    const bool small32 = M.m * M.n <= static_cast<int64_t>(UINT32_MAX);
     for (int64_t e = e0 + 4 * threadIdx.x; e < e1; e += 4 * kThreads) {
       float h[4];
       if (e + 3 < e1) {
@@ -201,7 +219,8 @@ __global__ void __launch_bounds__(kThreads, 8) momentum_x0_kernel(const MatInfo*
         }
       }
       ss += h[0] * h[0] + h[1] * h[1] + h[2] * h[2] + h[3] * h[3];
-      int64_t i = e / M.n, j = e - i * M.n;
+      int64_t i, j;
+      row_col(e, M.n, small32, i, j);
       if ((M.n & 3) == 0) {
         // four columns of one row (m n is then a multiple of 4, so e + 3 < e1)
         *reinterpret_cast<uint2*>(X + i * Gi.lp + j) = pack4_bf16(h[0], h[1], h[2], h[3]);
@@ -709,8 +728,10 @@ __global__ void __launch_bounds__(kThreads, 8) apply_kernel(const MatInfo* __res
   float* W = params[mi];
   if ((M.n & 3) == 0) {
     // four columns of one row per thread (m n is a multiple of 4, so e + 3 < e1)
+    const bool small32 = numel <= static_cast<int64_t>(UINT32_MAX);
     for (int64_t e = e0 + 4 * threadIdx.x; e < e1; e += 4 * kThreads) {
-      const int64_t i = e / M.n, j = e - i * M.n;
+      int64_t i, j;
+      row_col(e, M.n, small32, i, j);
       float4 w = *reinterpret_cast<const float4*>(W + e);
       float u[4];
       if (hidden) {
