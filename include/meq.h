@@ -66,7 +66,10 @@ typedef struct {
   float tie_atol;         /* Eq. (11) chooses row when gamma_r >= gamma_c - tie_atol; 1e-6 */
   int use_graph;          /* 1: the step's kernels are replayed from a CUDA graph (default) */
   int64_t workspace_limit_bytes; /* 0 = no limit; else init fails with MEQ_ERR_OOM above it */
-  float wait_timeout_ms;  /* bound of every device-side spin wait; default 4000 */
+  float wait_timeout_ms;  /* bound of every device-side spin wait; default 4000. An NS kernel's
+                             MMA thread starts waiting for its first operands while the kernel
+                             before it may still run, so the bound must exceed the longest kernel
+                             of a step (about 20 ms per NS product at Llama-7B-class sizes) */
   int ns_cta_pair;        /* 1 (default): NS GEMMs run on CTA pairs (tcgen05 cta_group::2,
                              256 x 256 tiles on two SMs); 0: one CTA per 128 x 256 tile */
   int ns_x0_fused;        /* 1 (default): the momentum pass also writes X_0, unnormalised in
